@@ -1,0 +1,247 @@
+"""Plain CPU oracle of the TReVS two-stage visual-token pruning path (fp64).
+
+TEST INFRASTRUCTURE ONLY. Nothing on the product path imports this module: only
+the tests, the smoke check and the CPU-baseline leg of the benchmark do. It
+shares no code with the CUDA library; the two meet only in the seeded input
+bytes produced by `workloads.synth`.
+
+Every function restates one step of the method in the paper's order and
+notation, with library primitives (matmul, exp, stable sort) as its only
+building blocks and no blocking, fusion or reordering. Inputs arrive as
+bfloat16 bit patterns (uint16) or float32 and are widened exactly to float64.
+
+Readings where the paper is silent (each listed with its reason in the design doc):
+  * A zero-norm vector has cosine 0 with everything (Eq. 4 divides by the norm).
+  * Med is the lower median: the ascending element of rank floor((N-1)/2) (Eq. 6).
+  * epsilon of Eq. 6 defaults to 1e-6.
+  * Textual-ratio selection (Sec. 3.1): K_t = floor(r*K1 + 0.5) textual tokens,
+    K_v = K1 - K_t saliency tokens; the saliency top-K_v is taken first, the
+    textual top-K_t over the remaining tokens; both rank the raw scores.
+  * TopK ties go to the lower token (or head) index; kept sets are returned in
+    ascending index order, which preserves the original token order.
+  * The text-to-vision softmax of Sec. 4.2 spans the K1 visual keys of each text
+    row (each row sums to 1); no causal mask (every visual token precedes the
+    text); scale 1/sqrt(d_h); query head h reads key head floor(h*Hkv/Hq).
+  * Var_i in Eq. 8 is the population variance (divide by K1), two-pass.
+  * H* holds n_keep_heads heads (the paper's default is half of the heads).
+
+Parity pins: every function here is pinned by tests/test_oracle_pins.py against
+closed forms, hand-derived worked examples (tests/golden/), brute force on tiny
+inputs and invariants; none is "parity unpinned".
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+# ---------------------------------------------------------------- encodings
+
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """bfloat16 bit patterns -> float64 (exact: bf16 is the top half of a float32)."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+# ---------------------------------------------------------------- stage 1 (Sec. 4.1)
+
+
+def rectified_cosine(Z: np.ndarray, T: np.ndarray) -> np.ndarray:
+    """Eq. 4: m[j, i] = max(tbar_j . zbar_i, 0) with zbar, tbar the L2-normalised rows.
+
+    Z is [N, d'] visual features, T is [M, d'] text embeddings; returns [M, N].
+    A zero-norm row has cosine 0 with every other row.
+    """
+    Z = np.asarray(Z, dtype=np.float64)
+    T = np.asarray(T, dtype=np.float64)
+    nz = np.sqrt(np.sum(Z * Z, axis=1))
+    nt = np.sqrt(np.sum(T * T, axis=1))
+    zbar = np.divide(Z, nz[:, None], out=np.zeros_like(Z), where=nz[:, None] > 0)
+    tbar = np.divide(T, nt[:, None], out=np.zeros_like(T), where=nt[:, None] > 0)
+    cos = tbar @ zbar.T
+    return np.maximum(cos, 0.0)
+
+
+def textual_relevance(Z: np.ndarray, T: np.ndarray) -> np.ndarray:
+    """Eq. 5: s^t_i = sqrt( (1/M) * sum_j m[j, i]^2 ), the RMS over the M text tokens."""
+    m = rectified_cosine(Z, T)
+    M = m.shape[0]
+    if M == 0:
+        raise ValueError("textual relevance needs at least one text token")
+    return np.sqrt(np.sum(m * m, axis=0) / M)
+
+
+def lower_median(x: np.ndarray) -> float:
+    """Med of Eq. 6: the ascending element of rank floor((N-1)/2)."""
+    x = np.sort(np.asarray(x, dtype=np.float64), kind="stable")
+    return float(x[(len(x) - 1) // 2])
+
+
+def mad(x: np.ndarray) -> float:
+    """MAD of Eq. 6: the median of |x_i - Med(x)|."""
+    x = np.asarray(x, dtype=np.float64)
+    return lower_median(np.abs(x - lower_median(x)))
+
+
+def robust_normalise(s: np.ndarray, tau: float, eps: float) -> np.ndarray:
+    """Eq. 6: shat_i = [ (s_i - Med(s)) / (MAD(s) + eps) ]_+ / tau."""
+    s = np.asarray(s, dtype=np.float64)
+    z = (s - lower_median(s)) / (mad(s) + eps)
+    return np.maximum(z, 0.0) / tau
+
+
+def fused_score(sv_hat: np.ndarray, st_hat: np.ndarray, lam: float) -> np.ndarray:
+    """Eq. 7: s_i = max(shat^v_i, shat^t_i) + lambda * sqrt(shat^v_i * shat^t_i)."""
+    sv_hat = np.asarray(sv_hat, dtype=np.float64)
+    st_hat = np.asarray(st_hat, dtype=np.float64)
+    return np.maximum(sv_hat, st_hat) + lam * np.sqrt(sv_hat * st_hat)
+
+
+def top_k(score: np.ndarray, k: int, allowed: np.ndarray | None = None) -> np.ndarray:
+    """TopK of Eq. 7 / Eq. 9: the k best entries by (score descending, index ascending).
+
+    `allowed` (bool mask) restricts the candidates. Returns indices in ascending order.
+    """
+    score = np.asarray(score, dtype=np.float64)
+    idx = np.arange(len(score))
+    if allowed is not None:
+        idx = idx[np.asarray(allowed, dtype=bool)]
+    if k < 0 or k > len(idx):
+        raise ValueError(f"top_k: k={k} outside [0, {len(idx)}]")
+    order = np.lexsort((idx, -score[idx]))     # primary: -score ascending; then index
+    return np.sort(idx[order[:k]])
+
+
+def textual_count(k1: int, ratio: float) -> int:
+    """K_t = floor(r * K1 + 0.5): the textual share of the keep budget (Sec. 3.1)."""
+    return int(math.floor(float(np.float32(ratio)) * k1 + 0.5))
+
+
+def select_ratio(s_v: np.ndarray, s_t: np.ndarray, k1: int, ratio: float) -> np.ndarray:
+    """Sec. 3.1 budget split: saliency top-K_v, then textual top-K_t over the rest."""
+    k_t = textual_count(k1, ratio)
+    k_v = k1 - k_t
+    S_v = top_k(s_v, k_v)
+    rest = np.ones(len(s_v), dtype=bool)
+    rest[S_v] = False
+    S_t = top_k(s_t, k_t, allowed=rest)
+    return np.sort(np.concatenate([S_v, S_t]))
+
+
+def select_fused(s_v, s_t, k1, tau_v=1.4, tau_t=1.0, lam=1.0, eps=1e-6):
+    """Eq. 6-7 pivot selection S_r = TopK(s, K_r) with K_r = K1 (no diversity tokens)."""
+    s = fused_score(robust_normalise(s_v, tau_v, eps), robust_normalise(s_t, tau_t, eps), lam)
+    return top_k(s, k1), s
+
+
+def gather_rows(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
+    """Sec. 4.1: the kept rows, in ascending index order, are passed to the LLM."""
+    return np.asarray(X)[np.asarray(idx, dtype=np.int64)]
+
+
+# ---------------------------------------------------------------- stage 2 (Sec. 4.2)
+
+
+def text_to_vision_attention(Q: np.ndarray, K: np.ndarray, scale: float | None = None):
+    """A^h_{T->V}[q, i] = softmax_i( Q[q, h] . K[i, g(h)] * scale ), g(h) = floor(h*Hkv/Hq).
+
+    Q is [L, Hq, dh] (text rows at layer l*), K is [K1, Hkv, dh] (visual keys).
+    Returns A as [Hq, L, K1]; every row is a distribution over the K1 visual keys.
+    """
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    L, Hq, dh = Q.shape
+    K1, Hkv, _ = K.shape
+    if scale is None:
+        scale = 1.0 / math.sqrt(dh)
+    A = np.empty((Hq, L, K1), dtype=np.float64)
+    for h in range(Hq):
+        g = (h * Hkv) // Hq
+        logits = (Q[:, h, :] @ K[:, g, :].T) * scale          # [L, K1]
+        e = np.exp(logits - logits.max(axis=1, keepdims=True))
+        A[h] = e / e.sum(axis=1, keepdims=True)
+    return A
+
+
+def head_variance(A: np.ndarray) -> np.ndarray:
+    """Eq. 8: u_h = (1/L) sum_q Var_i A^h[q, i] (population variance, two-pass)."""
+    A = np.asarray(A, dtype=np.float64)
+    K1 = A.shape[2]
+    mean = A.sum(axis=2, keepdims=True) / K1
+    var = ((A - mean) ** 2).sum(axis=2) / K1                 # [Hq, L]
+    return var.sum(axis=1) / A.shape[1]
+
+
+def select_heads(u: np.ndarray, n_keep: int) -> np.ndarray:
+    """H*: the n_keep heads of largest u_h (ties to the lower head), ascending."""
+    return top_k(u, n_keep)
+
+
+def token_scores(A: np.ndarray, heads: np.ndarray) -> np.ndarray:
+    """Eq. 9: p_i = max_q (1/|H*|) sum_{h in H*} A^h[q, i]."""
+    A = np.asarray(A, dtype=np.float64)
+    heads = np.asarray(heads, dtype=np.int64)
+    mean_over_heads = A[heads].sum(axis=0) / len(heads)      # [L, K1]
+    return mean_over_heads.max(axis=0)
+
+
+# ---------------------------------------------------------------- per-request drivers
+
+
+def pre_llm_request(Z_bits, T_bits, s_v, k1, ratio, mode="ratio", tau_v=1.4, tau_t=1.0,
+                    lam=1.0, eps=1e-6):
+    """Stage 1 for one request: s^t (Eq. 4-5), selection, gather of the kept rows."""
+    Z = bf16_bits_to_f64(Z_bits)
+    T = bf16_bits_to_f64(T_bits)
+    s_v = np.asarray(s_v, dtype=np.float64)
+    s_t = textual_relevance(Z, T)
+    out = {"s_t": s_t}
+    if mode == "ratio":
+        kept = select_ratio(s_v, s_t, k1, ratio)
+    elif mode == "fused":
+        kept, s = select_fused(s_v, s_t, k1, tau_v, tau_t, lam, eps)
+        out["s_fused"] = s
+    else:
+        raise ValueError(mode)
+    out["kept"] = kept
+    out["Z_out"] = gather_rows(np.asarray(Z_bits), kept)
+    return out
+
+
+def in_llm_request(Q_bits, K_bits, V_bits, hidden_bits, n_keep_heads, k2, scale=None):
+    """Stage 2 for one request: attention, Eq. 8 variance, H*, Eq. 9 scores, top-K2, compaction."""
+    Q = bf16_bits_to_f64(Q_bits)
+    K = bf16_bits_to_f64(K_bits)
+    A = text_to_vision_attention(Q, K, scale)
+    u = head_variance(A)
+    heads = select_heads(u, n_keep_heads)
+    p = token_scores(A, heads)
+    kept = top_k(p, k2)
+    return {
+        "u": u, "heads": heads, "p": p, "kept": kept,
+        "hidden_out": gather_rows(np.asarray(hidden_bits), kept),
+        "K_out": gather_rows(np.asarray(K_bits), kept),
+        "V_out": gather_rows(np.asarray(V_bits), kept),
+    }
+
+
+def run_workload(w, mode="ratio", stage1=True, stage2=True, requests=None, **params):
+    """Both stages over every request of a `workloads.synth.Workload` (or a subset)."""
+    n_off, m_off = w.offsets("n"), w.offsets("m")
+    k1_off, l_off = w.offsets("k1"), w.offsets("l")
+    out = []
+    for b in (range(w.B) if requests is None else requests):
+        r = w.reqs[b]
+        res = {}
+        if stage1:
+            res["pre"] = pre_llm_request(
+                w.Z[n_off[b]:n_off[b + 1]], w.T[m_off[b]:m_off[b + 1]],
+                w.s_v[n_off[b]:n_off[b + 1]], r.k1, r.ratio, mode, **params)
+        if stage2:
+            res["in"] = in_llm_request(
+                w.Q[l_off[b]:l_off[b + 1]], w.K[k1_off[b]:k1_off[b + 1]],
+                w.V[k1_off[b]:k1_off[b + 1]], w.hidden[k1_off[b]:k1_off[b + 1]],
+                w.n_keep_heads, r.k2)
+        out.append(res)
+    return out
