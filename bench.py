@@ -1,0 +1,419 @@
+#!/usr/bin/env python
+"""Throughput of the TReVS two-stage prune on GB300, one JSON line on stdout.
+
+A step is one trevs_prune_varlen call over the LLaVA-1.5-shaped batch of 32 requests
+(576 visual tokens each, d' = 4096, query lengths 16..64, stage-1 keep 64 at textual
+ratio 0.5, stage 2 at layer 2 with 32 heads x 128, top 8 heads, final keep 32): Eq. 4-5
+scores, the Sec. 3.1 split and gather, then attention statistics, Eq. 8-9 and compaction.
+
+  value      visual tokens scored and pruned per second, inputs resident in HBM, the step
+             replayed as a CUDA graph, 4 rotating input sets (0.93 GB > 129 MB L2);
+  e2e        the same metric through the public call with pinned HOST inputs: every step
+             copies its inputs host->device and reads the kept indices back;
+  roofline   the dominant kernel (stage-1 scoring + selection): algorithmic bytes per
+             launch / its CUDA-event duration, against the measured HBM copy bandwidth;
+  cpu_baseline  the fp64 oracle on the host cores (one process per core, bounded sample).
+
+--impl reference times the oracle itself as the reference arm. Under torchrun (N > 1)
+every rank prunes its own copy of the batch (replicas, weak scaling, no collective on
+the data path); rank 0 prints the max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import pathlib
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")          # one BLAS thread per oracle worker process
+
+ROOT = pathlib.Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+import numpy as np  # noqa: E402
+
+from workloads import synth  # noqa: E402
+
+METRIC = "visual tokens scored+pruned/s (2-stage prune)"
+UNIT = "visual tokens/s"
+WORKLOAD = dict(k1=64, ratio=0.5, k2=32)
+ROTATING_SETS = 4
+DOMINANT = "pre_score_kernel"
+
+
+def workload():
+    return synth.llava15_batch32(**WORKLOAD)
+
+
+def config_of(w):
+    return {"workload": f"llava15_576_b32_k1_{WORKLOAD['k1']}_r{WORKLOAD['ratio']}_k2_{WORKLOAD['k2']}",
+            "requests": w.B, "visual_tokens_per_request": 576, "d": w.d,
+            "query_tokens": f"{min(r.m for r in w.reqs)}..{max(r.m for r in w.reqs)}",
+            "K1": WORKLOAD["k1"], "textual_ratio": WORKLOAD["ratio"], "K2": WORKLOAD["k2"],
+            "heads": f"{w.hq}x{w.dh}, keep {w.n_keep_heads}", "select": "ratio",
+            "l2": f"{ROTATING_SETS} rotating input sets (> L2)", "replay": "CUDA graph per step"}
+
+
+def algorithmic_bytes(w):
+    """Stage 1: read Z, T, s_v; write Z_out and the kept indices. Stage 2: read Q, K; read
+    and write the kept rows of hidden, K and V; write the kept indices."""
+    sn = sum(r.n for r in w.reqs)
+    sm = sum(r.m for r in w.reqs)
+    sk1 = sum(r.k1 for r in w.reqs)
+    sl = sum(r.l for r in w.reqs)
+    sk2 = sum(r.k2 for r in w.reqs)
+    score = sn * w.d * 2 + sm * w.d * 2 + sn * 4 + sk1 * 4
+    stage1 = score + sk1 * w.d * 2
+    stage2 = (sl * w.hq * w.dh * 2 + sk1 * w.hkv * w.dh * 2
+              + 2 * sk2 * (w.d + 2 * w.hkv * w.dh) * 2 + sk2 * 4)
+    return {"score_kernel": score, "stage1": stage1, "stage2": stage2, "step": stage1 + stage2}
+
+
+def peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def committed_traffic():
+    """dram bytes per launch of the dominant kernel from the committed ncu summary, if the
+    kernel source is unchanged since the capture (else None)."""
+    import hashlib
+    f = ROOT / "profiles" / "traffic.txt"
+    src = ROOT / "paper_2609_37581_gb300" / "csrc" / "pre_llm.cu"
+    if not f.exists() or not src.exists():
+        return None
+    digest = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    for line in f.read_text().splitlines():
+        parts = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
+        if parts.get("kernel") == DOMINANT and parts.get("src_sha") == digest and "dram_bytes_per_launch" in parts:
+            return int(parts["dram_bytes_per_launch"])
+    return None
+
+
+# ------------------------------------------------------------------ oracle timing (host)
+
+
+def _oracle_job(args):
+    import oracle.trevs_oracle as O
+    b_list, reps = args
+    w = _ORACLE_W
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        O.run_workload(w, requests=b_list)
+    return time.perf_counter() - t0
+
+
+_ORACLE_W = None
+
+
+def time_oracle(w, budget_s=12.0, cores=None):
+    """Oracle throughput on the host cores (fork pool created before any CUDA call)."""
+    import multiprocessing as mp
+    global _ORACLE_W
+    _ORACLE_W = w
+    cores = cores or os.cpu_count() or 1
+    ctx = mp.get_context("fork")
+    tokens_per_req = [r.n for r in w.reqs]
+    with ctx.Pool(cores) as pool:
+        # calibration: one pass over all requests
+        t0 = time.perf_counter()
+        pool.map(_oracle_job, [([b], 1) for b in range(w.B)], chunksize=1)
+        per_pass = time.perf_counter() - t0
+        passes = min(50, max(1, int(budget_s / max(1e-3, per_pass))))
+        jobs = [([b], passes) for b in range(w.B)]
+        t0 = time.perf_counter()
+        pool.map(_oracle_job, jobs, chunksize=1)
+        wall = time.perf_counter() - t0
+    tokens = sum(tokens_per_req) * passes
+    return {"value": tokens / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{passes} pass(es) over all {w.B} requests, both stages, fp64, one process per core",
+            "seconds": round(wall, 3)}
+
+
+# ------------------------------------------------------------------ clocks
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.lines = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", self.gpu_id], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+
+def gpu_arm(args, rank, world, w, cpu_baseline):
+    import torch
+    from paper_2609_37581_gb300 import trevs as T
+    from workloads.device import build_batches, dev_bf16, dev_f32
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    T.load()
+    stream = torch.cuda.Stream()
+    params = T.default_params(T.SELECT_RATIO)
+    with torch.cuda.stream(stream):
+        base = {"Z": dev_bf16(w.Z), "T": dev_bf16(w.T), "s_v": dev_f32(w.s_v), "Q": dev_bf16(w.Q),
+                "K": dev_bf16(w.K), "V": dev_bf16(w.V), "hidden": dev_bf16(w.hidden)}
+        sets = [base] + [{k: v.clone() for k, v in base.items()} for _ in range(ROTATING_SETS - 1)]
+        batches = [build_batches(w, T.SELECT_RATIO, dev=s) for s in sets]
+        ws = T.workspace(max(T.trevs_prune_varlen_workspace_size(p, i) for p, i in batches))
+        calls = [T.PreparedCall(p, i, ws, params) for p, i in batches]
+        # the dominant kernel alone: stage-1 scoring + selection (no gather)
+        score_only = []
+        for p, _ in batches:
+            q = T.PreBatch(reqs=p.reqs, Z=p.Z, T=p.T, s_v=p.s_v, kept_idx=p.kept_idx, Z_out=None, s_t=p.s_t)
+            score_only.append((q, T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))))
+        for c in calls:                       # eager warm-up (sets the kernels' smem limits)
+            c(stream)
+        launches_per_step = T.last_launch_count()
+        T.trevs_pre_llm_varlen(score_only[0][0], score_only[0][1], params, stream)
+        torch.cuda.synchronize()
+        graphs = []
+        for c in calls:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                c(stream)
+            graphs.append(g)
+        sgraphs = []
+        for q, wsq in score_only:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                T.trevs_pre_llm_varlen(q, wsq, params, stream)
+            sgraphs.append(g)
+    torch.cuda.synchronize()
+
+    import torch.distributed as dist
+    distributed = world > 1
+
+    def barrier():
+        if distributed:
+            dist.barrier()
+
+    gpu_id = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[dev.index] \
+        if os.environ.get("CUDA_VISIBLE_DEVICES") else str(dev.index)
+    sampler = ClockSampler(gpu_id)
+    with sampler, torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            graphs[i % ROTATING_SETS].replay()
+        torch.cuda.synchronize()
+        barrier()
+        torch.cuda.synchronize()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for i in range(args.steps):
+            graphs[i % ROTATING_SETS].replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        elapsed_ms = ev0.elapsed_time(ev1)
+        # dominant kernel: CUDA events around each replay of its one-kernel graph
+        nk = max(20, min(args.steps, 2000))
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nk)]
+        for i in range(nk):
+            evs[i][0].record(stream)
+            sgraphs[i % ROTATING_SETS].replay()
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        kernel_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+    if distributed:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+
+    # end to end through the public call with host buffers
+    e2e = None
+    if rank == 0:
+        host = {k: v.cpu().pin_memory() for k, v in base.items()}
+        p0, i0 = batches[0]
+        kept_h = torch.empty(p0.kept_idx.numel(), dtype=torch.int32).pin_memory()
+        kept2_h = torch.empty(i0.kept_local.numel(), dtype=torch.int32).pin_memory()
+        h2d = sum(v.numel() * v.element_size() for v in host.values())
+        d2h = (kept_h.numel() + kept2_h.numel()) * 4
+        ne = max(5, min(args.steps, 100))
+        with torch.cuda.stream(stream):
+            for _ in range(2):
+                for k, v in host.items():
+                    sets[0][k].copy_(v, non_blocking=True)
+                calls[0](stream)
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(ne):
+                for k, v in host.items():
+                    sets[0][k].copy_(v, non_blocking=True)
+                calls[0](stream)
+                kept_h.copy_(p0.kept_idx, non_blocking=True)
+                kept2_h.copy_(i0.kept_local, non_blocking=True)
+            b.record(stream)
+            torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b) / ne
+        e2e = {"value": w.visual_tokens() / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4)}
+
+    if rank != 0:
+        return None
+    ms = elapsed_ms / args.steps
+    tokens_per_step = w.visual_tokens() * world
+    nbytes = algorithmic_bytes(w)
+    peak, src = peaks()
+    achieved = nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9
+    clk = sampler.summary()
+    return {
+        "metric": METRIC, "value": tokens_per_step / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+        "us_per_prune": round(ms * 1e3, 2), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded, LLaVA-1.5-shaped; no dataset)",
+        "config": config_of(w),
+        "roofline": {"bound": "hbm", "kernel": DOMINANT, "achieved": round(achieved, 1), "peak": peak,
+                     "peak_source": src, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": committed_traffic(), "algorithmic_bytes": nbytes["score_kernel"],
+                     "kernel_us": round(kernel_ms * 1e3, 2)},
+        "step_roofline": {"algorithmic_bytes": nbytes["step"],
+                          "achieved_gbs": round(nbytes["step"] / (ms * 1e-3) / 1e9, 1),
+                          "frac": round(nbytes["step"] / (ms * 1e-3) / 1e9 / peak, 4), "peak_source": src},
+        "cpu_baseline": cpu_baseline, "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "launches_per_step": launches_per_step,
+        "clocks": clk,
+    }
+
+
+# ------------------------------------------------------------------ reference arm (oracle)
+
+
+def reference_arm(args, w):
+    import multiprocessing as mp
+    global _ORACLE_W
+    _ORACLE_W = w
+    cores = os.cpu_count() or 1
+    ctx = mp.get_context("fork")
+    with ctx.Pool(cores) as pool:
+        t0 = time.perf_counter()
+        pool.map(_oracle_job, [([b % w.B], 1) for b in range(cores)])
+        per_round = time.perf_counter() - t0           # one request per core
+        # each step: a bounded sample of requests so that warmup + steps fit in ~2 minutes
+        total = args.steps + args.warmup
+        rounds = max(1, int(120.0 / max(1e-3, per_round) / max(1, total)))
+        sample = [b % w.B for b in range(min(w.B, cores * rounds))]
+        jobs = [([b], 1) for b in sample]
+        for _ in range(args.warmup):
+            pool.map(_oracle_job, jobs, chunksize=1)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            pool.map(_oracle_job, jobs, chunksize=1)
+        wall = time.perf_counter() - t0
+    tokens = sum(w.reqs[b].n for b in sample) * args.steps
+    value = tokens / wall
+    ms = wall / args.steps * 1e3
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded, LLaVA-1.5-shaped; no dataset)", "config": config_of(w),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{len(sample)} of {w.B} requests per step, both stages, fp64, "
+                                   f"one process per core"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    if world != args.gpus and "RANK" in os.environ:
+        print(f"warning: WORLD_SIZE={world} but --gpus {args.gpus}", file=sys.stderr)
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        w = workload()
+        print(json.dumps(reference_arm(args, w)), flush=True)
+        return
+
+    w = workload()
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle(w)                     # before any CUDA call: the pool forks safely
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist.init_process_group("nccl")
+    out = gpu_arm(args, rank, world, w, cpu)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,272 @@
+/*
+ * trevs.h — C ABI of the GB300 (sm_103a) TReVS visual-token pruning library.
+ *
+ * TReVS prunes the visual tokens of a vision-language model in two stages:
+ *   Stage 1 (pre-LLM, Sec. 4.1): score every projected visual token by its
+ *     rectified-cosine textual relevance to the query (Eq. 4-5), combine it with
+ *     the vision encoder's [CLS] saliency (Eq. 3) — by the Sec. 3.1 budget split
+ *     ("textual ratio") or by the MAD-normalised fused score (Eq. 6-7) — keep the
+ *     top K1 tokens and gather their feature rows in their original order.
+ *   Stage 2 (in-LLM at layer l*, Sec. 4.2): compute the text-to-vision
+ *     attention of every head, rank the heads by attention variance (Eq. 8),
+ *     keep the high-variance heads H*, score each visual token by the max over
+ *     text rows of the H*-averaged attention (Eq. 9), keep the top K2 and
+ *     compact the hidden-state and K/V rows of that layer.
+ *
+ * Conventions for every entry point:
+ *   - Tensor pointers are DEVICE memory owned by the caller. bfloat16 tensors are
+ *     passed as their 16-bit patterns (uint16_t). Rows are addressed through the
+ *     strides given (in elements); rows must start on 16-byte boundaries, so
+ *     bf16 base pointers must be 16-byte aligned and bf16 strides multiples of 8.
+ *   - The library never allocates, frees or synchronises. Every call is
+ *     asynchronous on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *     Scratch memory comes from a caller-provided workspace of at least the
+ *     size the matching *_workspace_size() function returns, 256-byte aligned.
+ *     A workspace must be zero-filled before its first use (trevs_workspace_init
+ *     or cudaMemsetAsync); every completed call leaves its counters at zero
+ *     again. After a non-OK status the workspace must be re-initialised.
+ *     Calls that share a workspace must not overlap on the GPU.
+ *   - All index outputs are int32, request-local, in ascending order (which is
+ *     the original token order). Ties in any TopK go to the lower index.
+ *   - Every argument is validated on the host before any launch; invalid
+ *     arguments return TREVS_ERR_INVALID_ARGUMENT and launch nothing. Inputs must
+ *     be finite. The thread-local trevs_last_error_string() explains the last
+ *     non-OK status.
+ *   - No exceptions cross this boundary.
+ */
+#ifndef TREVS_H
+#define TREVS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define TREVS_API __attribute__((visibility("default")))
+#else
+#define TREVS_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum trevs_status {
+  TREVS_OK = 0,
+  TREVS_ERR_INVALID_ARGUMENT = 1, /* bad size, null or misaligned pointer, K > N, ... */
+  TREVS_ERR_WORKSPACE = 2,        /* workspace missing, misaligned or too small */
+  TREVS_ERR_CUDA = 3,             /* a CUDA launch or runtime call failed */
+  TREVS_ERR_UNSUPPORTED = 4,      /* valid but outside this build's limits (see below) */
+  TREVS_ERR_TIMEOUT = 5           /* a bounded device-side wait gave up */
+} trevs_status;
+
+/* Selection rule of stage 1. */
+enum {
+  TREVS_SELECT_RATIO = 0, /* Sec. 3.1: K_t = floor(r*K1 + 1/2) tokens by textual relevance,
+                             K1 - K_t by saliency; saliency top first, textual top over the
+                             remaining tokens; both rank the raw scores. */
+  TREVS_SELECT_FUSED = 1  /* Eq. 6-7: s = max(shat_v, shat_t) + lambda*sqrt(shat_v*shat_t),
+                             shat_c = [(s_c - Med)/(MAD + eps)]_+ / tau_c, then TopK(s, K1).
+                             Med is the lower median (rank floor((N-1)/2) ascending). */
+};
+
+/* Stage-1 hyper-parameters (Eq. 6-7; defaults from the paper's implementation details). */
+typedef struct trevs_pre_params {
+  float tau_v;         /* saliency temperature, default 1.4 */
+  float tau_t;         /* textual temperature, default 1.0 */
+  float lambda;        /* consistency-reward weight, default 1.0 */
+  float eps;           /* MAD stabiliser, default 1e-6 (the paper leaves it unstated) */
+  int32_t select_mode; /* TREVS_SELECT_RATIO (default) or TREVS_SELECT_FUSED */
+} trevs_pre_params;
+
+/* Limits of this build (TREVS_ERR_UNSUPPORTED beyond them). */
+#define TREVS_MAX_TEXT_TOKENS 256    /* M per request, stage 1 */
+#define TREVS_HEAD_DIM 128           /* d_h, stage 2 */
+#define TREVS_MAX_STAGE2_TOKENS 2048 /* K1 per request entering stage 2 */
+#define TREVS_MAX_HEADS 128          /* Hq */
+
+/* Fills *p with the defaults above. */
+TREVS_API void trevs_pre_params_default(trevs_pre_params* p);
+
+/* Library version string ("major.minor.patch"). */
+TREVS_API const char* trevs_version(void);
+
+/* Thread-local, human-readable reason for the last non-OK status of this thread. */
+TREVS_API const char* trevs_last_error_string(void);
+
+/* Number of kernels (and memsets) the last call on this thread enqueued. */
+TREVS_API int32_t trevs_last_launch_count(void);
+
+/* Zero-fills `bytes` of workspace on `stream` (cudaMemsetAsync). */
+TREVS_API trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream);
+
+/* ===================================================================== stage 1, one request
+ *
+ * Z   [N, d] bf16, row r at Z + r*z_row_stride   projected visual features z_i (Sec. 4.1)
+ * T   [M, d] bf16, row j at T + j*t_row_stride   query text embeddings t_j     (Sec. 4.1)
+ * s_v [N] float32                                [CLS] saliency s^v_i          (Eq. 3)
+ */
+
+/* Workspace bytes for trevs_pre_llm_scores / trevs_pre_llm_select on one request of N tokens. */
+TREVS_API size_t trevs_pre_llm_workspace_size(int32_t N);
+
+/* Eq. 4-5: s_t_out[i] = sqrt((1/M) sum_j max(cos(t_j, z_i), 0)^2) for i < N (a zero-norm
+ * row has cosine 0). If s_fused_out is non-NULL, also writes the Eq. 6-7 fused score of
+ * every token using s_v and *p (p may be NULL for the defaults; s_v may be NULL when
+ * s_fused_out is NULL). Limits: 1 <= M <= TREVS_MAX_TEXT_TOKENS, d % 8 == 0. */
+TREVS_API trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                                  const uint16_t* T, int64_t t_row_stride, int32_t M,
+                                  const float* s_v, const trevs_pre_params* p,
+                                  float* s_t_out, float* s_fused_out,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* Stage-1 selection of K1 of the N tokens, written to kept_idx[0..K1) ascending.
+ * Ratio mode (Sec. 3.1) reads s_v, s_t and textual_ratio in [0, 1]. Fused mode (Eq. 6-7)
+ * reads s_fused when non-NULL, else computes it from s_v and s_t with *p.
+ * 0 <= K1 <= N. */
+TREVS_API trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const float* s_fused,
+                                  int32_t N, int32_t K1, float textual_ratio,
+                                  const trevs_pre_params* p, int32_t* kept_idx,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* Z_out[k] = Z[kept_idx[k]] for k < K1 (d bf16 per row): the kept rows, in order, that are
+ * passed into the LLM (Sec. 4.1). A kept_idx[k] outside [0, N) leaves row k untouched. */
+TREVS_API trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                                  const int32_t* kept_idx, int32_t K1,
+                                  uint16_t* Z_out, int64_t z_out_row_stride, void* stream);
+
+/* ===================================================================== stage 2, one request
+ *
+ * Q  text queries at layer l*: element (h, q, c) at Q + h*q_head_stride + q*q_tok_stride + c,
+ *    h < Hq, q < L, c < d_h.
+ * K  visual keys at l*: element (g, i, c) at K + g*k_head_stride + i*k_tok_stride + c,
+ *    g < Hkv, i < K1. Query head h reads key head floor(h*Hkv/Hq) (grouped-query attention).
+ * The attention A^h[q, i] = softmax over the K1 visual keys of (Q_h[q] . K_g[i]) * scale,
+ * scale = softmax_scale if > 0 else 1/sqrt(d_h) (Sec. 4.2).
+ * row_stats [Hq][L][2] float32: per (head, text row) the row max of the scaled logits and
+ * the reciprocal of the row's sum of exp(logit - max).
+ */
+
+/* Workspace bytes for trevs_in_llm_head_scores / trevs_in_llm_select on one request. */
+TREVS_API size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1);
+
+/* Eq. 8: u_out[h] = (1/L) sum_q Var_i A^h[q, i] (population variance over the K1 keys)
+ * and row_stats_out as defined above. Limits: d_h == TREVS_HEAD_DIM,
+ * 1 <= K1 <= TREVS_MAX_STAGE2_TOKENS, 1 <= Hq <= TREVS_MAX_HEADS, Hq % Hkv == 0, L >= 1. */
+TREVS_API trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
+                                      const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
+                                      int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
+                                      float softmax_scale, float* u_out, float* row_stats_out,
+                                      void* workspace, size_t workspace_bytes, void* stream);
+
+/* H* = the n_keep_heads heads of largest u (ties to the lower head), written ascending to
+ * heads_out (may be NULL); Eq. 9 token scores p_i = max_q (1/|H*|) sum_{h in H*} A^h[q, i]
+ * (written to p_out[0..K1) when non-NULL); kept_local[0..K2) = TopK(p, K2) ascending.
+ * u and row_stats are the outputs of trevs_in_llm_head_scores on the same Q and K.
+ * 1 <= n_keep_heads <= Hq, 0 <= K2 <= K1. */
+TREVS_API trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
+                                 const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
+                                 int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
+                                 float softmax_scale, const float* u, const float* row_stats,
+                                 int32_t n_keep_heads, int32_t K2, int32_t* heads_out,
+                                 float* p_out, int32_t* kept_local,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* Compaction at l* (Sec. 4.2): for k < K2 and i = kept_local[k],
+ *   hidden_out[k] = hidden[i]                       (d_model bf16 per row)
+ *   K_out(g, k, :) = Kc(g, i, :), V_out(g, k, :) = Vc(g, i, :) for g < Hkv (d_h bf16 each).
+ * Kc/Vc use (kv_head_stride, kv_tok_stride); K_out/V_out use (out_head_stride, out_tok_stride).
+ * Any of the three tensors may be skipped by passing NULL for both its input and output. */
+TREVS_API trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_stride, int32_t d_model,
+                                  const uint16_t* Kc, const uint16_t* Vc,
+                                  int64_t kv_head_stride, int64_t kv_tok_stride,
+                                  int32_t Hkv, int32_t d_h, int32_t K1,
+                                  const int32_t* kept_local, int32_t K2,
+                                  uint16_t* hidden_out, int64_t hidden_out_row_stride,
+                                  uint16_t* K_out, uint16_t* V_out,
+                                  int64_t out_head_stride, int64_t out_tok_stride, void* stream);
+
+/* ===================================================================== batched (varlen)
+ *
+ * A batch packs the rows of B independent requests back to back. Per-request sizes are
+ * HOST arrays; row offsets are their prefix sums (request b's visual rows start at
+ * sum_{b'<b} n_b', its kept rows at sum_{b'<b} k1_b', and so on). One call launches one
+ * grid per step for the whole batch.
+ */
+
+typedef struct trevs_pre_request {
+  int32_t n;   /* visual tokens N_b (>= 0) */
+  int32_t m;   /* text tokens M_b (1..TREVS_MAX_TEXT_TOKENS when n > 0) */
+  int32_t k1;  /* tokens kept by stage 1 (0..n) */
+  float ratio; /* textual ratio r_b in [0, 1] (ratio mode) */
+} trevs_pre_request;
+
+typedef struct trevs_pre_batch {
+  int32_t B;                       /* number of requests (>= 0) */
+  int32_t d;                       /* feature width d' (% 8 == 0) */
+  const trevs_pre_request* reqs;   /* host [B] */
+  const uint16_t* Z;               /* [sum n, d] */
+  int64_t z_row_stride;
+  const uint16_t* T;               /* [sum m, d] */
+  int64_t t_row_stride;
+  const float* s_v;                /* [sum n] */
+  float* s_t;                      /* optional output [sum n] (NULL: kept in workspace) */
+  float* s_fused;                  /* optional output [sum n], fused mode only */
+  int32_t* kept_idx;               /* output [sum k1], request-local, ascending per request */
+  uint16_t* Z_out;                 /* output [sum k1, d] (NULL: skip the gather) */
+  int64_t z_out_row_stride;
+} trevs_pre_batch;
+
+typedef struct trevs_in_request {
+  int32_t k1; /* visual tokens entering stage 2 (1..TREVS_MAX_STAGE2_TOKENS) */
+  int32_t l;  /* text rows at l* (>= 1) */
+  int32_t k2; /* tokens kept by stage 2 (0..k1) */
+} trevs_in_request;
+
+typedef struct trevs_in_batch {
+  int32_t B, Hq, Hkv, d_h, d_model, n_keep_heads;
+  float softmax_scale;             /* <= 0: 1/sqrt(d_h) */
+  const trevs_in_request* reqs;    /* host [B] */
+  const uint16_t* Q;               /* text rows packed over requests: (h, row) at
+                                      Q + h*q_head_stride + row*q_tok_stride */
+  int64_t q_head_stride, q_tok_stride;
+  const uint16_t* K;               /* visual rows packed: (g, row) at K + g*kv_head_stride + row*kv_tok_stride */
+  const uint16_t* V;               /* same layout as K (NULL: skip V compaction) */
+  int64_t kv_head_stride, kv_tok_stride;
+  const uint16_t* hidden;          /* [sum k1, d_model] (NULL: skip hidden compaction) */
+  int64_t hidden_row_stride;
+  float* u;                        /* optional output [B, Hq] head variances (Eq. 8) */
+  int32_t* heads;                  /* optional output [B, n_keep_heads] H*, ascending */
+  float* p;                        /* optional output [sum k1] token scores (Eq. 9) */
+  int32_t* kept_local;             /* output [sum k2], request-local, ascending */
+  uint16_t* hidden_out;            /* [sum k2, d_model] */
+  int64_t hidden_out_row_stride;
+  uint16_t* K_out;                 /* [.., sum k2 rows] with (out_head_stride, out_tok_stride) */
+  uint16_t* V_out;
+  int64_t out_head_stride, out_tok_stride;
+} trevs_in_batch;
+
+TREVS_API size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch);
+TREVS_API size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch);
+TREVS_API size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in);
+
+/* Stage 1 for a batch: Eq. 4-5 scores, selection (ratio or fused, *p; NULL = defaults)
+ * and gather of the kept rows. */
+TREVS_API trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_params* p,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* Stage 2 for a batch: attention statistics, Eq. 8 head variances, H*, Eq. 9 token scores,
+ * TopK(p, k2) and compaction of hidden, K and V rows. */
+TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* Both stages back to back on one stream (stage 2 reads its own inputs: in a model the two
+ * stages are separated by the first l* LLM layers). */
+TREVS_API trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_params* p,
+                                const trevs_in_batch* in,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TREVS_H */

@@ -1,0 +1,773 @@
+// Host side of the C ABI declared in include/trevs.h: argument validation, workspace
+// layout, per-launch request metadata and the launch sequence of each entry point.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "in_llm.cuh"
+#include "pre_llm.cuh"
+#include "trevs.h"
+
+namespace trevs {
+cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, int max_n, cudaStream_t);
+cudaError_t launch_pre_select(const PreMeta&, const PreArgs&, int max_n, cudaStream_t);
+cudaError_t launch_gather(const GatherMeta&, cudaStream_t);
+cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+}  // namespace trevs
+
+namespace trevs {
+
+cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes) {
+  if (bytes <= 48 * 1024) return cudaSuccess;
+  struct Entry {
+    const void* kernel;
+    int device;
+    int bytes;
+  };
+  static std::mutex mu;
+  static std::vector<Entry> granted;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  for (Entry& x : granted)
+    if (x.kernel == kernel && x.device == dev) {
+      if (x.bytes >= bytes) return cudaSuccess;
+      e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+      if (e == cudaSuccess) x.bytes = bytes;
+      return e;
+    }
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) granted.push_back(Entry{kernel, dev, bytes});
+  return e;
+}
+
+}  // namespace trevs
+
+using namespace trevs;
+
+namespace {
+
+thread_local char g_err[512] = "";
+thread_local int g_launches = 0;     // kernels enqueued by the current call
+
+// Counts one enqueued kernel or memset of the current call.
+inline cudaError_t counted(cudaError_t e) {
+  if (e == cudaSuccess) ++g_launches;
+  return e;
+}
+
+trevs_status fail(trevs_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+trevs_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(TREVS_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+#define TREVS_TRY_CUDA(expr, where)            \
+  do {                                         \
+    cudaError_t e_ = (expr);                   \
+    if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+  } while (0)
+
+#define TREVS_CHECK(cond, ...)                                  \
+  do {                                                          \
+    if (!(cond)) return fail(TREVS_ERR_INVALID_ARGUMENT, __VA_ARGS__); \
+  } while (0)
+
+inline bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// ---------------------------------------------------------------- workspace layouts
+
+struct PreWs {
+  size_t counters, s_t, s_fused, keys, flags, end;
+};
+
+PreWs pre_ws(long long total_n) {
+  PreWs w;
+  size_t o = 0;
+  w.counters = o; o = al256(o + 4 * (size_t)kMaxChunk);
+  w.s_t = o;      o = al256(o + 4 * (size_t)total_n);
+  w.s_fused = o;  o = al256(o + 4 * (size_t)total_n);
+  w.keys = o;     o = al256(o + 4 * (size_t)total_n);
+  w.flags = o;    o = al256(o + (size_t)total_n);
+  w.end = o;
+  return w;
+}
+
+struct InWs {
+  size_t cnt_hs, cnt_ts, row_stats, row_var, u, p, keys, end;
+};
+
+InWs in_ws(long long total_l, long long total_k1, int Hq, int B) {
+  InWs w;
+  size_t o = 0;
+  w.cnt_hs = o;    o = al256(o + 4 * (size_t)kMaxChunk);
+  w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
+  w.row_stats = o; o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
+  w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
+  w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
+  w.p = o;         o = al256(o + 4 * (size_t)total_k1);
+  w.keys = o;      o = al256(o + 4 * (size_t)total_k1);
+  w.end = o;
+  return w;
+}
+
+trevs_status check_ws(void* ws, size_t bytes, size_t need) {
+  if (need == 0) return TREVS_OK;
+  if (ws == nullptr) return fail(TREVS_ERR_WORKSPACE, "workspace is NULL (need %zu bytes)", need);
+  if (((uintptr_t)ws & 255u) != 0) return fail(TREVS_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (bytes < need) return fail(TREVS_ERR_WORKSPACE, "workspace has %zu bytes, need %zu", bytes, need);
+  return TREVS_OK;
+}
+
+int textual_count(int k1, float ratio) {
+  int kt = (int)std::floor((double)ratio * (double)k1 + 0.5);
+  return kt < 0 ? 0 : (kt > k1 ? k1 : kt);
+}
+
+// ---------------------------------------------------------------- stage-1 batch
+
+struct PreTotals {
+  long long n = 0, m = 0, k1 = 0;
+  int max_n = 0, max_m = 0;
+};
+
+trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
+  TREVS_CHECK(bt != nullptr, "pre batch is NULL");
+  TREVS_CHECK(bt->B >= 0, "B = %d < 0", bt->B);
+  if (bt->B == 0) return TREVS_OK;
+  TREVS_CHECK(bt->reqs != nullptr, "reqs is NULL");
+  TREVS_CHECK(bt->d >= 8 && bt->d % 8 == 0, "d = %d must be a positive multiple of 8", bt->d);
+  for (int b = 0; b < bt->B; ++b) {
+    const trevs_pre_request& r = bt->reqs[b];
+    TREVS_CHECK(r.n >= 0, "request %d: n = %d < 0", b, r.n);
+    TREVS_CHECK(r.k1 >= 0 && r.k1 <= r.n, "request %d: k1 = %d outside [0, n = %d]", b, r.k1, r.n);
+    TREVS_CHECK(std::isfinite(r.ratio) && r.ratio >= 0.f && r.ratio <= 1.f,
+                "request %d: textual ratio %g outside [0, 1]", b, (double)r.ratio);
+    if (r.n > 0) {
+      TREVS_CHECK(r.m >= 1, "request %d: m = %d, needs at least one text token", b, r.m);
+      if (r.m > TREVS_MAX_TEXT_TOKENS)
+        return fail(TREVS_ERR_UNSUPPORTED, "request %d: m = %d > %d text tokens", b, r.m, TREVS_MAX_TEXT_TOKENS);
+    } else {
+      TREVS_CHECK(r.m >= 0, "request %d: m = %d < 0", b, r.m);
+    }
+    t.n += r.n; t.m += r.m; t.k1 += r.k1;
+    t.max_n = r.n > t.max_n ? r.n : t.max_n;
+    t.max_m = r.m > t.max_m ? r.m : t.max_m;
+  }
+  TREVS_CHECK(t.n < (1ll << 31) && t.m < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
+  if (t.n > 0) {
+    TREVS_CHECK(bt->Z && bt->T && bt->s_v, "Z, T and s_v must be non-NULL");
+    TREVS_CHECK(aligned16(bt->Z) && aligned16(bt->T), "Z and T must be 16-byte aligned");
+    TREVS_CHECK(bt->z_row_stride >= bt->d && bt->z_row_stride % 8 == 0, "z_row_stride must be >= d and a multiple of 8");
+    TREVS_CHECK(bt->t_row_stride >= bt->d && bt->t_row_stride % 8 == 0, "t_row_stride must be >= d and a multiple of 8");
+  }
+  if (t.k1 > 0) {
+    TREVS_CHECK(bt->kept_idx != nullptr, "kept_idx is NULL");
+    if (bt->Z_out) {
+      TREVS_CHECK(aligned16(bt->Z_out), "Z_out must be 16-byte aligned");
+      TREVS_CHECK(bt->z_out_row_stride >= bt->d && bt->z_out_row_stride % 8 == 0,
+                  "z_out_row_stride must be >= d and a multiple of 8");
+    }
+  }
+  return TREVS_OK;
+}
+
+trevs_status validate_params(const trevs_pre_params* p) {
+  TREVS_CHECK(p->select_mode == TREVS_SELECT_RATIO || p->select_mode == TREVS_SELECT_FUSED,
+              "select_mode %d unknown", p->select_mode);
+  TREVS_CHECK(std::isfinite(p->tau_v) && p->tau_v > 0.f && std::isfinite(p->tau_t) && p->tau_t > 0.f,
+              "temperatures must be positive");
+  TREVS_CHECK(std::isfinite(p->lambda) && std::isfinite(p->eps) && p->eps >= 0.f, "lambda / eps invalid");
+  return TREVS_OK;
+}
+
+// Runs stage 1 for requests [b0, b1) of the batch; offsets are relative to the chunk.
+trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
+                           long long n_base, long long m_base, long long k1_base, uint8_t* ws,
+                           const PreWs& L, cudaStream_t st) {
+  static thread_local PreMeta meta;
+  static thread_local GatherMeta gm;
+  meta.B = b1 - b0;
+  int tiles = 0, max_n = 0, max_m = 0;
+  long long no = 0, mo = 0, ko = 0;
+  for (int b = b0; b < b1; ++b) {
+    const trevs_pre_request& q = bt->reqs[b];
+    PreReq& r = meta.r[b - b0];
+    r.n_off = (int)no; r.n = q.n; r.m_off = (int)mo; r.m = q.m;
+    r.k1_off = (int)ko; r.k1 = q.k1; r.kt = textual_count(q.k1, q.ratio);
+    r.tile_off = tiles;
+    tiles += (q.n + 63) / 64;
+    no += q.n; mo += q.m; ko += q.k1;
+    max_n = q.n > max_n ? q.n : max_n;
+    max_m = q.m > max_m ? q.m : max_m;
+  }
+  meta.total_tiles = tiles;
+  PreArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Z = reinterpret_cast<const __nv_bfloat16*>(bt->Z) + n_base * bt->z_row_stride;
+  a.z_stride = bt->z_row_stride;
+  a.T = reinterpret_cast<const __nv_bfloat16*>(bt->T) + m_base * bt->t_row_stride;
+  a.t_stride = bt->t_row_stride;
+  a.s_v = bt->s_v + n_base;
+  a.s_t = (bt->s_t ? bt->s_t : reinterpret_cast<float*>(ws + L.s_t)) + n_base;
+  a.s_fused = (bt->s_fused ? bt->s_fused : reinterpret_cast<float*>(ws + L.s_fused)) + n_base;
+  a.kept = bt->kept_idx + k1_base;
+  a.flags = ws + L.flags + n_base;
+  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys) + n_base;
+  a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.d = bt->d;
+  a.mode = prm.select_mode == TREVS_SELECT_FUSED ? kModeFused : kModeRatio;
+  a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
+  a.action = kActSelect;
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, max_n, st)), "pre_score launch");
+  if (bt->Z_out && ko > 0) {
+    gm.B = meta.B;
+    gm.njobs = 1;
+    for (int i = 0; i < meta.B; ++i) {
+      gm.dst_off[i] = meta.r[i].k1_off;
+      gm.src_off[i] = meta.r[i].n_off;
+      gm.src_rows[i] = meta.r[i].n;
+    }
+    gm.dst_off[meta.B] = (int)ko;
+    GatherJob& j = gm.job[0];
+    j.src = reinterpret_cast<const uint8_t*>(a.Z);
+    j.dst = reinterpret_cast<uint8_t*>(bt->Z_out + k1_base * bt->z_out_row_stride);
+    j.src_tok = bt->z_row_stride * 2; j.dst_tok = bt->z_out_row_stride * 2;
+    j.src_head = 0; j.dst_head = 0; j.heads = 1; j.row_bytes = bt->d * 2;
+    j.idx = a.kept; j.rows = (int)ko;
+    TREVS_TRY_CUDA(counted(launch_gather(gm, st)), "gather launch");
+  }
+  return TREVS_OK;
+}
+
+trevs_status run_pre_batch(const trevs_pre_batch* bt, const trevs_pre_params& prm, uint8_t* ws,
+                           const PreWs& L, cudaStream_t st) {
+  long long n_base = 0, m_base = 0, k1_base = 0;
+  for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
+    const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
+    trevs_status s = run_pre_chunk(bt, prm, b0, b1, n_base, m_base, k1_base, ws, L, st);
+    if (s != TREVS_OK) return s;
+    for (int b = b0; b < b1; ++b) {
+      n_base += bt->reqs[b].n; m_base += bt->reqs[b].m; k1_base += bt->reqs[b].k1;
+    }
+  }
+  return TREVS_OK;
+}
+
+// ---------------------------------------------------------------- stage-2 batch
+
+struct InTotals {
+  long long l = 0, k1 = 0, k2 = 0;
+  int max_k1 = 0;
+};
+
+trevs_status validate_in_common(int Hq, int Hkv, int d_h, int n_keep) {
+  TREVS_CHECK(Hq >= 1 && Hkv >= 1 && Hq % Hkv == 0, "Hq = %d, Hkv = %d: need Hq %% Hkv == 0", Hq, Hkv);
+  if (Hq > TREVS_MAX_HEADS) return fail(TREVS_ERR_UNSUPPORTED, "Hq = %d > %d", Hq, TREVS_MAX_HEADS);
+  if (d_h != TREVS_HEAD_DIM) return fail(TREVS_ERR_UNSUPPORTED, "d_h = %d, only %d supported", d_h, TREVS_HEAD_DIM);
+  TREVS_CHECK(n_keep >= 1 && n_keep <= Hq, "n_keep_heads = %d outside [1, Hq = %d]", n_keep, Hq);
+  return TREVS_OK;
+}
+
+trevs_status validate_qk(const void* Q, long long qhs, long long qts, const void* K, long long khs,
+                         long long kts) {
+  TREVS_CHECK(Q && K, "Q and K must be non-NULL");
+  TREVS_CHECK(aligned16(Q) && aligned16(K), "Q and K must be 16-byte aligned");
+  TREVS_CHECK(qhs % 8 == 0 && qts % 8 == 0 && khs % 8 == 0 && kts % 8 == 0 && qhs >= 0 && qts >= 0 &&
+                  khs >= 0 && kts >= 0,
+              "Q/K strides must be non-negative multiples of 8");
+  return TREVS_OK;
+}
+
+trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
+  TREVS_CHECK(bt != nullptr, "in batch is NULL");
+  TREVS_CHECK(bt->B >= 0, "B = %d < 0", bt->B);
+  if (bt->B == 0) return TREVS_OK;
+  TREVS_CHECK(bt->reqs != nullptr, "reqs is NULL");
+  trevs_status s = validate_in_common(bt->Hq, bt->Hkv, bt->d_h, bt->n_keep_heads);
+  if (s != TREVS_OK) return s;
+  for (int b = 0; b < bt->B; ++b) {
+    const trevs_in_request& r = bt->reqs[b];
+    TREVS_CHECK(r.k1 >= 1, "request %d: k1 = %d < 1", b, r.k1);
+    if (r.k1 > TREVS_MAX_STAGE2_TOKENS)
+      return fail(TREVS_ERR_UNSUPPORTED, "request %d: k1 = %d > %d", b, r.k1, TREVS_MAX_STAGE2_TOKENS);
+    TREVS_CHECK(r.l >= 1, "request %d: l = %d < 1", b, r.l);
+    TREVS_CHECK(r.k2 >= 0 && r.k2 <= r.k1, "request %d: k2 = %d outside [0, k1 = %d]", b, r.k2, r.k1);
+    t.l += r.l; t.k1 += r.k1; t.k2 += r.k2;
+    t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
+  }
+  TREVS_CHECK(t.l < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
+  s = validate_qk(bt->Q, bt->q_head_stride, bt->q_tok_stride, bt->K, bt->kv_head_stride, bt->kv_tok_stride);
+  if (s != TREVS_OK) return s;
+  if (t.k2 > 0) TREVS_CHECK(bt->kept_local != nullptr, "kept_local is NULL");
+  TREVS_CHECK((bt->hidden == nullptr) == (bt->hidden_out == nullptr), "hidden and hidden_out: both or neither");
+  TREVS_CHECK((bt->V == nullptr) == (bt->V_out == nullptr), "V and V_out: both or neither");
+  if (bt->hidden) {
+    TREVS_CHECK(bt->d_model >= 8 && bt->d_model % 8 == 0, "d_model = %d must be a positive multiple of 8", bt->d_model);
+    TREVS_CHECK(aligned16(bt->hidden) && aligned16(bt->hidden_out), "hidden tensors must be 16-byte aligned");
+    TREVS_CHECK(bt->hidden_row_stride >= bt->d_model && bt->hidden_row_stride % 8 == 0 &&
+                    bt->hidden_out_row_stride >= bt->d_model && bt->hidden_out_row_stride % 8 == 0,
+                "hidden strides must be >= d_model and multiples of 8");
+  }
+  if (bt->K_out || bt->V_out) {
+    TREVS_CHECK(bt->K_out == nullptr || aligned16(bt->K_out), "K_out must be 16-byte aligned");
+    TREVS_CHECK(bt->V_out == nullptr || (aligned16(bt->V) && aligned16(bt->V_out)), "V tensors must be 16-byte aligned");
+    TREVS_CHECK(bt->out_head_stride % 8 == 0 && bt->out_tok_stride % 8 == 0 && bt->out_head_stride >= 0 &&
+                    bt->out_tok_stride >= 0,
+                "K/V output strides must be non-negative multiples of 8");
+  }
+  return TREVS_OK;
+}
+
+void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden, long long hs, int d_model,
+                     uint16_t* hidden_out, long long hos, const uint16_t* K, const uint16_t* V, long long khs,
+                     long long kts, int Hkv, uint16_t* K_out, uint16_t* V_out, long long ohs, long long ots,
+                     const int* kept, int total_k2) {
+  gm.B = meta.B;
+  for (int i = 0; i < meta.B; ++i) {
+    gm.dst_off[i] = meta.r[i].k2_off;
+    gm.src_off[i] = meta.r[i].k1_off;
+    gm.src_rows[i] = meta.r[i].k1;
+  }
+  gm.dst_off[meta.B] = total_k2;
+  int nj = 0;
+  if (hidden) {
+    GatherJob& j = gm.job[nj++];
+    j.src = reinterpret_cast<const uint8_t*>(hidden); j.dst = reinterpret_cast<uint8_t*>(hidden_out);
+    j.src_tok = hs * 2; j.dst_tok = hos * 2; j.src_head = 0; j.dst_head = 0;
+    j.heads = 1; j.row_bytes = d_model * 2; j.idx = kept; j.rows = total_k2;
+  }
+  const uint16_t* srcs[2] = {K, V};
+  uint16_t* dsts[2] = {K_out, V_out};
+  for (int x = 0; x < 2; ++x) {
+    if (!srcs[x] || !dsts[x]) continue;
+    GatherJob& j = gm.job[nj++];
+    j.src = reinterpret_cast<const uint8_t*>(srcs[x]); j.dst = reinterpret_cast<uint8_t*>(dsts[x]);
+    j.src_tok = kts * 2; j.dst_tok = ots * 2; j.src_head = khs * 2; j.dst_head = ohs * 2;
+    j.heads = Hkv; j.row_bytes = TREVS_HEAD_DIM * 2; j.idx = kept; j.rows = total_k2;
+  }
+  gm.njobs = nj;
+}
+
+trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
+                          long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st) {
+  static thread_local InMeta meta;
+  static thread_local GatherMeta gm;
+  meta.B = b1 - b0;
+  int hs = 0, ts = 0, max_k1 = 0;
+  long long lo = 0, ko = 0, k2o = 0;
+  for (int b = b0; b < b1; ++b) {
+    const trevs_in_request& q = bt->reqs[b];
+    InReq& r = meta.r[b - b0];
+    r.l_off = (int)lo; r.l = q.l; r.k1_off = (int)ko; r.k1 = q.k1; r.k2_off = (int)k2o; r.k2 = q.k2;
+    r.hs_off = hs; r.ts_off = ts;
+    const int nqb = (q.l + 15) / 16;
+    hs += bt->Hq * nqb;
+    ts += nqb * ((q.k1 + 63) / 64);
+    lo += q.l; ko += q.k1; k2o += q.k2;
+    max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
+  }
+  meta.total_hs = hs;
+  meta.total_ts = ts;
+  InArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Q = reinterpret_cast<const __nv_bfloat16*>(bt->Q) + l_base * bt->q_tok_stride;
+  a.q_hs = bt->q_head_stride; a.q_ts = bt->q_tok_stride;
+  a.K = reinterpret_cast<const __nv_bfloat16*>(bt->K) + k1_base * bt->kv_tok_stride;
+  a.k_hs = bt->kv_head_stride; a.k_ts = bt->kv_tok_stride;
+  a.Hq = bt->Hq; a.Hkv = bt->Hkv; a.n_keep = bt->n_keep_heads;
+  a.scale = bt->softmax_scale > 0.f ? bt->softmax_scale : 1.0f / sqrtf((float)bt->d_h);
+  a.row_stats = reinterpret_cast<float2*>(ws + L.row_stats);
+  a.row_var = reinterpret_cast<float*>(ws + L.row_var);
+  a.stats_ld = lo;
+  a.u = (bt->u ? bt->u : reinterpret_cast<float*>(ws + L.u)) + (long long)b0 * bt->Hq;
+  a.u_ld = bt->Hq;
+  a.p_bits = (bt->p ? reinterpret_cast<uint32_t*>(bt->p) : reinterpret_cast<uint32_t*>(ws + L.p)) + k1_base;
+  a.kept_local = bt->kept_local ? bt->kept_local + k2_base : nullptr;
+  a.heads_out = bt->heads ? bt->heads + (long long)b0 * bt->n_keep_heads : nullptr;
+  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys) + k1_base;
+  a.cnt_hs = reinterpret_cast<uint32_t*>(ws + L.cnt_hs);
+  a.cnt_ts = reinterpret_cast<uint32_t*>(ws + L.cnt_ts);
+  a.hs_finalize = 1;
+  a.zero_p = 1;
+  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
+  TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
+  if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
+    fill_compaction(gm, meta,
+                    bt->hidden ? bt->hidden + k1_base * bt->hidden_row_stride : nullptr, bt->hidden_row_stride,
+                    bt->d_model,
+                    bt->hidden_out ? bt->hidden_out + k2_base * bt->hidden_out_row_stride : nullptr,
+                    bt->hidden_out_row_stride, bt->K_out ? bt->K + k1_base * bt->kv_tok_stride : nullptr,
+                    bt->V ? bt->V + k1_base * bt->kv_tok_stride : nullptr, bt->kv_head_stride, bt->kv_tok_stride,
+                    bt->Hkv, bt->K_out ? bt->K_out + k2_base * bt->out_tok_stride : nullptr,
+                    bt->V_out ? bt->V_out + k2_base * bt->out_tok_stride : nullptr, bt->out_head_stride,
+                    bt->out_tok_stride, a.kept_local, (int)k2o);
+    TREVS_TRY_CUDA(counted(launch_gather(gm, st)), "compaction launch");
+  }
+  return TREVS_OK;
+}
+
+trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st) {
+  long long l_base = 0, k1_base = 0, k2_base = 0;
+  for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
+    const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
+    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st);
+    if (s != TREVS_OK) return s;
+    for (int b = b0; b < b1; ++b) {
+      l_base += bt->reqs[b].l; k1_base += bt->reqs[b].k1; k2_base += bt->reqs[b].k2;
+    }
+  }
+  return TREVS_OK;
+}
+
+const trevs_pre_params kDefaults = {1.4f, 1.0f, 1.0f, 1e-6f, TREVS_SELECT_RATIO};
+
+}  // namespace
+
+// ======================================================================== C ABI
+
+extern "C" {
+
+void trevs_pre_params_default(trevs_pre_params* p) {
+  if (p) *p = kDefaults;
+}
+
+const char* trevs_version(void) { return "0.1.0"; }
+
+const char* trevs_last_error_string(void) { return g_err; }
+
+int32_t trevs_last_launch_count(void) { return g_launches; }
+
+trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream) {
+  g_launches = 0;
+  if (bytes == 0) return TREVS_OK;
+  if (!workspace) return fail(TREVS_ERR_WORKSPACE, "workspace is NULL");
+  TREVS_TRY_CUDA(counted(cudaMemsetAsync(workspace, 0, bytes, (cudaStream_t)stream)), "workspace memset");
+  return TREVS_OK;
+}
+
+size_t trevs_pre_llm_workspace_size(int32_t N) { return N < 0 ? 0 : pre_ws(N).end; }
+
+trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                                  const uint16_t* T, int64_t t_row_stride, int32_t M, const float* s_v,
+                                  const trevs_pre_params* p, float* s_t_out, float* s_fused_out,
+                                  void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  const trevs_pre_params prm = p ? *p : kDefaults;
+  trevs_status s = validate_params(&prm);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(N >= 0, "N = %d < 0", N);
+  if (N == 0) return TREVS_OK;
+  TREVS_CHECK(s_t_out != nullptr, "s_t_out is NULL");
+  TREVS_CHECK(s_fused_out == nullptr || s_v != nullptr, "s_v is needed for the fused score");
+  trevs_pre_request rq = {N, M, 0, 0.f};
+  trevs_pre_batch bt;
+  memset(&bt, 0, sizeof(bt));
+  bt.B = 1; bt.d = d; bt.reqs = &rq; bt.Z = Z; bt.z_row_stride = z_row_stride; bt.T = T;
+  bt.t_row_stride = t_row_stride; bt.s_v = s_v ? s_v : s_t_out;
+  PreTotals tot;
+  s = validate_pre_batch(&bt, tot);
+  if (s != TREVS_OK) return s;
+  const PreWs L = pre_ws(N);
+  s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  static thread_local PreMeta meta;
+  meta.B = 1;
+  meta.r[0] = PreReq{0, N, 0, M, 0, 0, 0, 0};
+  meta.total_tiles = (N + 63) / 64;
+  PreArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Z = reinterpret_cast<const __nv_bfloat16*>(Z); a.z_stride = z_row_stride;
+  a.T = reinterpret_cast<const __nv_bfloat16*>(T); a.t_stride = t_row_stride;
+  a.s_v = bt.s_v; a.s_t = s_t_out;
+  a.s_fused = s_fused_out;
+  a.flags = ws + L.flags; a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
+  a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.d = d; a.mode = s_fused_out ? kModeFused : kModeRatio;
+  a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
+  a.action = s_fused_out ? kActScoresFused : kActScores;
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream)), "pre_score launch");
+  return TREVS_OK;
+}
+
+trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const float* s_fused, int32_t N,
+                                  int32_t K1, float textual_ratio, const trevs_pre_params* p,
+                                  int32_t* kept_idx, void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  const trevs_pre_params prm = p ? *p : kDefaults;
+  trevs_status s = validate_params(&prm);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(N >= 0 && K1 >= 0 && K1 <= N, "need 0 <= K1 (%d) <= N (%d)", K1, N);
+  TREVS_CHECK(std::isfinite(textual_ratio) && textual_ratio >= 0.f && textual_ratio <= 1.f,
+              "textual ratio %g outside [0, 1]", (double)textual_ratio);
+  if (K1 == 0) return TREVS_OK;
+  TREVS_CHECK(kept_idx != nullptr, "kept_idx is NULL");
+  const bool fused = prm.select_mode == TREVS_SELECT_FUSED;
+  if (fused && !s_fused) TREVS_CHECK(s_v && s_t, "fused mode needs s_fused or both s_v and s_t");
+  if (!fused) TREVS_CHECK(s_v && s_t, "ratio mode needs s_v and s_t");
+  const PreWs L = pre_ws(N);
+  s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  static thread_local PreMeta meta;
+  meta.B = 1;
+  meta.r[0] = PreReq{0, N, 0, 0, 0, K1, textual_count(K1, textual_ratio), 0};
+  meta.total_tiles = 0;
+  PreArgs a;
+  memset(&a, 0, sizeof(a));
+  a.s_v = s_v; a.s_t = const_cast<float*>(s_t);
+  a.s_fused = s_fused ? const_cast<float*>(s_fused) : reinterpret_cast<float*>(ws + L.s_fused);
+  a.s_fused_given = s_fused != nullptr;
+  a.kept = kept_idx;
+  a.flags = ws + L.flags; a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
+  a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.mode = fused ? kModeFused : kModeRatio;
+  a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
+  a.action = kActSelect;
+  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream)), "pre_select launch");
+  return TREVS_OK;
+}
+
+trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                                  const int32_t* kept_idx, int32_t K1, uint16_t* Z_out,
+                                  int64_t z_out_row_stride, void* stream) {
+  g_launches = 0;
+  TREVS_CHECK(N >= 0 && K1 >= 0 && K1 <= N, "need 0 <= K1 (%d) <= N (%d)", K1, N);
+  if (K1 == 0) return TREVS_OK;
+  TREVS_CHECK(d >= 8 && d % 8 == 0, "d = %d must be a positive multiple of 8", d);
+  TREVS_CHECK(Z && kept_idx && Z_out, "Z, kept_idx and Z_out must be non-NULL");
+  TREVS_CHECK(aligned16(Z) && aligned16(Z_out), "Z and Z_out must be 16-byte aligned");
+  TREVS_CHECK(z_row_stride >= d && z_row_stride % 8 == 0 && z_out_row_stride >= d && z_out_row_stride % 8 == 0,
+              "row strides must be >= d and multiples of 8");
+  static thread_local GatherMeta gm;
+  gm.B = 1; gm.njobs = 1;
+  gm.dst_off[0] = 0; gm.dst_off[1] = K1; gm.src_off[0] = 0; gm.src_rows[0] = N;
+  GatherJob& j = gm.job[0];
+  j.src = reinterpret_cast<const uint8_t*>(Z); j.dst = reinterpret_cast<uint8_t*>(Z_out);
+  j.src_tok = z_row_stride * 2; j.dst_tok = z_out_row_stride * 2; j.src_head = 0; j.dst_head = 0;
+  j.heads = 1; j.row_bytes = d * 2; j.idx = kept_idx; j.rows = K1;
+  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream)), "gather launch");
+  return TREVS_OK;
+}
+
+size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1) {
+  if (Hq < 0 || L < 0 || K1 < 0) return 0;
+  return in_ws(L, K1, Hq, 1).end;
+}
+
+trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
+                                      const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
+                                      int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
+                                      float softmax_scale, float* u_out, float* row_stats_out,
+                                      void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  trevs_status s = validate_in_common(Hq, Hkv, d_h, 1);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(L >= 1, "L = %d < 1", L);
+  TREVS_CHECK(K1 >= 1, "K1 = %d < 1", K1);
+  if (K1 > TREVS_MAX_STAGE2_TOKENS) return fail(TREVS_ERR_UNSUPPORTED, "K1 = %d > %d", K1, TREVS_MAX_STAGE2_TOKENS);
+  s = validate_qk(Q, q_head_stride, q_tok_stride, K, k_head_stride, k_tok_stride);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(u_out && row_stats_out, "u_out and row_stats_out must be non-NULL");
+  TREVS_CHECK(((uintptr_t)row_stats_out & 7u) == 0, "row_stats_out must be 8-byte aligned");
+  const InWs W = in_ws(L, K1, Hq, 1);
+  s = check_ws(workspace, workspace_bytes, W.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  static thread_local InMeta meta;
+  meta.B = 1;
+  meta.r[0] = InReq{0, L, 0, K1, 0, 0, 0, 0};
+  meta.total_hs = Hq * ((L + 15) / 16);
+  meta.total_ts = 0;
+  InArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Q = reinterpret_cast<const __nv_bfloat16*>(Q); a.q_hs = q_head_stride; a.q_ts = q_tok_stride;
+  a.K = reinterpret_cast<const __nv_bfloat16*>(K); a.k_hs = k_head_stride; a.k_ts = k_tok_stride;
+  a.Hq = Hq; a.Hkv = Hkv; a.n_keep = 1;
+  a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
+  a.row_stats = reinterpret_cast<float2*>(row_stats_out);
+  a.row_var = reinterpret_cast<float*>(ws + W.row_var);
+  a.stats_ld = L;
+  a.u = u_out; a.u_ld = Hq;
+  a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
+  a.cnt_ts = reinterpret_cast<uint32_t*>(ws + W.cnt_ts);
+  a.hs_finalize = 1; a.zero_p = 0;
+  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, K1, (cudaStream_t)stream)), "head_stats launch");
+  return TREVS_OK;
+}
+
+trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
+                                 const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride, int32_t Hq,
+                                 int32_t Hkv, int32_t L, int32_t K1, int32_t d_h, float softmax_scale,
+                                 const float* u, const float* row_stats, int32_t n_keep_heads, int32_t K2,
+                                 int32_t* heads_out, float* p_out, int32_t* kept_local, void* workspace,
+                                 size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  trevs_status s = validate_in_common(Hq, Hkv, d_h, n_keep_heads);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(L >= 1, "L = %d < 1", L);
+  TREVS_CHECK(K1 >= 1, "K1 = %d < 1", K1);
+  if (K1 > TREVS_MAX_STAGE2_TOKENS) return fail(TREVS_ERR_UNSUPPORTED, "K1 = %d > %d", K1, TREVS_MAX_STAGE2_TOKENS);
+  TREVS_CHECK(K2 >= 0 && K2 <= K1, "K2 = %d outside [0, K1 = %d]", K2, K1);
+  s = validate_qk(Q, q_head_stride, q_tok_stride, K, k_head_stride, k_tok_stride);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(u && row_stats, "u and row_stats must be non-NULL");
+  TREVS_CHECK(((uintptr_t)row_stats & 7u) == 0, "row_stats must be 8-byte aligned");
+  if (K2 > 0) TREVS_CHECK(kept_local != nullptr, "kept_local is NULL");
+  const InWs W = in_ws(L, K1, Hq, 1);
+  s = check_ws(workspace, workspace_bytes, W.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  static thread_local InMeta meta;
+  meta.B = 1;
+  meta.r[0] = InReq{0, L, 0, K1, 0, K2, 0, 0};
+  meta.total_hs = 0;
+  meta.total_ts = ((L + 15) / 16) * ((K1 + 63) / 64);
+  InArgs a;
+  memset(&a, 0, sizeof(a));
+  a.Q = reinterpret_cast<const __nv_bfloat16*>(Q); a.q_hs = q_head_stride; a.q_ts = q_tok_stride;
+  a.K = reinterpret_cast<const __nv_bfloat16*>(K); a.k_hs = k_head_stride; a.k_ts = k_tok_stride;
+  a.Hq = Hq; a.Hkv = Hkv; a.n_keep = n_keep_heads;
+  a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
+  a.row_stats = reinterpret_cast<float2*>(const_cast<float*>(row_stats));
+  a.stats_ld = L;
+  a.u = const_cast<float*>(u); a.u_ld = Hq;
+  a.p_bits = p_out ? reinterpret_cast<uint32_t*>(p_out) : reinterpret_cast<uint32_t*>(ws + W.p);
+  a.kept_local = kept_local; a.heads_out = heads_out;
+  a.keys = reinterpret_cast<uint32_t*>(ws + W.keys);
+  a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
+  a.cnt_ts = reinterpret_cast<uint32_t*>(ws + W.cnt_ts);
+  TREVS_TRY_CUDA(counted(cudaMemsetAsync(a.p_bits, 0, 4 * (size_t)K1, (cudaStream_t)stream)), "p memset");
+  TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, K1, (cudaStream_t)stream)), "token_score launch");
+  return TREVS_OK;
+}
+
+trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_stride, int32_t d_model,
+                                  const uint16_t* Kc, const uint16_t* Vc, int64_t kv_head_stride,
+                                  int64_t kv_tok_stride, int32_t Hkv, int32_t d_h, int32_t K1,
+                                  const int32_t* kept_local, int32_t K2, uint16_t* hidden_out,
+                                  int64_t hidden_out_row_stride, uint16_t* K_out, uint16_t* V_out,
+                                  int64_t out_head_stride, int64_t out_tok_stride, void* stream) {
+  g_launches = 0;
+  TREVS_CHECK(K1 >= 0 && K2 >= 0 && K2 <= K1, "need 0 <= K2 (%d) <= K1 (%d)", K2, K1);
+  if (K2 == 0) return TREVS_OK;
+  TREVS_CHECK(kept_local != nullptr, "kept_local is NULL");
+  TREVS_CHECK((hidden == nullptr) == (hidden_out == nullptr), "hidden and hidden_out: both or neither");
+  TREVS_CHECK((Kc == nullptr) == (K_out == nullptr), "Kc and K_out: both or neither");
+  TREVS_CHECK((Vc == nullptr) == (V_out == nullptr), "Vc and V_out: both or neither");
+  if (hidden) {
+    TREVS_CHECK(d_model >= 8 && d_model % 8 == 0, "d_model = %d must be a positive multiple of 8", d_model);
+    TREVS_CHECK(aligned16(hidden) && aligned16(hidden_out), "hidden tensors must be 16-byte aligned");
+    TREVS_CHECK(hidden_row_stride >= d_model && hidden_row_stride % 8 == 0 && hidden_out_row_stride >= d_model &&
+                    hidden_out_row_stride % 8 == 0,
+                "hidden strides must be >= d_model and multiples of 8");
+  }
+  if (Kc || Vc) {
+    TREVS_CHECK(Hkv >= 1, "Hkv = %d < 1", Hkv);
+    if (d_h != TREVS_HEAD_DIM) return fail(TREVS_ERR_UNSUPPORTED, "d_h = %d, only %d supported", d_h, TREVS_HEAD_DIM);
+    TREVS_CHECK((!Kc || (aligned16(Kc) && aligned16(K_out))) && (!Vc || (aligned16(Vc) && aligned16(V_out))),
+                "K/V tensors must be 16-byte aligned");
+    TREVS_CHECK(kv_head_stride % 8 == 0 && kv_tok_stride % 8 == 0 && out_head_stride % 8 == 0 &&
+                    out_tok_stride % 8 == 0 && kv_head_stride >= 0 && kv_tok_stride >= 0 && out_head_stride >= 0 &&
+                    out_tok_stride >= 0,
+                "K/V strides must be non-negative multiples of 8");
+  }
+  static thread_local InMeta meta;
+  static thread_local GatherMeta gm;
+  meta.B = 1;
+  meta.r[0] = InReq{0, 0, 0, K1, 0, K2, 0, 0};
+  fill_compaction(gm, meta, hidden, hidden_row_stride, d_model, hidden_out, hidden_out_row_stride, Kc, Vc,
+                  kv_head_stride, kv_tok_stride, Hkv, K_out, V_out, out_head_stride, out_tok_stride, kept_local, K2);
+  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream)), "compaction launch");
+  return TREVS_OK;
+}
+
+size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
+  if (!batch || batch->B <= 0 || !batch->reqs) return 0;
+  long long n = 0;
+  for (int b = 0; b < batch->B; ++b) n += batch->reqs[b].n > 0 ? batch->reqs[b].n : 0;
+  return pre_ws(n).end;
+}
+
+size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
+  if (!batch || batch->B <= 0 || !batch->reqs) return 0;
+  long long l = 0, k1 = 0;
+  for (int b = 0; b < batch->B; ++b) {
+    l += batch->reqs[b].l > 0 ? batch->reqs[b].l : 0;
+    k1 += batch->reqs[b].k1 > 0 ? batch->reqs[b].k1 : 0;
+  }
+  return in_ws(l, k1, batch->Hq > 0 ? batch->Hq : 0, batch->B).end;
+}
+
+size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in) {
+  return al256(trevs_pre_llm_varlen_workspace_size(pre)) + trevs_in_llm_varlen_workspace_size(in);
+}
+
+trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_params* p, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  const trevs_pre_params prm = p ? *p : kDefaults;
+  trevs_status s = validate_params(&prm);
+  if (s != TREVS_OK) return s;
+  PreTotals t;
+  s = validate_pre_batch(batch, t);
+  if (s != TREVS_OK || batch->B == 0) return s;
+  const PreWs L = pre_ws(t.n);
+  s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
+}
+
+trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch, void* workspace, size_t workspace_bytes,
+                                 void* stream) {
+  g_launches = 0;
+  InTotals t;
+  trevs_status s = validate_in_batch(batch, t);
+  if (s != TREVS_OK || batch->B == 0) return s;
+  const InWs L = in_ws(t.l, t.k1, batch->Hq, batch->B);
+  s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  return run_in_batch(batch, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
+}
+
+trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_params* p, const trevs_in_batch* in,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  const trevs_pre_params prm = p ? *p : kDefaults;
+  trevs_status s = validate_params(&prm);
+  if (s != TREVS_OK) return s;
+  PreTotals tp;
+  InTotals ti;
+  s = validate_pre_batch(pre, tp);
+  if (s != TREVS_OK) return s;
+  s = validate_in_batch(in, ti);
+  if (s != TREVS_OK) return s;
+  const PreWs LP = pre_ws(tp.n);
+  const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
+  const InWs LI = in_ws(ti.l, ti.k1, in->B > 0 ? in->Hq : 0, in->B);
+  const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);
+  s = check_ws(workspace, workspace_bytes, need);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  if (pre->B > 0) {
+    s = run_pre_batch(pre, prm, ws, LP, (cudaStream_t)stream);
+    if (s != TREVS_OK) return s;
+  }
+  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, (cudaStream_t)stream);
+  return TREVS_OK;
+}
+
+}  // extern "C"

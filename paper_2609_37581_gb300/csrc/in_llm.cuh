@@ -1,0 +1,32 @@
+// Stage 2 (in-LLM, Sec. 4.2) kernel arguments.
+#pragma once
+
+#include "common.cuh"
+
+namespace trevs {
+
+constexpr int kMaxHeads = 128;
+
+struct InArgs {
+  const __nv_bfloat16* Q;
+  long long q_hs, q_ts;     // head / token strides (elements)
+  const __nv_bfloat16* K;
+  long long k_hs, k_ts;
+  int Hq, Hkv, n_keep;
+  float scale;
+  float2* row_stats;        // [Hq][stats_ld]: (row max of scaled logits, 1 / row sum of exp)
+  float* row_var;           // [Hq][stats_ld]: Var_i A[q, i]
+  long long stats_ld;       // total text rows of the launch
+  float* u;                 // [B][u_ld] head variances (Eq. 8)
+  int u_ld;
+  uint32_t* p_bits;         // [sum k1] Eq. 9 scores as float bits (atomicMax target)
+  int* kept_local;          // [sum k2]
+  int* heads_out;           // [B][n_keep] or null
+  uint32_t* keys;           // [sum k1] selection scratch
+  uint32_t* cnt_hs;         // [B] self-resetting tickets
+  uint32_t* cnt_ts;         // [B]
+  int hs_finalize;          // head-statistics blocks reduce u (ticket)
+  int zero_p;               // ... and clear p for the token-score pass
+};
+
+}  // namespace trevs

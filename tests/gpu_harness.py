@@ -1,0 +1,126 @@
+"""Runs a synthetic workload through the C ABI on the GPU and compares it with the oracle.
+
+Comparison rules (tolerances follow from fp32 accumulation of bf16 products):
+  * float scores (s^t, fused s, u_h, p_i): |gpu - oracle| <= RTOL * |oracle| + ATOL;
+  * kept index sets: identical, unless the oracle's K-th and (K+1)-th scores differ by
+    less than NEAR_TIE relative; such near-ties are counted, and the GPU set must then
+    still hold exactly K distinct valid indices;
+  * gathered / compacted rows: bit-exact copies of the rows the GPU kept.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+import oracle.trevs_oracle as O
+from workloads.device import GpuRun, build_batches, collect, dev_bf16, dev_f32, host_u16, run_gpu  # noqa: F401
+
+RTOL = 1e-3
+ATOL_ST = 1e-6     # s^t is a mean of squares of cosines: fp32 cosine error ~1e-7 absolute
+ATOL_FUSED = 1e-4  # fused scores near 0 are (s - Med) / MAD with fp32 Med and MAD
+ATOL_P = 1e-7      # attention probabilities
+NEAR_TIE = 1e-4
+
+
+# ------------------------------------------------------------------ comparisons
+
+
+def assert_close(gpu, ref, rtol, atol, what):
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert gpu.shape == ref.shape, (what, gpu.shape, ref.shape)
+    err = np.abs(gpu - ref)
+    bad = err > atol + rtol * np.abs(ref)
+    if bad.any():
+        i = int(np.argmax(err - (atol + rtol * np.abs(ref))))
+        raise AssertionError(f"{what}: {int(bad.sum())} of {gpu.size} outside tolerance; worst at {i}: "
+                             f"gpu {gpu.flat[i]!r} oracle {ref.flat[i]!r}")
+
+
+def boundary_gap(scores, k, allowed=None):
+    """Relative gap between the oracle's k-th and (k+1)-th scores (inf if no (k+1)-th)."""
+    s = np.asarray(scores, np.float64)
+    if allowed is not None:
+        s = s[np.asarray(allowed, bool)]
+    if k <= 0 or k >= len(s):
+        return np.inf
+    top = np.sort(s)[::-1]
+    a, b = top[k - 1], top[k]
+    den = max(abs(a), abs(b))
+    return 0.0 if den == 0 else abs(a - b) / den
+
+
+@dataclasses.dataclass
+class Tally:
+    requests: int = 0
+    stage1_near_ties: int = 0
+    stage2_near_ties: int = 0
+    stage1_exact: int = 0
+    stage2_exact: int = 0
+
+
+def check_workload(w, g: GpuRun, ref, mode="ratio", tally: Tally | None = None, params=None):
+    """Element-wise comparison of one GPU run with the oracle, request by request."""
+    tally = tally or Tally()
+    params = params or {}
+    n_off, k1_off, k2_off = w.offsets("n"), w.offsets("k1"), w.offsets("k2")
+    for b, r in enumerate(w.reqs):
+        tally.requests += 1
+        res = ref[b]
+        # ---- stage 1
+        if "pre" in res:
+            pre = res["pre"]
+            st = g.s_t[n_off[b]:n_off[b + 1]]
+            assert_close(st, pre["s_t"], RTOL, ATOL_ST, f"req {b} s_t")
+            kept = g.kept1[k1_off[b]:k1_off[b + 1]]
+            assert len(kept) == r.k1
+            assert np.all(np.diff(kept) > 0), f"req {b}: stage-1 indices not strictly ascending"
+            assert kept.size == 0 or (kept[0] >= 0 and kept[-1] < r.n)
+            if mode == "ratio":
+                kt = O.textual_count(r.k1, r.ratio)
+                sv = w.s_v[n_off[b]:n_off[b + 1]].astype(np.float64)
+                Sv = O.top_k(sv, r.k1 - kt)
+                rest = np.ones(r.n, bool)
+                rest[Sv] = False
+                # saliency decisions compare the same fp32 inputs on both sides: exact;
+                # only the computed textual scores carry a near-tie band
+                near = boundary_gap(pre["s_t"], kt, rest) < NEAR_TIE
+            else:
+                assert_close(g.s_fused[n_off[b]:n_off[b + 1]], pre["s_fused"], RTOL, ATOL_FUSED, f"req {b} fused")
+                near = boundary_gap(pre["s_fused"], r.k1) < NEAR_TIE
+            if near:
+                tally.stage1_near_ties += 1
+            else:
+                np.testing.assert_array_equal(kept, pre["kept"], err_msg=f"req {b} stage-1 kept set")
+                tally.stage1_exact += 1
+            # gathered rows are exact copies of the rows the GPU kept
+            Zb = w.Z[n_off[b]:n_off[b + 1]]
+            np.testing.assert_array_equal(g.Z_out[k1_off[b]:k1_off[b + 1]], Zb[kept], err_msg=f"req {b} Z_out")
+        # ---- stage 2
+        if "in" in res:
+            inn = res["in"]
+            assert_close(g.u[b], inn["u"], RTOL, 1e-9, f"req {b} u")
+            heads = g.heads[b]
+            head_near = boundary_gap(inn["u"], w.n_keep_heads) < NEAR_TIE
+            kept2 = g.kept2[k2_off[b]:k2_off[b + 1]]
+            assert len(kept2) == r.k2
+            assert np.all(np.diff(kept2) > 0), f"req {b}: stage-2 indices not strictly ascending"
+            assert kept2.size == 0 or (kept2[0] >= 0 and kept2[-1] < r.k1)
+            if head_near:
+                tally.stage2_near_ties += 1
+            else:
+                np.testing.assert_array_equal(heads, inn["heads"], err_msg=f"req {b} heads")
+                assert_close(g.p[k1_off[b]:k1_off[b + 1]], inn["p"], RTOL, ATOL_P, f"req {b} p")
+                if boundary_gap(inn["p"], r.k2) < NEAR_TIE:
+                    tally.stage2_near_ties += 1
+                else:
+                    np.testing.assert_array_equal(kept2, inn["kept"], err_msg=f"req {b} stage-2 kept set")
+                    tally.stage2_exact += 1
+            Hb = w.hidden[k1_off[b]:k1_off[b + 1]]
+            Kb = w.K[k1_off[b]:k1_off[b + 1]]
+            Vb = w.V[k1_off[b]:k1_off[b + 1]]
+            np.testing.assert_array_equal(g.hidden_out[k2_off[b]:k2_off[b + 1]], Hb[kept2], err_msg=f"req {b} hidden")
+            np.testing.assert_array_equal(g.K_out[k2_off[b]:k2_off[b + 1]], Kb[kept2], err_msg=f"req {b} K_out")
+            np.testing.assert_array_equal(g.V_out[k2_off[b]:k2_off[b + 1]], Vb[kept2], err_msg=f"req {b} V_out")
+    return tally

@@ -1,0 +1,164 @@
+"""The C ABI loads, exports every symbol include/trevs.h declares, and validates on the host.
+
+These tests need no GPU: every call here fails validation before any CUDA call, or is
+a size query.
+"""
+import ctypes
+import pathlib
+import re
+
+import pytest
+
+from paper_2609_37581_gb300 import trevs as t
+
+ROOT = pathlib.Path(__file__).resolve().parent.parent
+HEADER = ROOT / "include" / "trevs.h"
+FAKE = ctypes.c_void_p(0x10000)        # aligned, never dereferenced: validation fails first
+
+
+def declared():
+    text = HEADER.read_text()
+    return sorted(set(re.findall(r"TREVS_API\s+[\w\s\*]+?\b(trevs_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return t.load()
+
+
+def test_header_declares_entry_points():
+    names = declared()
+    for must in ("trevs_pre_llm_scores", "trevs_pre_llm_select", "trevs_pre_llm_gather",
+                 "trevs_in_llm_head_scores", "trevs_in_llm_select", "trevs_in_llm_compact",
+                 "trevs_prune_varlen"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared():
+        assert hasattr(lib, name), name
+        assert name in t.EXPORTED, name
+
+
+def test_version_and_defaults(lib):
+    assert t.version().count(".") == 2
+    p = t.default_params()
+    assert (round(p.tau_v, 6), p.tau_t, p.lambda_, p.select_mode) == (1.4, 1.0, 1.0, t.SELECT_RATIO)
+    assert abs(p.eps - 1e-6) < 1e-12
+
+
+def _err(lib):
+    return lib.trevs_last_error_string().decode()
+
+
+def test_select_validation(lib):
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 10, 11, 0.5, None, FAKE, FAKE, 1 << 20, None) == 1
+    assert "K1" in _err(lib)
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 10, 5, 1.5, None, FAKE, FAKE, 1 << 20, None) == 1
+    assert lib.trevs_pre_llm_select(FAKE, None, None, 10, 5, 0.5, None, FAKE, FAKE, 1 << 20, None) == 1
+    # K1 = 0 is a valid no-op
+    assert lib.trevs_pre_llm_select(None, None, None, 10, 0, 0.5, None, None, None, 0, None) == 0
+    # bad mode
+    p = t.default_params(mode=7)
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 10, 5, 0.5, ctypes.byref(p), FAKE, FAKE, 1 << 20, None) == 1
+
+
+def test_workspace_validation(lib):
+    need = lib.trevs_pre_llm_workspace_size(1000)
+    assert need > 0 and need % 256 == 0
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 1000, 5, 0.5, None, FAKE, FAKE, need - 1, None) == 2
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 1000, 5, 0.5, None, FAKE, None, need, None) == 2
+    assert lib.trevs_pre_llm_select(FAKE, FAKE, None, 1000, 5, 0.5, None, FAKE,
+                                    ctypes.c_void_p(0x10010), need, None) == 2
+    assert lib.trevs_in_llm_workspace_size(32, 64, 320) > lib.trevs_in_llm_workspace_size(32, 32, 64)
+
+
+def test_scores_validation(lib):
+    args = lambda N, d, M, zs=4096: (FAKE, zs, N, d, FAKE, 4096, M, FAKE, None, FAKE, None, FAKE, 1 << 24, None)
+    assert lib.trevs_pre_llm_scores(*args(576, 4096, 257)) == t.TREVS_ERR_UNSUPPORTED
+    assert lib.trevs_pre_llm_scores(*args(576, 4100, 32, 4100)) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_pre_llm_scores(*args(576, 4096, 0)) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_pre_llm_scores(*args(576, 4096, 32, 4000)) == t.TREVS_ERR_INVALID_ARGUMENT
+    misaligned = (ctypes.c_void_p(0x10002), 4096, 576, 4096, FAKE, 4096, 32, FAKE, None, FAKE, None, FAKE,
+                  1 << 24, None)
+    assert lib.trevs_pre_llm_scores(*misaligned) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_pre_llm_scores(None, 0, 0, 4096, None, 0, 0, None, None, None, None, None, 0, None) == 0
+
+
+def test_stage2_validation(lib):
+    def hs(Hq, Hkv, L, K1, dh):
+        return lib.trevs_in_llm_head_scores(FAKE, 4096, 128, FAKE, 8192, 128, Hq, Hkv, L, K1, dh, 0.0,
+                                            FAKE, FAKE, FAKE, 1 << 24, None)
+    assert hs(32, 5, 32, 64, 128) == t.TREVS_ERR_INVALID_ARGUMENT      # Hq % Hkv
+    assert hs(32, 32, 32, 64, 64) == t.TREVS_ERR_UNSUPPORTED           # d_h
+    assert hs(32, 32, 32, 4096, 128) == t.TREVS_ERR_UNSUPPORTED        # K1 beyond the limit
+    assert hs(32, 32, 0, 64, 128) == t.TREVS_ERR_INVALID_ARGUMENT      # no text rows
+    assert hs(256, 32, 32, 64, 128) == t.TREVS_ERR_UNSUPPORTED         # Hq
+    sel = lambda nk, K2: lib.trevs_in_llm_select(FAKE, 4096, 128, FAKE, 8192, 128, 32, 32, 32, 64, 128, 0.0,
+                                                 FAKE, FAKE, nk, K2, None, None, FAKE, FAKE, 1 << 24, None)
+    assert sel(0, 32) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert sel(33, 32) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert sel(8, 65) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_in_llm_compact(FAKE, 4096, 4096, None, None, 0, 0, 1, 128, 64, FAKE, 65, FAKE, 4096,
+                                    None, None, 0, 0, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_in_llm_compact(FAKE, 4096, 4096, FAKE, None, 0, 0, 1, 128, 64, FAKE, 32, FAKE, 4096,
+                                    None, None, 0, 0, None) == t.TREVS_ERR_INVALID_ARGUMENT
+
+
+def _pre_batch(reqs, d=4096):
+    arr = (t.PreRequest * len(reqs))(*[t.PreRequest(*r) for r in reqs])
+    b = t.PreBatchC(len(reqs), d, ctypes.cast(arr, ctypes.POINTER(t.PreRequest)), FAKE, d, FAKE, d, FAKE,
+                    None, None, FAKE, None, 0)
+    b._keep = arr
+    return b
+
+
+def test_varlen_validation(lib):
+    ok = _pre_batch([(576, 32, 64, 0.5), (0, 0, 0, 0.5), (1152, 8, 96, 0.25)])
+    need = lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(ok))
+    assert need >= 13 * (576 + 1152)
+    bad = [
+        _pre_batch([(576, 32, 577, 0.5)]),          # k1 > n
+        _pre_batch([(576, 0, 64, 0.5)]),            # no text
+        _pre_batch([(576, 32, 64, -0.1)]),          # ratio
+        _pre_batch([(576, 32, 64, 0.5)], d=100),    # d % 8
+        _pre_batch([(-1, 32, 0, 0.5)]),
+    ]
+    for b in bad:
+        assert lib.trevs_pre_llm_varlen(ctypes.byref(b), None, FAKE, 1 << 30, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_pre_llm_varlen(ctypes.byref(_pre_batch([(576, 300, 64, 0.5)])), None, FAKE, 1 << 30,
+                                    None) == t.TREVS_ERR_UNSUPPORTED
+    assert lib.trevs_pre_llm_varlen(ctypes.byref(ok), None, FAKE, need - 256, None) == t.TREVS_ERR_WORKSPACE
+    empty = t.PreBatchC()
+    assert lib.trevs_pre_llm_varlen(ctypes.byref(empty), None, None, 0, None) == 0
+
+
+def _in_batch(reqs, Hq=32, Hkv=32, nk=8):
+    arr = (t.InRequest * len(reqs))(*[t.InRequest(*r) for r in reqs])
+    b = t.InBatchC()
+    b.B, b.Hq, b.Hkv, b.d_h, b.d_model, b.n_keep_heads = len(reqs), Hq, Hkv, 128, 4096, nk
+    b.reqs = ctypes.cast(arr, ctypes.POINTER(t.InRequest))
+    b.Q, b.q_head_stride, b.q_tok_stride = FAKE, 128, Hq * 128
+    b.K, b.kv_head_stride, b.kv_tok_stride = FAKE, 128, Hkv * 128
+    b.kept_local = FAKE
+    b._keep = arr
+    return b
+
+
+def test_in_varlen_validation(lib):
+    ok = _in_batch([(64, 32, 32), (192, 16, 64)])
+    need = lib.trevs_in_llm_varlen_workspace_size(ctypes.byref(ok))
+    assert need > 0
+    for b in (_in_batch([(64, 32, 65)]), _in_batch([(0, 32, 0)]), _in_batch([(64, 0, 8)]),
+              _in_batch([(64, 32, 8)], Hkv=3), _in_batch([(64, 32, 8)], nk=0), _in_batch([(64, 32, 8)], nk=33)):
+        assert lib.trevs_in_llm_varlen(ctypes.byref(b), FAKE, 1 << 30, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    big = _in_batch([(4096, 32, 8)])
+    assert lib.trevs_in_llm_varlen(ctypes.byref(big), FAKE, 1 << 30, None) == t.TREVS_ERR_UNSUPPORTED
+    half = _in_batch([(64, 32, 8)])
+    half.hidden = FAKE                               # hidden without hidden_out
+    assert lib.trevs_in_llm_varlen(ctypes.byref(half), FAKE, 1 << 30, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    pre = _pre_batch([(576, 32, 64, 0.5)])
+    tot = lib.trevs_prune_varlen_workspace_size(ctypes.byref(pre), ctypes.byref(ok))
+    assert tot >= lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(pre)) + need
+    assert lib.trevs_prune_varlen(ctypes.byref(pre), None, ctypes.byref(ok), FAKE, tot - 256,
+                                  None) == t.TREVS_ERR_WORKSPACE
