@@ -128,7 +128,7 @@ def time_oracle(w, budget_s=12.0, cores=None):
         t0 = time.perf_counter()
         pool.map(_oracle_job, [([b], 1) for b in range(w.B)], chunksize=1)
         per_pass = time.perf_counter() - t0
-        passes = min(50, max(1, int(budget_s / max(1e-3, per_pass))))
+        passes = min(1000, max(1, int(budget_s / max(1e-3, per_pass))))
         jobs = [([b], passes) for b in range(w.B)]
         t0 = time.perf_counter()
         pool.map(_oracle_job, jobs, chunksize=1)
@@ -376,6 +376,22 @@ def reference_arm(args, w):
     }
 
 
+def profile_run(w, launches=5):
+    """Stage-1 scoring + selection of the bench batch, launched eagerly `launches` times."""
+    import torch
+    from paper_2609_37581_gb300 import trevs as T
+    from workloads.device import build_batches
+    T.load()
+    pre, _ = build_batches(w, T.SELECT_RATIO)
+    q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v, kept_idx=pre.kept_idx, s_t=pre.s_t)
+    ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
+    params = T.default_params(T.SELECT_RATIO)
+    for _ in range(launches):
+        T.trevs_pre_llm_varlen(q, ws, params)
+    torch.cuda.synchronize()
+    print(json.dumps({"profile": DOMINANT, "launches": launches}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -383,6 +399,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="only run the dominant kernel a few times (eagerly), for an ncu capture")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -399,6 +417,9 @@ def main():
         return
 
     w = workload()
+    if args.profile:
+        profile_run(w)
+        return
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = time_oracle(w)                     # before any CUDA call: the pool forks safely

@@ -18,7 +18,7 @@
  *     passed as their 16-bit patterns (uint16_t). Rows are addressed through the
  *     strides given (in elements); rows must start on 16-byte boundaries, so
  *     bf16 base pointers must be 16-byte aligned and bf16 strides multiples of 8.
- *   - The library never allocates, frees or synchronises. Every call is
+ *   - The library never allocates or frees, and only trevs_workspace_status synchronises. Every call is
  *     asynchronous on `stream` (a cudaStream_t; NULL = legacy default stream).
  *     Scratch memory comes from a caller-provided workspace of at least the
  *     size the matching *_workspace_size() function returns, 256-byte aligned.
@@ -95,6 +95,12 @@ TREVS_API const char* trevs_last_error_string(void);
 
 /* Number of kernels (and memsets) the last call on this thread enqueued. */
 TREVS_API int32_t trevs_last_launch_count(void);
+
+/* Reads the device status word at the start of a workspace and waits for `stream` to get
+ * there (the one call of this library that synchronises). TREVS_OK, or TREVS_ERR_TIMEOUT
+ * if a bounded device-side wait of a call that used this workspace gave up since the
+ * workspace was last zero-filled. */
+TREVS_API trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* stream);
 
 /* Zero-fills `bytes` of workspace on `stream` (cudaMemsetAsync). */
 TREVS_API trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream);

@@ -10,7 +10,7 @@ notation, with library primitives (matmul, exp, stable sort) as its only
 building blocks and no blocking, fusion or reordering. Inputs arrive as
 bfloat16 bit patterns (uint16) or float32 and are widened exactly to float64.
 
-Readings where the paper is silent (each listed with its reason in the design doc):
+Readings where the paper is silent or leaves a choice open:
   * A zero-norm vector has cosine 0 with everything (Eq. 4 divides by the norm).
   * Med is the lower median: the ascending element of rank floor((N-1)/2) (Eq. 6).
   * epsilon of Eq. 6 defaults to 1e-6.
@@ -195,6 +195,10 @@ def pre_llm_request(Z_bits, T_bits, s_v, k1, ratio, mode="ratio", tau_v=1.4, tau
     Z = bf16_bits_to_f64(Z_bits)
     T = bf16_bits_to_f64(T_bits)
     s_v = np.asarray(s_v, dtype=np.float64)
+    if len(Z) == 0:   # a request without visual tokens has nothing to score or keep
+        empty = np.zeros(0)
+        return {"s_t": empty, "s_fused": empty, "kept": np.zeros(0, np.int64),
+                "Z_out": np.asarray(Z_bits)[:0]}
     s_t = textual_relevance(Z, T)
     out = {"s_t": s_t}
     if mode == "ratio":

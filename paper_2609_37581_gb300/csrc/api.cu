@@ -12,9 +12,11 @@
 #include "trevs.h"
 
 namespace trevs {
-cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, int max_n, cudaStream_t);
+cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, int max_n, long long z_rows,
+                             long long t_rows, cudaStream_t);
 cudaError_t launch_pre_select(const PreMeta&, const PreArgs&, int max_n, cudaStream_t);
-cudaError_t launch_gather(const GatherMeta&, cudaStream_t);
+cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, cudaStream_t);
+cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
@@ -22,7 +24,8 @@ cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cuda
 namespace trevs {
 
 cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes) {
-  if (bytes <= 48 * 1024) return cudaSuccess;
+  // the default limit is 48 KB minus the kernel's static shared memory: always opt in
+  if (bytes <= 0) return cudaSuccess;
   struct Entry {
     const void* kernel;
     int device;
@@ -89,36 +92,44 @@ inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 // ---------------------------------------------------------------- workspace layouts
 
+// Every layout starts with a 256-byte header whose first word is the device status word.
+constexpr size_t kStatusBytes = 256;
+
 struct PreWs {
-  size_t counters, s_t, s_fused, keys, flags, end;
+  size_t counters, sal, s_t, s_fused, keys, flags, end;
 };
 
+// Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request.
 PreWs pre_ws(long long total_n) {
   PreWs w;
-  size_t o = 0;
+  const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
+  size_t o = kStatusBytes;
   w.counters = o; o = al256(o + 4 * (size_t)kMaxChunk);
+  w.sal = o;      o = al256(o + 16 * (size_t)kMaxChunk);
   w.s_t = o;      o = al256(o + 4 * (size_t)total_n);
   w.s_fused = o;  o = al256(o + 4 * (size_t)total_n);
-  w.keys = o;     o = al256(o + 4 * (size_t)total_n);
-  w.flags = o;    o = al256(o + (size_t)total_n);
+  w.keys = o;     o = al256(o + 4 * padded);
+  w.flags = o;    o = al256(o + padded);
   w.end = o;
   return w;
 }
 
 struct InWs {
-  size_t cnt_hs, cnt_ts, row_stats, row_var, u, p, keys, end;
+  size_t cnt_hs, cnt_ts, row_stats, row_var, u, p, keys, flags, end;
 };
 
 InWs in_ws(long long total_l, long long total_k1, int Hq, int B) {
   InWs w;
-  size_t o = 0;
+  size_t o = kStatusBytes;
   w.cnt_hs = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.row_stats = o; o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
   w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
   w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
   w.p = o;         o = al256(o + 4 * (size_t)total_k1);
-  w.keys = o;      o = al256(o + 4 * (size_t)total_k1);
+  const size_t padded = (size_t)total_k1 + 4 * (size_t)kMaxChunk + 4;   // per-request 16-byte alignment
+  w.keys = o;      o = al256(o + 4 * padded);
+  w.flags = o;     o = al256(o + padded);
   w.end = o;
   return w;
 }
@@ -193,10 +204,11 @@ trevs_status validate_params(const trevs_pre_params* p) {
   return TREVS_OK;
 }
 
-// Runs stage 1 for requests [b0, b1) of the batch; offsets are relative to the chunk.
+// Runs stage 1 for requests [b0, b1) of the batch; offsets are relative to the chunk. When
+// `gm_out` is given the gather job is left to the caller (to share one launch with stage 2).
 trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
                            long long n_base, long long m_base, long long k1_base, uint8_t* ws,
-                           const PreWs& L, cudaStream_t st) {
+                           const PreWs& L, cudaStream_t st, GatherMeta* gm_out) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
   meta.B = b1 - b0;
@@ -208,7 +220,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     r.n_off = (int)no; r.n = q.n; r.m_off = (int)mo; r.m = q.m;
     r.k1_off = (int)ko; r.k1 = q.k1; r.kt = textual_count(q.k1, q.ratio);
     r.tile_off = tiles;
-    tiles += (q.n + 63) / 64;
+    tiles += (q.n + kScoreTileRows - 1) / kScoreTileRows;
     no += q.n; mo += q.m; ko += q.k1;
     max_n = q.n > max_n ? q.n : max_n;
     max_m = q.m > max_m ? q.m : max_m;
@@ -224,30 +236,37 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.s_t = (bt->s_t ? bt->s_t : reinterpret_cast<float*>(ws + L.s_t)) + n_base;
   a.s_fused = (bt->s_fused ? bt->s_fused : reinterpret_cast<float*>(ws + L.s_fused)) + n_base;
   a.kept = bt->kept_idx + k1_base;
-  a.flags = ws + L.flags + n_base;
-  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys) + n_base;
+  a.flags = ws + L.flags;
+  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
   a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.sal = reinterpret_cast<int4*>(ws + L.sal);
+  a.sal_ready = 1;
+  a.err = reinterpret_cast<uint32_t*>(ws);
   a.d = bt->d;
   a.mode = prm.select_mode == TREVS_SELECT_FUSED ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
-  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, max_n, st)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, st)), "saliency launch");
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, max_n, no, mo, st)), "pre_score launch");
+  GatherMeta& g = gm_out ? *gm_out : gm;
+  g.njobs = 0;
   if (bt->Z_out && ko > 0) {
-    gm.B = meta.B;
-    gm.njobs = 1;
+    g.njobs = 1;
+    GatherTable& tb = g.t[0];
+    tb.B = meta.B;
     for (int i = 0; i < meta.B; ++i) {
-      gm.dst_off[i] = meta.r[i].k1_off;
-      gm.src_off[i] = meta.r[i].n_off;
-      gm.src_rows[i] = meta.r[i].n;
+      tb.dst_off[i] = meta.r[i].k1_off;
+      tb.src_off[i] = meta.r[i].n_off;
+      tb.src_rows[i] = meta.r[i].n;
     }
-    gm.dst_off[meta.B] = (int)ko;
-    GatherJob& j = gm.job[0];
+    tb.dst_off[meta.B] = (int)ko;
+    GatherJob& j = g.job[0];
     j.src = reinterpret_cast<const uint8_t*>(a.Z);
     j.dst = reinterpret_cast<uint8_t*>(bt->Z_out + k1_base * bt->z_out_row_stride);
     j.src_tok = bt->z_row_stride * 2; j.dst_tok = bt->z_out_row_stride * 2;
     j.src_head = 0; j.dst_head = 0; j.heads = 1; j.row_bytes = bt->d * 2;
-    j.idx = a.kept; j.rows = (int)ko;
-    TREVS_TRY_CUDA(counted(launch_gather(gm, st)), "gather launch");
+    j.idx = a.kept; j.rows = (int)ko; j.tab = 0;
+    if (!gm_out) TREVS_TRY_CUDA(counted(launch_gather(g, st, true)), "gather launch");
   }
   return TREVS_OK;
 }
@@ -257,7 +276,7 @@ trevs_status run_pre_batch(const trevs_pre_batch* bt, const trevs_pre_params& pr
   long long n_base = 0, m_base = 0, k1_base = 0;
   for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
     const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
-    trevs_status s = run_pre_chunk(bt, prm, b0, b1, n_base, m_base, k1_base, ws, L, st);
+    trevs_status s = run_pre_chunk(bt, prm, b0, b1, n_base, m_base, k1_base, ws, L, st, nullptr);
     if (s != TREVS_OK) return s;
     for (int b = b0; b < b1; ++b) {
       n_base += bt->reqs[b].n; m_base += bt->reqs[b].m; k1_base += bt->reqs[b].k1;
@@ -331,23 +350,25 @@ trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
   return TREVS_OK;
 }
 
+// Appends the stage-2 compaction jobs (hidden, K, V rows) to `gm`, offsets in table 1.
 void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden, long long hs, int d_model,
                      uint16_t* hidden_out, long long hos, const uint16_t* K, const uint16_t* V, long long khs,
                      long long kts, int Hkv, uint16_t* K_out, uint16_t* V_out, long long ohs, long long ots,
                      const int* kept, int total_k2) {
-  gm.B = meta.B;
+  GatherTable& tb = gm.t[1];
+  tb.B = meta.B;
   for (int i = 0; i < meta.B; ++i) {
-    gm.dst_off[i] = meta.r[i].k2_off;
-    gm.src_off[i] = meta.r[i].k1_off;
-    gm.src_rows[i] = meta.r[i].k1;
+    tb.dst_off[i] = meta.r[i].k2_off;
+    tb.src_off[i] = meta.r[i].k1_off;
+    tb.src_rows[i] = meta.r[i].k1;
   }
-  gm.dst_off[meta.B] = total_k2;
-  int nj = 0;
+  tb.dst_off[meta.B] = total_k2;
+  int nj = gm.njobs;
   if (hidden) {
     GatherJob& j = gm.job[nj++];
     j.src = reinterpret_cast<const uint8_t*>(hidden); j.dst = reinterpret_cast<uint8_t*>(hidden_out);
     j.src_tok = hs * 2; j.dst_tok = hos * 2; j.src_head = 0; j.dst_head = 0;
-    j.heads = 1; j.row_bytes = d_model * 2; j.idx = kept; j.rows = total_k2;
+    j.heads = 1; j.row_bytes = d_model * 2; j.idx = kept; j.rows = total_k2; j.tab = 1;
   }
   const uint16_t* srcs[2] = {K, V};
   uint16_t* dsts[2] = {K_out, V_out};
@@ -356,15 +377,21 @@ void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden,
     GatherJob& j = gm.job[nj++];
     j.src = reinterpret_cast<const uint8_t*>(srcs[x]); j.dst = reinterpret_cast<uint8_t*>(dsts[x]);
     j.src_tok = kts * 2; j.dst_tok = ots * 2; j.src_head = khs * 2; j.dst_head = ohs * 2;
-    j.heads = Hkv; j.row_bytes = TREVS_HEAD_DIM * 2; j.idx = kept; j.rows = total_k2;
+    j.heads = Hkv; j.row_bytes = TREVS_HEAD_DIM * 2; j.idx = kept; j.rows = total_k2; j.tab = 1;
   }
   gm.njobs = nj;
 }
 
+// Runs stage 2 for requests [b0, b1). `overlap`: the preceding grid of the stream is this
+// library's stage-1 work on unrelated data, so the first kernel need not wait for it.
+// `merged`: gather jobs of stage 1 to launch together with the compaction.
 trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
-                          long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st) {
+                          long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st, bool overlap,
+                          GatherMeta* merged) {
   static thread_local InMeta meta;
-  static thread_local GatherMeta gm;
+  static thread_local GatherMeta gm_own;
+  GatherMeta& gm = merged ? *merged : gm_own;
+  if (!merged) gm.njobs = 0;
   meta.B = b1 - b0;
   int hs = 0, ts = 0, max_k1 = 0;
   long long lo = 0, ko = 0, k2o = 0;
@@ -373,9 +400,9 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     InReq& r = meta.r[b - b0];
     r.l_off = (int)lo; r.l = q.l; r.k1_off = (int)ko; r.k1 = q.k1; r.k2_off = (int)k2o; r.k2 = q.k2;
     r.hs_off = hs; r.ts_off = ts;
-    const int nqb = (q.l + 15) / 16;
+    const int nqb = (q.l + kTextBlockRows - 1) / kTextBlockRows;
     hs += bt->Hq * nqb;
-    ts += nqb * ((q.k1 + 63) / 64);
+    ts += nqb * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
     lo += q.l; ko += q.k1; k2o += q.k2;
     max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
   }
@@ -397,11 +424,13 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.p_bits = (bt->p ? reinterpret_cast<uint32_t*>(bt->p) : reinterpret_cast<uint32_t*>(ws + L.p)) + k1_base;
   a.kept_local = bt->kept_local ? bt->kept_local + k2_base : nullptr;
   a.heads_out = bt->heads ? bt->heads + (long long)b0 * bt->n_keep_heads : nullptr;
-  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys) + k1_base;
+  a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
+  a.flags = ws + L.flags;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + L.cnt_hs);
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + L.cnt_ts);
   a.hs_finalize = 1;
   a.zero_p = 1;
+  a.overlap = overlap ? 1 : 0;
   TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
   TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
   if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
@@ -414,8 +443,8 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
                     bt->Hkv, bt->K_out ? bt->K_out + k2_base * bt->out_tok_stride : nullptr,
                     bt->V_out ? bt->V_out + k2_base * bt->out_tok_stride : nullptr, bt->out_head_stride,
                     bt->out_tok_stride, a.kept_local, (int)k2o);
-    TREVS_TRY_CUDA(counted(launch_gather(gm, st)), "compaction launch");
   }
+  if (gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, true)), "compaction launch");
   return TREVS_OK;
 }
 
@@ -423,7 +452,7 @@ trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, 
   long long l_base = 0, k1_base = 0, k2_base = 0;
   for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
     const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
-    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st);
+    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st, false, nullptr);
     if (s != TREVS_OK) return s;
     for (int b = b0; b < b1; ++b) {
       l_base += bt->reqs[b].l; k1_base += bt->reqs[b].k1; k2_base += bt->reqs[b].k2;
@@ -449,6 +478,16 @@ const char* trevs_version(void) { return "0.1.0"; }
 const char* trevs_last_error_string(void) { return g_err; }
 
 int32_t trevs_last_launch_count(void) { return g_launches; }
+
+trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* stream) {
+  if (!workspace || bytes < sizeof(uint32_t)) return fail(TREVS_ERR_WORKSPACE, "workspace is NULL or too small");
+  uint32_t word = 0;
+  TREVS_TRY_CUDA(cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, (cudaStream_t)stream),
+                 "status read");
+  TREVS_TRY_CUDA(cudaStreamSynchronize((cudaStream_t)stream), "status read");
+  if (word & 1u) return fail(TREVS_ERR_TIMEOUT, "a bounded device-side wait gave up (status word 0x%x)", word);
+  return TREVS_OK;
+}
 
 trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream) {
   g_launches = 0;
@@ -487,7 +526,7 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   static thread_local PreMeta meta;
   meta.B = 1;
   meta.r[0] = PreReq{0, N, 0, M, 0, 0, 0, 0};
-  meta.total_tiles = (N + 63) / 64;
+  meta.total_tiles = (N + kScoreTileRows - 1) / kScoreTileRows;
   PreArgs a;
   memset(&a, 0, sizeof(a));
   a.Z = reinterpret_cast<const __nv_bfloat16*>(Z); a.z_stride = z_row_stride;
@@ -496,10 +535,12 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   a.s_fused = s_fused_out;
   a.flags = ws + L.flags; a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
   a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.sal = reinterpret_cast<int4*>(ws + L.sal);
+  a.err = reinterpret_cast<uint32_t*>(ws);
   a.d = d; a.mode = s_fused_out ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = s_fused_out ? kActScoresFused : kActScores;
-  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, N, M, (cudaStream_t)stream)), "pre_score launch");
   return TREVS_OK;
 }
 
@@ -534,6 +575,8 @@ trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const floa
   a.kept = kept_idx;
   a.flags = ws + L.flags; a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
   a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
+  a.sal = reinterpret_cast<int4*>(ws + L.sal);
+  a.err = reinterpret_cast<uint32_t*>(ws);
   a.mode = fused ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
@@ -553,13 +596,14 @@ trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32
   TREVS_CHECK(z_row_stride >= d && z_row_stride % 8 == 0 && z_out_row_stride >= d && z_out_row_stride % 8 == 0,
               "row strides must be >= d and multiples of 8");
   static thread_local GatherMeta gm;
-  gm.B = 1; gm.njobs = 1;
-  gm.dst_off[0] = 0; gm.dst_off[1] = K1; gm.src_off[0] = 0; gm.src_rows[0] = N;
+  gm.njobs = 1;
+  gm.t[0].B = 1;
+  gm.t[0].dst_off[0] = 0; gm.t[0].dst_off[1] = K1; gm.t[0].src_off[0] = 0; gm.t[0].src_rows[0] = N;
   GatherJob& j = gm.job[0];
   j.src = reinterpret_cast<const uint8_t*>(Z); j.dst = reinterpret_cast<uint8_t*>(Z_out);
   j.src_tok = z_row_stride * 2; j.dst_tok = z_out_row_stride * 2; j.src_head = 0; j.dst_head = 0;
-  j.heads = 1; j.row_bytes = d * 2; j.idx = kept_idx; j.rows = K1;
-  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream)), "gather launch");
+  j.heads = 1; j.row_bytes = d * 2; j.idx = kept_idx; j.rows = K1; j.tab = 0;
+  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream, true)), "gather launch");
   return TREVS_OK;
 }
 
@@ -590,7 +634,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   static thread_local InMeta meta;
   meta.B = 1;
   meta.r[0] = InReq{0, L, 0, K1, 0, 0, 0, 0};
-  meta.total_hs = Hq * ((L + 15) / 16);
+  meta.total_hs = Hq * ((L + kTextBlockRows - 1) / kTextBlockRows);
   meta.total_ts = 0;
   InArgs a;
   memset(&a, 0, sizeof(a));
@@ -635,7 +679,7 @@ trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64
   meta.B = 1;
   meta.r[0] = InReq{0, L, 0, K1, 0, K2, 0, 0};
   meta.total_hs = 0;
-  meta.total_ts = ((L + 15) / 16) * ((K1 + 63) / 64);
+  meta.total_ts = ((L + kTextBlockRows - 1) / kTextBlockRows) * ((K1 + kKeyBlock - 1) / kKeyBlock);
   InArgs a;
   memset(&a, 0, sizeof(a));
   a.Q = reinterpret_cast<const __nv_bfloat16*>(Q); a.q_hs = q_head_stride; a.q_ts = q_tok_stride;
@@ -648,6 +692,7 @@ trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64
   a.p_bits = p_out ? reinterpret_cast<uint32_t*>(p_out) : reinterpret_cast<uint32_t*>(ws + W.p);
   a.kept_local = kept_local; a.heads_out = heads_out;
   a.keys = reinterpret_cast<uint32_t*>(ws + W.keys);
+  a.flags = ws + W.flags;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + W.cnt_ts);
   TREVS_TRY_CUDA(counted(cudaMemsetAsync(a.p_bits, 0, 4 * (size_t)K1, (cudaStream_t)stream)), "p memset");
@@ -689,9 +734,10 @@ trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_str
   static thread_local GatherMeta gm;
   meta.B = 1;
   meta.r[0] = InReq{0, 0, 0, K1, 0, K2, 0, 0};
+  gm.njobs = 0;
   fill_compaction(gm, meta, hidden, hidden_row_stride, d_model, hidden_out, hidden_out_row_stride, Kc, Vc,
                   kv_head_stride, kv_tok_stride, Hkv, K_out, V_out, out_head_stride, out_tok_stride, kept_local, K2);
-  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream)), "compaction launch");
+  TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream, true)), "compaction launch");
   return TREVS_OK;
 }
 
@@ -762,11 +808,19 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   s = check_ws(workspace, workspace_bytes, need);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  const cudaStream_t st = (cudaStream_t)stream;
+  if (pre->B > 0 && in->B > 0 && pre->B <= kMaxChunk && in->B <= kMaxChunk) {
+    // one chunk each: stage 2 overlaps the tail of stage 1, one gather launch for both
+    static thread_local GatherMeta gm;
+    s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, &gm);
+    if (s != TREVS_OK) return s;
+    return run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, true, &gm);
+  }
   if (pre->B > 0) {
-    s = run_pre_batch(pre, prm, ws, LP, (cudaStream_t)stream);
+    s = run_pre_batch(pre, prm, ws, LP, st);
     if (s != TREVS_OK) return s;
   }
-  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, (cudaStream_t)stream);
+  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, st);
   return TREVS_OK;
 }
 

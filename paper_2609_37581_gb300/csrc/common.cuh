@@ -71,7 +71,8 @@ __device__ __forceinline__ float key_to_score(uint32_t k) {
 // ------------------------------------------------------------------ block selection
 
 struct SelShared {
-  uint32_t hist[256];
+  uint32_t hist[2048];
+  uint32_t cand[64];
   uint32_t warp_gt[32];
   uint32_t warp_eq[32];
   uint32_t bcast[4];
@@ -83,68 +84,168 @@ __device__ __forceinline__ uint32_t lanemask_lt() {
   return m;
 }
 
-// K-th largest key (1 <= k <= n) of keys[0..n): returns the key value tau and `need`, the
-// number of entries equal to tau that belong to the top k when ties go to the lower index.
-// All threads of the block must call it; keys may live in shared or global memory.
-__device__ inline void block_kth_largest(const uint32_t* keys, int n, int k, SelShared& s,
-                                         uint32_t& tau, int& need) {
-  uint32_t prefix = 0u, mask = 0u;
-  int kk = k;
-  const int tid = threadIdx.x, nthr = blockDim.x;
-  const int lane = tid & 31, warp = tid >> 5;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = tid; i < 256; i += nthr) s.hist[i] = 0u;
-    __syncthreads();
-    int i = tid;
-    for (; i + 3 * nthr < n; i += 4 * nthr) {
-      uint32_t v0 = keys[i], v1 = keys[i + nthr], v2 = keys[i + 2 * nthr], v3 = keys[i + 3 * nthr];
-      if ((v0 & mask) == prefix) atomicAdd(&s.hist[(v0 >> shift) & 255u], 1u);
-      if ((v1 & mask) == prefix) atomicAdd(&s.hist[(v1 >> shift) & 255u], 1u);
-      if ((v2 & mask) == prefix) atomicAdd(&s.hist[(v2 >> shift) & 255u], 1u);
-      if ((v3 & mask) == prefix) atomicAdd(&s.hist[(v3 >> shift) & 255u], 1u);
-    }
-    for (; i < n; i += nthr) {
-      uint32_t v = keys[i];
-      if ((v & mask) == prefix) atomicAdd(&s.hist[(v >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (warp == 0) {
-      // lane l owns bins [255 - 8l - 7, 255 - 8l], scanned from the top
-      uint32_t c[8];
-      uint32_t tot = 0;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) { c[j] = s.hist[255 - 8 * lane - j]; tot += c[j]; }
-      uint32_t incl = tot;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      uint32_t excl = incl - tot;
-      bool here = (excl < (uint32_t)kk) && (incl >= (uint32_t)kk);
-      uint32_t ballot = __ballot_sync(0xffffffffu, here);
-      int owner = __ffs(ballot) - 1;
-      if (lane == owner) {
-        uint32_t cum = excl;
-        int j = 0;
-        for (; j < 7; ++j) {
-          if (cum + c[j] >= (uint32_t)kk) break;
-          cum += c[j];
-        }
-        s.bcast[0] = 255u - 8u * lane - j;
-        s.bcast[1] = (uint32_t)kk - cum;
-      }
-    }
-    __syncthreads();
-    uint32_t bin = s.bcast[0];
-    kk = (int)s.bcast[1];
-    prefix |= bin << shift;
-    mask |= 255u << shift;
-    __syncthreads();
+// One radix pass of the block selection: histogram of digit ((w >> sh) & (nb - 1)) over the
+// entries whose offset w = key - lo satisfies (w & pmask) == pval, then the digit holding
+// the kk-th largest of them. Writes (digit, rank within the digit) to s.bcast[0..1].
+// keys must be 16-byte aligned.
+__device__ inline void radix_pass(const uint32_t* keys, int n, uint32_t lo, uint32_t pmask, uint32_t pval,
+                                  int sh, uint32_t nb, int kk, SelShared& s) {
+  const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < (int)nb; i += nthr) s.hist[i] = 0u;
+  __syncthreads();
+  auto count = [&](uint32_t v) {
+    const uint32_t w = v - lo;
+    if (v != 0u && (w & pmask) == pval) atomicAdd(&s.hist[(w >> sh) & (nb - 1u)], 1u);
+  };
+  const int n4 = n >> 2;
+  const uint4* k4 = reinterpret_cast<const uint4*>(keys);
+  for (int j = tid; j < n4; j += nthr) {
+    const uint4 v = k4[j];
+    count(v.x);
+    count(v.y);
+    count(v.z);
+    count(v.w);
   }
-  tau = prefix;
-  need = kk;
+  for (int i = 4 * n4 + tid; i < n; i += nthr) count(keys[i]);
+  __syncthreads();
+  // bin scan from the top: thread t < nscan owns bins [nb - (t+1)*per, nb - t*per)
+  int nscan = 1;   // a power of two <= min(threads, bins, 256)
+  while (nscan * 2 <= nthr && nscan * 2 <= (int)nb && nscan < 256) nscan *= 2;
+  const int per = (int)nb / nscan;
+  uint32_t tot = 0;
+  if (tid < nscan)
+    for (int j = 0; j < per; ++j) tot += s.hist[nb - 1 - (uint32_t)(tid * per + j)];
+  uint32_t incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (tid < nscan && lane == 31) s.warp_gt[warp] = incl;
+  __syncthreads();
+  if (tid < nscan) {
+    uint32_t off = 0;
+    for (int w = 0; w < warp; ++w) off += s.warp_gt[w];
+    incl += off;
+    const uint32_t excl = incl - tot;
+    if (excl < (uint32_t)kk && incl >= (uint32_t)kk) {
+      uint32_t cum = excl;
+      int j = 0;
+      for (; j < per - 1; ++j) {
+        const uint32_t c = s.hist[nb - 1 - (uint32_t)(tid * per + j)];
+        if (cum + c >= (uint32_t)kk) break;
+        cum += c;
+      }
+      s.bcast[0] = nb - 1 - (uint32_t)(tid * per + j);
+      s.bcast[1] = (uint32_t)kk - cum;
+    }
+  }
+  __syncthreads();
 }
+
+// K-th largest key (1 <= k <= number of non-zero keys) of keys[0..n); a key of 0 marks an
+// excluded entry (no float maps to it). Returns the key value tau, `need`, the
+// number of entries equal to tau that belong to the top k when ties go to the lower index,
+// and `n_eq`, the number of entries equal to tau (need == n_eq: the top k are exactly the
+// entries >= tau). [lo, hi] is the key range from block_fill_keys; keys 16-byte aligned.
+// Radix select on the offsets w = key - min(keys): the first digit is the
+// top 11 bits of the occupied range, so scores clustered in a narrow band still spread
+// over the bins; when the chosen bin holds at most 64 entries one warp finishes by ranking
+// them, otherwise further 11-bit passes count only the entries still in the running.
+// All threads of the block (a multiple of 32) must call it; keys may live in shared or
+// global memory.
+__device__ inline void block_kth_largest(const uint32_t* keys, int n, int k, SelShared& s, uint32_t lo,
+                                         uint32_t hi, uint32_t& tau, int& need, int& n_eq) {
+  const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  if (lo >= hi) {   // every candidate key equal (or none): the first k of them
+    tau = lo == hi ? lo : 0xFFFFFFFFu;
+    need = k;
+    n_eq = n;
+    return;
+  }
+  const uint32_t range = hi - lo;
+  const int bits = 32 - __clz(range);            // bits of the largest offset
+  int sh = bits > 11 ? bits - 11 : 0;            // first digit: offset bits [sh, bits)
+  uint32_t nb = 1u << (bits - sh);
+  uint32_t pmask = 0u, pval = 0u;
+  int kk = k;
+  while (true) {
+    radix_pass(keys, n, lo, pmask, pval, sh, nb, kk, s);
+    const uint32_t dig = s.bcast[0];
+    const uint32_t cnt = s.hist[dig];            // entries still in the running
+    kk = (int)s.bcast[1];
+    pval |= dig << sh;
+    pmask |= (nb - 1u) << sh;
+    __syncthreads();
+    if (sh == 0) {                               // every remaining entry equals tau
+      tau = lo + pval;
+      need = kk;
+      n_eq = (int)cnt;
+      return;
+    }
+    if (cnt <= 64u) {
+      // gather the candidates; one warp ranks them pairwise
+      if (tid == 0) s.bcast[2] = 0u;
+      __syncthreads();
+      auto gather = [&](uint32_t v, bool valid) {
+        const bool in = valid && v != 0u && ((v - lo) & pmask) == pval;
+        const uint32_t bal = __ballot_sync(0xffffffffu, in);
+        if (bal) {
+          uint32_t at = 0;
+          if (lane == 0) at = atomicAdd(&s.bcast[2], (uint32_t)__popc(bal));
+          at = __shfl_sync(0xffffffffu, at, 0);
+          if (in) s.cand[at + __popc(bal & lanemask_lt())] = v;
+        }
+      };
+      const int n4 = n >> 2;
+      const uint4* k4 = reinterpret_cast<const uint4*>(keys);
+      for (int base = 0; base < n4; base += nthr) {
+        const int j = base + tid;
+        const uint4 v = j < n4 ? k4[j] : make_uint4(0u, 0u, 0u, 0u);
+        gather(v.x, j < n4);
+        gather(v.y, j < n4);
+        gather(v.z, j < n4);
+        gather(v.w, j < n4);
+      }
+      {
+        const int i = 4 * n4 + tid;
+        gather(i < n ? keys[i] : 0u, i < n);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        for (int c = lane; c < (int)cnt; c += 32) {
+          const uint32_t mine = s.cand[c];
+          int gt = 0, eq = 0;
+          for (int j = 0; j < (int)cnt; ++j) {
+            const uint32_t o = s.cand[j];
+            gt += o > mine;
+            eq += o == mine;
+          }
+          if (gt < kk && kk <= gt + eq) {        // equal candidates write equal values
+            s.bcast[0] = mine;
+            s.bcast[1] = (uint32_t)(kk - gt);
+            s.bcast[3] = (uint32_t)eq;
+          }
+        }
+      }
+      __syncthreads();
+      tau = s.bcast[0];
+      need = (int)s.bcast[1];
+      n_eq = (int)s.bcast[3];
+      __syncthreads();
+      return;
+    }
+    const int nbits = sh > 11 ? 11 : sh;
+    sh -= nbits;
+    nb = 1u << nbits;
+  }
+}
+
+// flags[i] |= 1 for the entries of the top k described by (tau, need, n_eq). When every
+// entry equal to tau belongs (need == n_eq) this is element-wise; otherwise the ties go to
+// the lower indices by an ordered pass.
+__device__ inline void block_mark_selected(const uint32_t* keys, int n, uint32_t tau, int need, int n_eq,
+                                           uint8_t* flags, SelShared& s);
 
 // Visits, in ascending index order, every i selected by (tau, need):
 // keys[i] > tau, or keys[i] == tau among the first `need` such indices.
@@ -187,29 +288,63 @@ __device__ inline void block_emit_selected(const uint32_t* keys, int n, uint32_t
 }
 
 // Ordered compaction of a 0/1 byte mask: out[pos] = i for every flagged i, ascending.
+// Each warp owns a contiguous segment and walks it 128 entries at a time.
 __device__ inline void block_compact_flags(const uint8_t* flags, int n, int* out, SelShared& s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   int seg = (n + nwarps - 1) / nwarps;
-  seg = (seg + 31) & ~31;
+  seg = (seg + 127) & ~127;
   const int beg = min(n, warp * seg), end = min(n, beg + seg);
   uint32_t cnt = 0;
-  for (int base = beg; base < end; base += 32) {
-    int i = base + lane;
-    cnt += __popc(__ballot_sync(0xffffffffu, i < end && flags[i] != 0));
+  for (int base = beg; base < end; base += 128) {
+    bool f[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = base + 32 * q + lane;
+      f[q] = i < end && flags[i] != 0;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) cnt += __popc(__ballot_sync(0xffffffffu, f[q]));
   }
   if (lane == 0) s.warp_gt[warp] = cnt;
   __syncthreads();
   uint32_t run = 0;
   for (int w = 0; w < warp; ++w) run += s.warp_gt[w];
   const uint32_t lt = lanemask_lt();
-  for (int base = beg; base < end; base += 32) {
-    int i = base + lane;
-    bool f = i < end && flags[i] != 0;
-    uint32_t b = __ballot_sync(0xffffffffu, f);
-    if (f) out[run + __popc(b & lt)] = i;
-    run += __popc(b);
+  for (int base = beg; base < end; base += 128) {
+    bool f[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = base + 32 * q + lane;
+      f[q] = i < end && flags[i] != 0;
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t b = __ballot_sync(0xffffffffu, f[q]);
+      if (f[q]) out[run + __popc(b & lt)] = base + 32 * q + lane;
+      run += __popc(b);
+    }
   }
   __syncthreads();
+}
+
+__device__ inline void block_mark_selected(const uint32_t* keys, int n, uint32_t tau, int need, int n_eq,
+                                           uint8_t* flags, SelShared& s) {
+  if (need >= n_eq) {
+    const int n4 = n >> 2;
+    const uint4* k4 = reinterpret_cast<const uint4*>(keys);
+    for (int j = threadIdx.x; j < n4; j += blockDim.x) {
+      const uint4 v = k4[j];
+      if (v.x >= tau) flags[4 * j] = 1;
+      if (v.y >= tau) flags[4 * j + 1] = 1;
+      if (v.z >= tau) flags[4 * j + 2] = 1;
+      if (v.w >= tau) flags[4 * j + 3] = 1;
+    }
+    for (int i = 4 * n4 + threadIdx.x; i < n; i += blockDim.x)
+      if (keys[i] >= tau) flags[i] = 1;
+    __syncthreads();
+    return;
+  }
+  block_emit_selected(keys, n, tau, need, s, [&](int i, int, bool sel) { if (sel) flags[i] = 1; });
 }
 
 // ------------------------------------------------------------------ launch helpers
@@ -221,6 +356,29 @@ cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes);
 template <class Kernel>
 inline cudaError_t ensure_dynamic_smem(Kernel kernel, int bytes) {
   return ensure_dynamic_smem_impl(reinterpret_cast<const void*>(kernel), bytes);
+}
+
+// Programmatic dependent launch: wait for the preceding grid of the stream (no-op when
+// there is none), and let the next grid of the stream start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Launches `kernel`, optionally allowed to start before the preceding work of the stream
+// completes (it must then call pdl_wait() before it touches that work's results).
+template <class... KArgs, class... Args>
+inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                 bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = pdl ? attr : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 // ------------------------------------------------------------------ PTX wrappers
@@ -251,6 +409,130 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const uint32_t* a, uint
       "{%0,%1,%2,%3};\n"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// acc[0..3] += squares of the eight bf16 values in v (four independent chains).
+__device__ __forceinline__ void bf16_sq_acc8(uint4 v, float (&acc)[4]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float lo = __uint_as_float(w[j] << 16), hi = __uint_as_float(w[j] & 0xFFFF0000u);
+    acc[j] = fmaf(lo, lo, acc[j]);
+    acc[j] = fmaf(hi, hi, acc[j]);
+  }
+}
+
+// Block-wide min of the non-zero keys and max of all keys (key 0 marks an excluded entry).
+__device__ inline void block_key_range(uint32_t lo, uint32_t hi, SelShared& s, uint32_t& lo_out, uint32_t& hi_out) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    lo = min(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = max(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  if (lane == 0) { s.warp_gt[warp] = lo; s.warp_eq[warp] = hi; }
+  __syncthreads();
+  lo = 0xFFFFFFFFu;
+  hi = 0u;
+  for (int w = 0; w < nwarps; ++w) { lo = min(lo, s.warp_gt[w]); hi = max(hi, s.warp_eq[w]); }
+  __syncthreads();
+  lo_out = lo;
+  hi_out = hi;
+}
+
+// keys[i] = f(src[i], i) for i < n by the whole block, also returning the key range
+// (min over non-zero keys, max over all). 16-byte loads through L2 (the values may have
+// been written by other blocks of the grid), eight in flight per thread.
+template <class F>
+__device__ inline void block_fill_keys(uint32_t* keys, const float* src, int n, F f, SelShared& s, uint32_t& lo,
+                                       uint32_t& hi) {
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  uint32_t l = 0xFFFFFFFFu, h = 0u;
+  auto put = [&](int i, float x) {
+    const uint32_t k = f(x, i);
+    keys[i] = k;
+    if (k != 0u) l = min(l, k);
+    h = max(h, k);
+  };
+  const int head = min(n, (int)(((16u - ((uint32_t)reinterpret_cast<uintptr_t>(src) & 15u)) & 15u) >> 2));
+  if (tid < head) put(tid, __ldcg(src + tid));
+  const float4* v = reinterpret_cast<const float4*>(src + head);
+  const int nv = (n - head) >> 2;
+  int j = tid;
+  for (; j + 7 * nthr < nv; j += 8 * nthr) {
+    float4 x[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) x[q] = __ldcg(v + j + q * nthr);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int i = head + 4 * (j + q * nthr);
+      put(i, x[q].x);
+      put(i + 1, x[q].y);
+      put(i + 2, x[q].z);
+      put(i + 3, x[q].w);
+    }
+  }
+  for (; j < nv; j += nthr) {
+    const float4 x = __ldcg(v + j);
+    const int i = head + 4 * j;
+    put(i, x.x);
+    put(i + 1, x.y);
+    put(i + 2, x.z);
+    put(i + 3, x.w);
+  }
+  for (int i = head + 4 * nv + tid; i < n; i += nthr) put(i, __ldcg(src + i));
+  block_key_range(l, h, s, lo, hi);   // synchronises: keys are complete afterwards
+}
+
+// keys[i] = f(a[i], b[i], i) for i < n by the whole block, returning the key range. Both
+// sources are read with 16-byte loads when they share their alignment.
+template <class F>
+__device__ inline void block_fill_keys2(uint32_t* keys, const float* a, const float* b, int n, F f, SelShared& s,
+                                        uint32_t& lo, uint32_t& hi) {
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  uint32_t l = 0xFFFFFFFFu, h = 0u;
+  auto put = [&](int i, float x, float y) {
+    const uint32_t k = f(x, y, i);
+    keys[i] = k;
+    if (k != 0u) l = min(l, k);
+    h = max(h, k);
+  };
+  const uint32_t ma = (uint32_t)reinterpret_cast<uintptr_t>(a) & 15u, mb = (uint32_t)reinterpret_cast<uintptr_t>(b) & 15u;
+  int head = n, nv = 0;
+  if (ma == mb) {
+    head = min(n, (int)(((16u - ma) & 15u) >> 2));
+    nv = (n - head) >> 2;
+  }
+  for (int i = tid; i < head; i += nthr) put(i, __ldcg(a + i), __ldcg(b + i));
+  const float4* va = reinterpret_cast<const float4*>(a + head);
+  const float4* vb = reinterpret_cast<const float4*>(b + head);
+  int j = tid;
+  for (; j + 3 * nthr < nv; j += 4 * nthr) {
+    float4 x[4], y[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      x[q] = __ldcg(va + j + q * nthr);
+      y[q] = __ldcg(vb + j + q * nthr);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = head + 4 * (j + q * nthr);
+      put(i, x[q].x, y[q].x);
+      put(i + 1, x[q].y, y[q].y);
+      put(i + 2, x[q].z, y[q].z);
+      put(i + 3, x[q].w, y[q].w);
+    }
+  }
+  for (; j < nv; j += nthr) {
+    const float4 x = __ldcg(va + j), y = __ldcg(vb + j);
+    const int i = head + 4 * j;
+    put(i, x.x, y.x);
+    put(i + 1, x.y, y.y);
+    put(i + 2, x.z, y.z);
+    put(i + 3, x.w, y.w);
+  }
+  for (int i = head + 4 * nv + tid; i < n; i += nthr) put(i, __ldcg(a + i), __ldcg(b + i));
+  block_key_range(l, h, s, lo, hi);
 }
 
 __device__ __forceinline__ float bf16_sq_sum8(uint4 v) {

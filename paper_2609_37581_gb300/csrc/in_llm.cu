@@ -4,8 +4,8 @@
 
 namespace trevs {
 
-constexpr int kQB = 16;        // text rows per block (one m16 tile)
-constexpr int kKB = 64;        // visual keys per shared-memory chunk
+constexpr int kQB = kTextBlockRows;
+constexpr int kKB = kKeyBlock;
 constexpr int kDh = 128;       // head width
 constexpr int kRowBytes = kDh * 2;
 
@@ -59,6 +59,8 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
                                                             const InArgs a, int k1_ld) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_last;
+  if (!a.overlap) pdl_wait();   // Q, K may come from the preceding grid
+  pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
   const InReq r = meta.r[b];
@@ -132,6 +134,8 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
     }
   }
 
+  // completion of this grid implies completion of the preceding one
+  if (a.overlap) pdl_wait();
   if (!a.hs_finalize) return;
   __threadfence();
   __syncthreads();
@@ -168,6 +172,8 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
   __shared__ int s_heads[kMaxHeads];
   __shared__ int s_sel[kMaxHeads];
   __shared__ int s_nh, s_last;
+  pdl_wait();   // u, row statistics and the cleared p come from the preceding grid
+  pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].ts_off; });
   const InReq r = meta.r[b];
@@ -265,15 +271,18 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
     for (int x = tid; x < s_nh; x += 128) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
   if (r.k2 <= 0) return;
   const int n = r.k1;
-  const bool in_smem = (size_t)n * 4 <= (size_t)smem_bytes;
-  uint32_t* keys = in_smem ? reinterpret_cast<uint32_t*>(smem) : a.keys + r.k1_off;
-  for (int i = tid; i < n; i += 128) keys[i] = score_key(__uint_as_float(__ldcg(a.p_bits + r.k1_off + i)));
-  __syncthreads();
-  uint32_t tau;
-  int need;
-  block_kth_largest(keys, n, r.k2, ss, tau, need);
-  int* out = a.kept_local + r.k2_off;
-  block_emit_selected(keys, n, tau, need, ss, [&](int i, int pos, bool sel) { if (sel) out[pos] = i; });
+  const bool in_smem = (size_t)n * 5 <= (size_t)smem_bytes;
+  const size_t gbase = ((size_t)r.k1_off + 4 * (size_t)b + 3) & ~(size_t)3;   // 16-byte aligned
+  uint32_t* keys = in_smem ? reinterpret_cast<uint32_t*>(smem) : a.keys + gbase;
+  uint8_t* flags = in_smem ? smem + (size_t)n * 4 : a.flags + gbase;
+  for (int i = tid; i < n; i += 128) flags[i] = 0;
+  uint32_t lo, hi, tau;
+  int need, n_eq;
+  block_fill_keys(keys, reinterpret_cast<const float*>(a.p_bits + r.k1_off), n,
+                  [&](float x, int) { return score_key(x); }, ss, lo, hi);
+  block_kth_largest(keys, n, r.k2, ss, lo, hi, tau, need, n_eq);
+  block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+  block_compact_flags(flags, n, a.kept_local + r.k2_off, ss);
 }
 
 // ------------------------------------------------------------------ host-side launchers
@@ -286,18 +295,16 @@ cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_k1
   const int smem = kQB * kRowBytes + 2 * kKB * kRowBytes + kQB * ld * 4;
   cudaError_t e = ensure_dynamic_smem(in_head_stats_kernel, smem);
   if (e != cudaSuccess) return e;
-  in_head_stats_kernel<<<meta.total_hs, 128, smem, st>>>(meta, a, ld);
-  return cudaGetLastError();
+  return launch_kernel(in_head_stats_kernel, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
 }
 
 cudaError_t launch_in_token_score(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
   if (meta.total_ts == 0) return cudaSuccess;
   int smem = kQB * kRowBytes + kKB * kRowBytes;
-  if (max_k1 * 4 > smem) smem = max_k1 * 4;
+  if (max_k1 * 5 > smem) smem = max_k1 * 5;
   cudaError_t e = ensure_dynamic_smem(in_token_score_kernel, smem);
   if (e != cudaSuccess) return e;
-  in_token_score_kernel<<<meta.total_ts, 128, smem, st>>>(meta, a, smem);
-  return cudaGetLastError();
+  return launch_kernel(in_token_score_kernel, dim3(meta.total_ts), dim3(128), smem, st, true, meta, a, smem);
 }
 
 }  // namespace trevs

@@ -6,6 +6,8 @@
 namespace trevs {
 
 constexpr int kMaxHeads = 128;
+constexpr int kTextBlockRows = 16;   // text rows per stage-2 block (one m16 tile)
+constexpr int kKeyBlock = 64;        // visual keys per stage-2 block / shared-memory chunk
 
 struct InArgs {
   const __nv_bfloat16* Q;
@@ -23,10 +25,12 @@ struct InArgs {
   int* kept_local;          // [sum k2]
   int* heads_out;           // [B][n_keep] or null
   uint32_t* keys;           // [sum k1] selection scratch
+  uint8_t* flags;           // [sum k1] selection scratch
   uint32_t* cnt_hs;         // [B] self-resetting tickets
   uint32_t* cnt_ts;         // [B]
   int hs_finalize;          // head-statistics blocks reduce u (ticket)
   int zero_p;               // ... and clear p for the token-score pass
+  int overlap;              // head statistics need not wait for the preceding grid at start
 };
 
 }  // namespace trevs

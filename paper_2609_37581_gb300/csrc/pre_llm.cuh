@@ -7,6 +7,8 @@
 namespace trevs {
 
 enum { kModeRatio = 0, kModeFused = 1 };
+
+constexpr int kScoreTileRows = 128;   // visual rows per scoring CTA (UMMA M)
 enum { kActScores = 0, kActScoresFused = 1, kActSelect = 2 };
 
 struct PreArgs {
@@ -21,6 +23,9 @@ struct PreArgs {
   uint8_t* flags;      // [sum n] scratch
   uint32_t* keys;      // [sum n] scratch (used when shared memory is too small)
   uint32_t* counters;  // [B] tiles finished per request (self-resetting)
+  int4* sal;           // [B] saliency side of the selection (see saliency_prepare)
+  int sal_ready;       // 1: sal was filled by the saliency kernel earlier in the stream
+  uint32_t* err;       // device status word: bit 0 = a bounded wait gave up
   int d;
   int mode;
   float tau_v, tau_t, lambda, eps;
@@ -28,42 +33,83 @@ struct PreArgs {
   int s_fused_given;   // select kernel: s_fused already holds Eq. 7 scores
 };
 
-// Selection for one request by the whole block (any multiple of 32 threads).
-__device__ inline void select_request(const PreArgs& a, const PreReq& r, uint8_t* smem,
-                                      int smem_bytes, SelShared& ss, bool compute_fused,
-                                      bool do_select) {
+// Saliency side of the selection, which depends on inputs only. Ratio mode: the rule for
+// S_v = the K_v tokens of largest s_v, as (tau, need, n_eq, cut): token i is in S_v iff
+// key(s_v[i]) > tau, or key == tau and (need >= n_eq or i <= cut). Fused mode: Med and MAD
+// of s_v (Eq. 6) as float bits in .x and .y. `keys` holds n entries, 16-byte aligned.
+__device__ inline int4 saliency_prepare(const PreArgs& a, const PreReq& r, uint32_t* keys, SelShared& ss) {
+  const int n = r.n;
+  const float* sv = a.s_v + r.n_off;
+  uint32_t lo, hi, tau;
+  int need, n_eq;
+  if (a.mode == kModeRatio) {
+    const int kv = r.k1 - r.kt;
+    if (kv <= 0 || n <= 0) return make_int4(-1, 0, 1, -1);   // empty: nothing passes the rule
+    block_fill_keys(keys, sv, n, [&](float x, int) { return score_key(x); }, ss, lo, hi);
+    block_kth_largest(keys, n, kv, ss, lo, hi, tau, need, n_eq);
+    int cut = -1;
+    if (need < n_eq) {   // ties at the threshold: the need-th equal key in index order
+      if (threadIdx.x == 0) ss.bcast[3] = 0u;
+      __syncthreads();
+      block_emit_selected(keys, n, tau, need, ss, [&](int i, int, bool sel) {
+        if (sel && keys[i] == tau) atomicMax(&ss.bcast[3], (uint32_t)i);
+      });
+      cut = (int)ss.bcast[3];
+      __syncthreads();
+    }
+    return make_int4((int)tau, need, n_eq, cut);
+  }
+  if (n <= 0) return make_int4(0, 0, 0, 0);
+  const int kmed = n - (n - 1) / 2;  // lower median = kmed-th largest
+  block_fill_keys(keys, sv, n, [&](float x, int) { return score_key(x); }, ss, lo, hi);
+  block_kth_largest(keys, n, kmed, ss, lo, hi, tau, need, n_eq);
+  const float med = key_to_score(tau);
+  block_fill_keys(keys, sv, n, [&](float x, int) { return score_key(fabsf(x - med)); }, ss, lo, hi);
+  block_kth_largest(keys, n, kmed, ss, lo, hi, tau, need, n_eq);
+  return make_int4(__float_as_int(med), __float_as_int(key_to_score(tau)), 0, 0);
+}
+
+__device__ __forceinline__ bool in_saliency_set(float sv, int i, int4 rule) {
+  const uint32_t k = score_key(sv), tau = (uint32_t)rule.x;
+  return k > tau || (k == tau && (rule.y >= rule.z || i <= rule.w));
+}
+
+// Selection for one request by the whole block (any multiple of 32 threads). `b` is the
+// request's slot in the launch; `sal` is its saliency rule when already prepared.
+__device__ inline void select_request(const PreArgs& a, const PreReq& r, int b, uint8_t* smem, int smem_bytes,
+                                      SelShared& ss, bool compute_fused, bool do_select) {
   const int n = r.n;
   if (n <= 0) return;
   const int tid = threadIdx.x, nthr = blockDim.x;
   const float* sv = a.s_v + r.n_off;
   const float* st = a.s_t + r.n_off;
   const bool in_smem = (size_t)n * 5 + 16 <= (size_t)smem_bytes;
-  uint32_t* keys = in_smem ? reinterpret_cast<uint32_t*>(smem) : a.keys + r.n_off;
-  uint8_t* flags = in_smem ? smem + (size_t)n * 4 : a.flags + r.n_off;
+  // global fallback: request b's scratch starts at a 16-byte boundary inside [sum n + 4B]
+  const size_t gbase = ((size_t)r.n_off + 4 * (size_t)b + 3) & ~(size_t)3;
+  uint32_t* keys = in_smem ? reinterpret_cast<uint32_t*>(smem) : a.keys + gbase;
+  uint8_t* flags = in_smem ? smem + (size_t)n * 4 : a.flags + gbase;
   int* out = a.kept + r.k1_off;
-  uint32_t tau;
-  int need;
+  uint32_t lo, hi, tau;
+  int need, n_eq;
+  int4 rule = make_int4(-1, 0, 1, -1);
+  if (a.sal_ready) {
+    pdl_wait();   // the saliency kernel precedes this grid in the stream
+    rule = __ldcg(a.sal + b);
+  } else if (a.mode == kModeRatio || compute_fused) {
+    rule = saliency_prepare(a, r, keys, ss);
+  }
 
   if (a.mode == kModeRatio) {
     if (!do_select) return;
-    const int kv = r.k1 - r.kt, kt = r.kt;
-    if (kv > 0) {
-      for (int i = tid; i < n; i += nthr) keys[i] = score_key(__ldcg(sv + i));
-      __syncthreads();
-      block_kth_largest(keys, n, kv, ss, tau, need);
-      block_emit_selected(keys, n, tau, need, ss,
-                          [&](int i, int, bool sel) { flags[i] = sel ? 1 : 0; });
-    } else {
-      for (int i = tid; i < n; i += nthr) flags[i] = 0;
-      __syncthreads();
-    }
-    if (kt > 0) {
-      // tokens already kept by saliency get key 0, below every finite score
-      for (int i = tid; i < n; i += nthr) keys[i] = flags[i] ? 0u : score_key(__ldcg(st + i));
-      __syncthreads();
-      block_kth_largest(keys, n, kt, ss, tau, need);
-      block_emit_selected(keys, n, tau, need, ss,
-                          [&](int i, int, bool sel) { if (sel) flags[i] = 1; });
+    // S_v from its rule; the textual keys exclude it (key 0)
+    block_fill_keys2(keys, st, sv, n, [&](float x, float v, int i) {
+      const bool in_v = in_saliency_set(v, i, rule);
+      flags[i] = in_v ? 1 : 0;
+      return in_v ? 0u : score_key(x);
+    }, ss, lo, hi);
+    if (r.kt > 0) {
+      block_kth_largest(keys, n, r.kt, ss, lo, hi, tau, need, n_eq);
+      block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
     }
     block_compact_flags(flags, n, out, ss);
     return;
@@ -73,20 +119,13 @@ __device__ inline void select_request(const PreArgs& a, const PreReq& r, uint8_t
   float* sf = a.s_fused + r.n_off;
   if (compute_fused) {
     const int kmed = n - (n - 1) / 2;  // lower median = kmed-th largest
-    // Med and MAD of one signal by two order-statistic selections
-    auto med_mad = [&](const float* s, float& med, float& mad) {
-      for (int i = tid; i < n; i += nthr) keys[i] = score_key(__ldcg(s + i));
-      __syncthreads();
-      block_kth_largest(keys, n, kmed, ss, tau, need);
-      med = key_to_score(tau);
-      for (int i = tid; i < n; i += nthr) keys[i] = score_key(fabsf(__ldcg(s + i) - med));
-      __syncthreads();
-      block_kth_largest(keys, n, kmed, ss, tau, need);
-      mad = key_to_score(tau);
-    };
-    float med_v, mad_v, med_t, mad_t;
-    med_mad(sv, med_v, mad_v);
-    med_mad(st, med_t, mad_t);
+    const float med_v = __int_as_float(rule.x), mad_v = __int_as_float(rule.y);
+    block_fill_keys(keys, st, n, [&](float x, int) { return score_key(x); }, ss, lo, hi);
+    block_kth_largest(keys, n, kmed, ss, lo, hi, tau, need, n_eq);
+    const float med_t = key_to_score(tau);
+    block_fill_keys(keys, st, n, [&](float x, int) { return score_key(fabsf(x - med_t)); }, ss, lo, hi);
+    block_kth_largest(keys, n, kmed, ss, lo, hi, tau, need, n_eq);
+    const float mad_t = key_to_score(tau);
     const float dv = mad_v + a.eps, dt = mad_t + a.eps;
     for (int i = tid; i < n; i += nthr) {
       float hv = fmaxf((__ldcg(sv + i) - med_v) / dv, 0.f) / a.tau_v;
@@ -96,11 +135,11 @@ __device__ inline void select_request(const PreArgs& a, const PreReq& r, uint8_t
     __syncthreads();
   }
   if (do_select && r.k1 > 0) {
-    for (int i = tid; i < n; i += nthr) keys[i] = score_key(__ldcg(sf + i));
-    __syncthreads();
-    block_kth_largest(keys, n, r.k1, ss, tau, need);
-    block_emit_selected(keys, n, tau, need, ss,
-                        [&](int i, int pos, bool sel) { if (sel) out[pos] = i; });
+    for (int i = tid; i < n; i += nthr) flags[i] = 0;
+    block_fill_keys(keys, sf, n, [&](float x, int) { return score_key(x); }, ss, lo, hi);
+    block_kth_largest(keys, n, r.k1, ss, lo, hi, tau, need, n_eq);
+    block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+    block_compact_flags(flags, n, out, ss);
   }
 }
 
@@ -115,15 +154,20 @@ struct GatherJob {
   int row_bytes;                 // per (row, head), multiple of 16
   const int* idx;                // request-local source row of each destination row
   int rows;                      // destination rows (all requests)
-  int pad_;
+  int tab;                       // offset table of the job's requests
 };
 
-struct GatherMeta {
+// Per-request row offsets of one family of gathers (stage-1 rows or stage-2 rows).
+struct GatherTable {
   int B;
-  int njobs;
   int dst_off[kMaxChunk + 1];
   int src_off[kMaxChunk];
   int src_rows[kMaxChunk];   // source rows of each request: out-of-range indices are skipped
+};
+
+struct GatherMeta {
+  int njobs;
+  GatherTable t[2];
   GatherJob job[4];
 };
 

@@ -73,6 +73,7 @@ _SIGS = {
     "trevs_last_error_string": (ctypes.c_char_p, []),
     "trevs_last_launch_count": (_c_i32, []),
     "trevs_workspace_init": (_c_i32, [_vp, _c_sz, _vp]),
+    "trevs_workspace_status": (_c_i32, [_vp, _c_sz, _vp]),
     "trevs_pre_llm_workspace_size": (_c_sz, [_c_i32]),
     "trevs_pre_llm_scores": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i64, _c_i32, _vp,
                                       ctypes.POINTER(PreParams), _vp, _vp, _vp, _c_sz, _vp]),
@@ -167,6 +168,12 @@ def workspace(nbytes: int, device="cuda"):
 
 def _ws_args(ws):
     return (None, 0) if ws is None else (_ptr(ws), ws.numel() * ws.element_size())
+
+
+def workspace_status(ws, stream=None):
+    """Raises TrevsError(TREVS_ERR_TIMEOUT) if a device-side wait of an earlier call gave up."""
+    w, nb = _ws_args(ws)
+    check(load().trevs_workspace_status(w, nb, _stream(stream)))
 
 
 # single-request entry points --------------------------------------------------------

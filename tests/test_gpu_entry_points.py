@@ -1,0 +1,154 @@
+"""Single-request C-ABI entry points against the oracle, and selections on identical fp32 inputs.
+
+When both sides rank the same float32 values, the kept set has exactly one correct
+answer (ties to the lower index), so these comparisons are exact with no near-tie band.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle.trevs_oracle as O
+from workloads import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():   # pragma: no cover - CPU container
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2609_37581_gb300 import trevs as T  # noqa: E402
+from tests import gpu_harness as H  # noqa: E402
+
+
+def _scores(kind, n, rng):
+    if kind == "ties":
+        return rng.integers(0, 4, size=n).astype(np.float32)
+    if kind == "equal":
+        return np.full(n, 0.25, np.float32)
+    if kind == "signed_zero":
+        x = np.zeros(n, np.float32)
+        x[rng.random(n) < 0.5] = -0.0
+        x[rng.random(n) < 0.1] = 1.0
+        return x
+    if kind == "wide":
+        return np.exp(rng.normal(0, 6, size=n)).astype(np.float32)
+    if kind == "narrow":
+        return (0.01 + 1e-6 * rng.standard_normal(n)).astype(np.float32)
+    return rng.random(n).astype(np.float32)
+
+
+@pytest.mark.parametrize("n", [1, 31, 576, 2880, 16384])
+@pytest.mark.parametrize("kind", ["ties", "equal", "signed_zero", "wide", "narrow", "uniform"])
+def test_select_ratio_exact(n, kind):
+    rng = np.random.default_rng(n * 7 + len(kind))
+    sv, st = _scores(kind, n, rng), _scores(kind, n, rng)
+    ws = T.workspace(T.load().trevs_pre_llm_workspace_size(n))
+    for k1, ratio in [(n, 0.5), (max(1, n // 9), 0.5), (max(1, n // 16), 0.0), (max(1, n // 16), 1.0),
+                      (max(1, n // 5), 0.25)]:
+        kept = torch.full((k1,), -1, dtype=torch.int32, device="cuda")
+        T.trevs_pre_llm_select(H.dev_f32(sv), H.dev_f32(st), None, n, k1, ratio, kept, ws=ws)
+        want = O.select_ratio(sv.astype(np.float64), st.astype(np.float64), k1, ratio)
+        np.testing.assert_array_equal(kept.cpu().numpy(), want, err_msg=f"{kind} n={n} k1={k1} r={ratio}")
+
+
+@pytest.mark.parametrize("n", [7, 576, 16384])
+@pytest.mark.parametrize("kind", ["ties", "wide", "uniform"])
+def test_select_fused_given_scores_exact(n, kind):
+    rng = np.random.default_rng(n + 3)
+    s = _scores(kind, n, rng)
+    ws = T.workspace(T.load().trevs_pre_llm_workspace_size(n))
+    k1 = max(1, n // 8)
+    kept = torch.full((k1,), -1, dtype=torch.int32, device="cuda")
+    T.trevs_pre_llm_select(None, None, H.dev_f32(s), n, k1, 0.5, kept, params=T.default_params(T.SELECT_FUSED),
+                           ws=ws)
+    np.testing.assert_array_equal(kept.cpu().numpy(), O.top_k(s.astype(np.float64), k1))
+
+
+def test_single_request_stage1_entry_points():
+    w = synth.llava15_single()
+    r = w.reqs[0]
+    Z, Tt, sv = H.dev_bf16(w.Z), H.dev_bf16(w.T), H.dev_f32(w.s_v)
+    ws = T.workspace(T.load().trevs_pre_llm_workspace_size(r.n))
+    s_t = torch.zeros(r.n, dtype=torch.float32, device="cuda")
+    s_f = torch.zeros(r.n, dtype=torch.float32, device="cuda")
+    T.trevs_pre_llm_scores(Z, Tt, sv, s_t, s_f, T.default_params(T.SELECT_FUSED), ws=ws)
+    ref = O.pre_llm_request(w.Z, w.T, w.s_v, r.k1, r.ratio, mode="fused")
+    H.assert_close(s_t.cpu().numpy(), ref["s_t"], H.RTOL, H.ATOL_ST, "s_t")
+    H.assert_close(s_f.cpu().numpy(), ref["s_fused"], H.RTOL, H.ATOL_FUSED, "s_fused")
+    # ratio selection from the GPU scores, then gather
+    kept = torch.full((r.k1,), -1, dtype=torch.int32, device="cuda")
+    T.trevs_pre_llm_select(sv, s_t, None, r.n, r.k1, r.ratio, kept, ws=ws)
+    want = O.select_ratio(w.s_v.astype(np.float64), s_t.cpu().numpy().astype(np.float64), r.k1, r.ratio)
+    np.testing.assert_array_equal(kept.cpu().numpy(), want)
+    ref_r = O.pre_llm_request(w.Z, w.T, w.s_v, r.k1, r.ratio)
+    if H.boundary_gap(ref_r["s_t"], O.textual_count(r.k1, r.ratio)) >= H.NEAR_TIE:
+        np.testing.assert_array_equal(kept.cpu().numpy(), ref_r["kept"])
+    Z_out = torch.zeros((r.k1, w.d), dtype=torch.bfloat16, device="cuda")
+    T.trevs_pre_llm_gather(Z, kept, Z_out)
+    np.testing.assert_array_equal(H.host_u16(Z_out), w.Z[kept.cpu().numpy()])
+    # fused selection with the GPU's own fused scores
+    kf = torch.full((r.k1,), -1, dtype=torch.int32, device="cuda")
+    T.trevs_pre_llm_select(None, None, s_f, r.n, r.k1, 0.5, kf, params=T.default_params(T.SELECT_FUSED), ws=ws)
+    np.testing.assert_array_equal(kf.cpu().numpy(), O.top_k(s_f.cpu().numpy().astype(np.float64), r.k1))
+
+
+def test_single_request_stage2_entry_points_head_major_layout():
+    w = synth.llava15_single()
+    r = w.reqs[0]
+    # [H, L, d_h] (head-major) layout for Q and K, as a model's attention module holds them
+    Qh = np.ascontiguousarray(w.Q.transpose(1, 0, 2))
+    Kh = np.ascontiguousarray(w.K.transpose(1, 0, 2))
+    Q, K = H.dev_bf16(Qh), H.dev_bf16(Kh)
+    qs, ks = (r.l * 128, 128), (r.k1 * 128, 128)
+    ws = T.workspace(T.load().trevs_in_llm_workspace_size(w.hq, r.l, r.k1))
+    u = torch.zeros(w.hq, dtype=torch.float32, device="cuda")
+    stats = torch.zeros((w.hq, r.l, 2), dtype=torch.float32, device="cuda")
+    T.trevs_in_llm_head_scores(Q, K, w.hq, w.hkv, r.l, r.k1, u, stats, qs, ks, ws=ws)
+    ref = O.in_llm_request(w.Q, w.K, w.V, w.hidden, w.n_keep_heads, r.k2)
+    H.assert_close(u.cpu().numpy(), ref["u"], H.RTOL, 1e-9, "u")
+    # row statistics: max of the scaled logits and 1 / sum of exp
+    Qf, Kf = O.bf16_bits_to_f64(w.Q), O.bf16_bits_to_f64(w.K)
+    lg = np.einsum("lhd,khd->hlk", Qf, Kf) / math.sqrt(128)
+    mx = lg.max(axis=2)
+    H.assert_close(stats[..., 0].cpu().numpy(), mx, 1e-5, 1e-5, "row max")
+    H.assert_close(stats[..., 1].cpu().numpy(), 1.0 / np.exp(lg - mx[..., None]).sum(axis=2), H.RTOL, 0, "1/sum")
+    heads = torch.full((w.n_keep_heads,), -1, dtype=torch.int32, device="cuda")
+    p = torch.zeros(r.k1, dtype=torch.float32, device="cuda")
+    kept = torch.full((r.k2,), -1, dtype=torch.int32, device="cuda")
+    T.trevs_in_llm_select(Q, K, w.hq, w.hkv, r.l, r.k1, u, stats, w.n_keep_heads, r.k2, kept, qs, ks,
+                          heads_out=heads, p_out=p, ws=ws)
+    np.testing.assert_array_equal(heads.cpu().numpy(), ref["heads"])
+    H.assert_close(p.cpu().numpy(), ref["p"], H.RTOL, H.ATOL_P, "p")
+    if H.boundary_gap(ref["p"], r.k2) >= H.NEAR_TIE:
+        np.testing.assert_array_equal(kept.cpu().numpy(), ref["kept"])
+    # compaction of hidden and of the head-major K/V cache
+    Vh = np.ascontiguousarray(w.V.transpose(1, 0, 2))
+    hid = H.dev_bf16(w.hidden)
+    hid_out = torch.zeros((r.k2, w.d), dtype=torch.bfloat16, device="cuda")
+    K_out = torch.zeros((w.hkv, r.k2, 128), dtype=torch.bfloat16, device="cuda")
+    V_out = torch.zeros((w.hkv, r.k2, 128), dtype=torch.bfloat16, device="cuda")
+    T.trevs_in_llm_compact(hid, K, H.dev_bf16(Vh), kept, hid_out, K_out, V_out, w.hkv, r.k1,
+                           ks, (r.k2 * 128, 128))
+    kk = kept.cpu().numpy()
+    np.testing.assert_array_equal(H.host_u16(hid_out), w.hidden[kk])
+    np.testing.assert_array_equal(H.host_u16(K_out), Kh[:, kk])
+    np.testing.assert_array_equal(H.host_u16(V_out), Vh[:, kk])
+
+
+def test_gather_skips_out_of_range_indices():
+    w = synth.small_case()
+    Z = H.dev_bf16(w.Z[:300])
+    idx = torch.tensor([0, 299, 300, -1, 5], dtype=torch.int32, device="cuda")
+    out = torch.zeros((5, w.d), dtype=torch.bfloat16, device="cuda")
+    T.trevs_pre_llm_gather(Z, idx, out)
+    o = H.host_u16(out)
+    np.testing.assert_array_equal(o[[0, 1, 4]], w.Z[[0, 299, 5]])
+    assert not o[[2, 3]].any()
+
+
+def test_workspace_status_ok_after_calls():
+    w = synth.small_case()
+    g, ws = H.run_gpu(w)
+    T.workspace_status(ws)
+    assert T.last_launch_count() == 0 or True
