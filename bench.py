@@ -376,20 +376,25 @@ def reference_arm(args, w):
     }
 
 
-def profile_run(w, launches=5):
-    """Stage-1 scoring + selection of the bench batch, launched eagerly `launches` times."""
+def profile_run(w, stage="stage1", launches=5):
+    """Stage 1 (scoring + selection) or stage 2 of the bench batch, launched eagerly."""
     import torch
     from paper_2609_37581_gb300 import trevs as T
     from workloads.device import build_batches
     T.load()
-    pre, _ = build_batches(w, T.SELECT_RATIO)
-    q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v, kept_idx=pre.kept_idx, s_t=pre.s_t)
-    ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
-    params = T.default_params(T.SELECT_RATIO)
-    for _ in range(launches):
-        T.trevs_pre_llm_varlen(q, ws, params)
+    pre, inb = build_batches(w, T.SELECT_RATIO)
+    if stage == "stage1":
+        q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v, kept_idx=pre.kept_idx, s_t=pre.s_t)
+        ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
+        params = T.default_params(T.SELECT_RATIO)
+        for _ in range(launches):
+            T.trevs_pre_llm_varlen(q, ws, params)
+    else:
+        ws = T.workspace(T.trevs_in_llm_varlen_workspace_size(inb))
+        for _ in range(launches):
+            T.trevs_in_llm_varlen(inb, ws)
     torch.cuda.synchronize()
-    print(json.dumps({"profile": DOMINANT, "launches": launches}))
+    print(json.dumps({"profile": stage, "launches": launches}))
 
 
 def main():
@@ -399,8 +404,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--profile", action="store_true",
-                    help="only run the dominant kernel a few times (eagerly), for an ncu capture")
+    ap.add_argument("--profile", nargs="?", const="stage1", choices=["stage1", "stage2"],
+                    help="only run stage 1 (or stage 2) of the bench batch a few times, for an ncu capture")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -418,7 +423,7 @@ def main():
 
     w = workload()
     if args.profile:
-        profile_run(w)
+        profile_run(w, args.profile)
         return
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -148,31 +148,27 @@ TREVS_API trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_str
  *    g < Hkv, i < K1. Query head h reads key head floor(h*Hkv/Hq) (grouped-query attention).
  * The attention A^h[q, i] = softmax over the K1 visual keys of (Q_h[q] . K_g[i]) * scale,
  * scale = softmax_scale if > 0 else 1/sqrt(d_h) (Sec. 4.2).
- * row_stats [Hq][L][2] float32: per (head, text row) the row max of the scaled logits and
- * the reciprocal of the row's sum of exp(logit - max).
+ * attn [Hq][L][K1] float32 (dense): A^h[q, i] at attn[(h*L + q)*K1 + i].
  */
 
 /* Workspace bytes for trevs_in_llm_head_scores / trevs_in_llm_select on one request. */
 TREVS_API size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1);
 
-/* Eq. 8: u_out[h] = (1/L) sum_q Var_i A^h[q, i] (population variance over the K1 keys)
- * and row_stats_out as defined above. Limits: d_h == TREVS_HEAD_DIM,
+/* Eq. 8: u_out[h] = (1/L) sum_q Var_i A^h[q, i] (population variance over the K1 keys), and
+ * the attention probabilities in attn_out (layout above). Limits: d_h == TREVS_HEAD_DIM,
  * 1 <= K1 <= TREVS_MAX_STAGE2_TOKENS, 1 <= Hq <= TREVS_MAX_HEADS, Hq % Hkv == 0, L >= 1. */
 TREVS_API trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
                                       const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
                                       int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
-                                      float softmax_scale, float* u_out, float* row_stats_out,
+                                      float softmax_scale, float* u_out, float* attn_out,
                                       void* workspace, size_t workspace_bytes, void* stream);
 
 /* H* = the n_keep_heads heads of largest u (ties to the lower head), written ascending to
  * heads_out (may be NULL); Eq. 9 token scores p_i = max_q (1/|H*|) sum_{h in H*} A^h[q, i]
  * (written to p_out[0..K1) when non-NULL); kept_local[0..K2) = TopK(p, K2) ascending.
- * u and row_stats are the outputs of trevs_in_llm_head_scores on the same Q and K.
- * 1 <= n_keep_heads <= Hq, 0 <= K2 <= K1. */
-TREVS_API trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
-                                 const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
-                                 int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
-                                 float softmax_scale, const float* u, const float* row_stats,
+ * u and attn are the outputs of trevs_in_llm_head_scores. 1 <= n_keep_heads <= Hq,
+ * 0 <= K2 <= K1. */
+TREVS_API trevs_status trevs_in_llm_select(const float* u, const float* attn, int32_t Hq, int32_t L, int32_t K1,
                                  int32_t n_keep_heads, int32_t K2, int32_t* heads_out,
                                  float* p_out, int32_t* kept_local,
                                  void* workspace, size_t workspace_bytes, void* stream);
@@ -265,8 +261,11 @@ TREVS_API trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const 
 TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,
                                  void* workspace, size_t workspace_bytes, void* stream);
 
-/* Both stages back to back on one stream (stage 2 reads its own inputs: in a model the two
- * stages are separated by the first l* LLM layers). */
+/* Both stages on independent inputs (in a model the two stages are separated by the first l*
+ * LLM layers). Stage 2 runs as a parallel branch on an internal stream forked from and
+ * joined back into `stream` with two events; the stream and events are created on the
+ * first call of each host thread on each device and kept for the thread's life. The
+ * call stays asynchronous and can be captured into a CUDA graph. */
 TREVS_API trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_params* p,
                                 const trevs_in_batch* in,
                                 void* workspace, size_t workspace_bytes, void* stream);

@@ -19,6 +19,8 @@ cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, cudaS
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+bool in_cluster_fits(int Hq, int max_l, int max_k1);
+cudaError_t launch_in_cluster(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
 
 namespace trevs {
@@ -47,6 +49,38 @@ cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes) {
   e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e == cudaSuccess) granted.push_back(Entry{kernel, dev, bytes});
   return e;
+}
+
+// A second stream with fork / join events, created once per (host thread, device), so that
+// trevs_prune_varlen can run its two independent stages as parallel branches (also under
+// stream capture). Kept for the life of the thread.
+struct AuxStream {
+  int device = -1;
+  cudaStream_t stream = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+
+cudaError_t aux_stream(AuxStream*& out) {
+  static thread_local AuxStream aux[8];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  for (AuxStream& x : aux)
+    if (x.device == dev) {
+      out = &x;
+      return cudaSuccess;
+    }
+  for (AuxStream& x : aux)
+    if (x.device < 0) {
+      e = cudaStreamCreateWithFlags(&x.stream, cudaStreamNonBlocking);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.fork, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.join, cudaEventDisableTiming);
+      if (e != cudaSuccess) return e;
+      x.device = dev;
+      out = &x;
+      return cudaSuccess;
+    }
+  return cudaErrorInvalidDevice;
 }
 
 }  // namespace trevs
@@ -115,15 +149,16 @@ PreWs pre_ws(long long total_n) {
 }
 
 struct InWs {
-  size_t cnt_hs, cnt_ts, row_stats, row_var, u, p, keys, flags, end;
+  size_t cnt_hs, cnt_ts, attn, row_var, u, p, keys, flags, end;
 };
 
-InWs in_ws(long long total_l, long long total_k1, int Hq, int B) {
+// total_lk1 = sum over requests of l * k1 (attention probabilities per head).
+InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, int B) {
   InWs w;
   size_t o = kStatusBytes;
   w.cnt_hs = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
-  w.row_stats = o; o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
+  w.attn = o;      o = al256(o + 4 * (size_t)Hq * (size_t)total_lk1);
   w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
   w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
   w.p = o;         o = al256(o + 4 * (size_t)total_k1);
@@ -288,7 +323,7 @@ trevs_status run_pre_batch(const trevs_pre_batch* bt, const trevs_pre_params& pr
 // ---------------------------------------------------------------- stage-2 batch
 
 struct InTotals {
-  long long l = 0, k1 = 0, k2 = 0;
+  long long l = 0, k1 = 0, k2 = 0, lk1 = 0;
   int max_k1 = 0;
 };
 
@@ -324,7 +359,7 @@ trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
       return fail(TREVS_ERR_UNSUPPORTED, "request %d: k1 = %d > %d", b, r.k1, TREVS_MAX_STAGE2_TOKENS);
     TREVS_CHECK(r.l >= 1, "request %d: l = %d < 1", b, r.l);
     TREVS_CHECK(r.k2 >= 0 && r.k2 <= r.k1, "request %d: k2 = %d outside [0, k1 = %d]", b, r.k2, r.k1);
-    t.l += r.l; t.k1 += r.k1; t.k2 += r.k2;
+    t.l += r.l; t.k1 += r.k1; t.k2 += r.k2; t.lk1 += (long long)r.l * r.k1;
     t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
   }
   TREVS_CHECK(t.l < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
@@ -387,24 +422,33 @@ void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden,
 // `merged`: gather jobs of stage 1 to launch together with the compaction.
 trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
                           long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st, bool overlap,
-                          GatherMeta* merged) {
+                          GatherMeta* merged, bool launch_gather_here = true) {
   static thread_local InMeta meta;
   static thread_local GatherMeta gm_own;
   GatherMeta& gm = merged ? *merged : gm_own;
   if (!merged) gm.njobs = 0;
   meta.B = b1 - b0;
-  int hs = 0, ts = 0, max_k1 = 0;
-  long long lo = 0, ko = 0, k2o = 0;
+  int hs = 0, ts = 0, max_k1 = 0, max_l = 0;
+  long long lo = 0, ko = 0, k2o = 0, ao = 0;
   for (int b = b0; b < b1; ++b) {
     const trevs_in_request& q = bt->reqs[b];
     InReq& r = meta.r[b - b0];
+    r.attn_off = ao;
+    ao += (long long)bt->Hq * q.l * q.k1;
     r.l_off = (int)lo; r.l = q.l; r.k1_off = (int)ko; r.k1 = q.k1; r.k2_off = (int)k2o; r.k2 = q.k2;
-    r.hs_off = hs; r.ts_off = ts;
-    const int nqb = (q.l + kTextBlockRows - 1) / kTextBlockRows;
-    hs += bt->Hq * nqb;
-    ts += nqb * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
     lo += q.l; ko += q.k1; k2o += q.k2;
     max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
+    max_l = q.l > max_l ? q.l : max_l;
+  }
+  // block counts per request: text chunks of the head-statistics and token-score grids
+  const int qc = stats_text_rows(max_k1);
+  for (int b = b0; b < b1; ++b) {
+    const trevs_in_request& q = bt->reqs[b];
+    InReq& r = meta.r[b - b0];
+    r.hs_off = hs;
+    r.ts_off = ts;
+    hs += bt->Hq * ((q.l + qc - 1) / qc);
+    ts += ((q.l + kScoreTextRows - 1) / kScoreTextRows) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
   }
   meta.total_hs = hs;
   meta.total_ts = ts;
@@ -416,7 +460,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.k_hs = bt->kv_head_stride; a.k_ts = bt->kv_tok_stride;
   a.Hq = bt->Hq; a.Hkv = bt->Hkv; a.n_keep = bt->n_keep_heads;
   a.scale = bt->softmax_scale > 0.f ? bt->softmax_scale : 1.0f / sqrtf((float)bt->d_h);
-  a.row_stats = reinterpret_cast<float2*>(ws + L.row_stats);
+  a.attn = reinterpret_cast<float*>(ws + L.attn);
   a.row_var = reinterpret_cast<float*>(ws + L.row_var);
   a.stats_ld = lo;
   a.u = (bt->u ? bt->u : reinterpret_cast<float*>(ws + L.u)) + (long long)b0 * bt->Hq;
@@ -431,8 +475,12 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.hs_finalize = 1;
   a.zero_p = 1;
   a.overlap = overlap ? 1 : 0;
-  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
-  TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
+  if (in_cluster_fits(bt->Hq, max_l, max_k1)) {
+    TREVS_TRY_CUDA(counted(launch_in_cluster(meta, a, max_k1, st)), "fused stage-2 launch");
+  } else {
+    TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
+    TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
+  }
   if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
     fill_compaction(gm, meta,
                     bt->hidden ? bt->hidden + k1_base * bt->hidden_row_stride : nullptr, bt->hidden_row_stride,
@@ -444,7 +492,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
                     bt->V_out ? bt->V_out + k2_base * bt->out_tok_stride : nullptr, bt->out_head_stride,
                     bt->out_tok_stride, a.kept_local, (int)k2o);
   }
-  if (gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, true)), "compaction launch");
+  if (launch_gather_here && gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, true)), "compaction launch");
   return TREVS_OK;
 }
 
@@ -609,13 +657,13 @@ trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32
 
 size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1) {
   if (Hq < 0 || L < 0 || K1 < 0) return 0;
-  return in_ws(L, K1, Hq, 1).end;
+  return in_ws(L, K1, 0, Hq, 1).end;   // the attention probabilities live in the caller's buffer
 }
 
 trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
                                       const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
                                       int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
-                                      float softmax_scale, float* u_out, float* row_stats_out,
+                                      float softmax_scale, float* u_out, float* attn_out,
                                       void* workspace, size_t workspace_bytes, void* stream) {
   g_launches = 0;
   trevs_status s = validate_in_common(Hq, Hkv, d_h, 1);
@@ -625,16 +673,15 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   if (K1 > TREVS_MAX_STAGE2_TOKENS) return fail(TREVS_ERR_UNSUPPORTED, "K1 = %d > %d", K1, TREVS_MAX_STAGE2_TOKENS);
   s = validate_qk(Q, q_head_stride, q_tok_stride, K, k_head_stride, k_tok_stride);
   if (s != TREVS_OK) return s;
-  TREVS_CHECK(u_out && row_stats_out, "u_out and row_stats_out must be non-NULL");
-  TREVS_CHECK(((uintptr_t)row_stats_out & 7u) == 0, "row_stats_out must be 8-byte aligned");
-  const InWs W = in_ws(L, K1, Hq, 1);
+  TREVS_CHECK(u_out && attn_out, "u_out and attn_out must be non-NULL");
+  const InWs W = in_ws(L, K1, 0, Hq, 1);
   s = check_ws(workspace, workspace_bytes, W.end);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
   static thread_local InMeta meta;
   meta.B = 1;
-  meta.r[0] = InReq{0, L, 0, K1, 0, 0, 0, 0};
-  meta.total_hs = Hq * ((L + kTextBlockRows - 1) / kTextBlockRows);
+  meta.r[0] = InReq{0, 0, L, 0, K1, 0, 0, 0, 0};
+  meta.total_hs = Hq * ((L + stats_text_rows(K1) - 1) / stats_text_rows(K1));
   meta.total_ts = 0;
   InArgs a;
   memset(&a, 0, sizeof(a));
@@ -642,7 +689,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.K = reinterpret_cast<const __nv_bfloat16*>(K); a.k_hs = k_head_stride; a.k_ts = k_tok_stride;
   a.Hq = Hq; a.Hkv = Hkv; a.n_keep = 1;
   a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
-  a.row_stats = reinterpret_cast<float2*>(row_stats_out);
+  a.attn = attn_out;
   a.row_var = reinterpret_cast<float*>(ws + W.row_var);
   a.stats_ld = L;
   a.u = u_out; a.u_ld = Hq;
@@ -653,40 +700,32 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   return TREVS_OK;
 }
 
-trevs_status trevs_in_llm_select(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
-                                 const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride, int32_t Hq,
-                                 int32_t Hkv, int32_t L, int32_t K1, int32_t d_h, float softmax_scale,
-                                 const float* u, const float* row_stats, int32_t n_keep_heads, int32_t K2,
-                                 int32_t* heads_out, float* p_out, int32_t* kept_local, void* workspace,
-                                 size_t workspace_bytes, void* stream) {
+trevs_status trevs_in_llm_select(const float* u, const float* attn, int32_t Hq, int32_t L, int32_t K1,
+                                 int32_t n_keep_heads, int32_t K2, int32_t* heads_out, float* p_out,
+                                 int32_t* kept_local, void* workspace, size_t workspace_bytes, void* stream) {
   g_launches = 0;
-  trevs_status s = validate_in_common(Hq, Hkv, d_h, n_keep_heads);
-  if (s != TREVS_OK) return s;
+  TREVS_CHECK(Hq >= 1, "Hq = %d < 1", Hq);
+  if (Hq > TREVS_MAX_HEADS) return fail(TREVS_ERR_UNSUPPORTED, "Hq = %d > %d", Hq, TREVS_MAX_HEADS);
+  TREVS_CHECK(n_keep_heads >= 1 && n_keep_heads <= Hq, "n_keep_heads = %d outside [1, Hq = %d]", n_keep_heads, Hq);
   TREVS_CHECK(L >= 1, "L = %d < 1", L);
   TREVS_CHECK(K1 >= 1, "K1 = %d < 1", K1);
   if (K1 > TREVS_MAX_STAGE2_TOKENS) return fail(TREVS_ERR_UNSUPPORTED, "K1 = %d > %d", K1, TREVS_MAX_STAGE2_TOKENS);
   TREVS_CHECK(K2 >= 0 && K2 <= K1, "K2 = %d outside [0, K1 = %d]", K2, K1);
-  s = validate_qk(Q, q_head_stride, q_tok_stride, K, k_head_stride, k_tok_stride);
-  if (s != TREVS_OK) return s;
-  TREVS_CHECK(u && row_stats, "u and row_stats must be non-NULL");
-  TREVS_CHECK(((uintptr_t)row_stats & 7u) == 0, "row_stats must be 8-byte aligned");
+  TREVS_CHECK(u && attn, "u and attn must be non-NULL");
   if (K2 > 0) TREVS_CHECK(kept_local != nullptr, "kept_local is NULL");
-  const InWs W = in_ws(L, K1, Hq, 1);
-  s = check_ws(workspace, workspace_bytes, W.end);
+  const InWs W = in_ws(L, K1, 0, Hq, 1);
+  trevs_status s = check_ws(workspace, workspace_bytes, W.end);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
   static thread_local InMeta meta;
   meta.B = 1;
-  meta.r[0] = InReq{0, L, 0, K1, 0, K2, 0, 0};
+  meta.r[0] = InReq{0, 0, L, 0, K1, 0, K2, 0, 0};
   meta.total_hs = 0;
-  meta.total_ts = ((L + kTextBlockRows - 1) / kTextBlockRows) * ((K1 + kKeyBlock - 1) / kKeyBlock);
+  meta.total_ts = ((L + kScoreTextRows - 1) / kScoreTextRows) * ((K1 + kKeyBlock - 1) / kKeyBlock);
   InArgs a;
   memset(&a, 0, sizeof(a));
-  a.Q = reinterpret_cast<const __nv_bfloat16*>(Q); a.q_hs = q_head_stride; a.q_ts = q_tok_stride;
-  a.K = reinterpret_cast<const __nv_bfloat16*>(K); a.k_hs = k_head_stride; a.k_ts = k_tok_stride;
-  a.Hq = Hq; a.Hkv = Hkv; a.n_keep = n_keep_heads;
-  a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
-  a.row_stats = reinterpret_cast<float2*>(const_cast<float*>(row_stats));
+  a.Hq = Hq; a.n_keep = n_keep_heads;
+  a.attn = const_cast<float*>(attn);
   a.stats_ld = L;
   a.u = const_cast<float*>(u); a.u_ld = Hq;
   a.p_bits = p_out ? reinterpret_cast<uint32_t*>(p_out) : reinterpret_cast<uint32_t*>(ws + W.p);
@@ -733,7 +772,7 @@ trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_str
   static thread_local InMeta meta;
   static thread_local GatherMeta gm;
   meta.B = 1;
-  meta.r[0] = InReq{0, 0, 0, K1, 0, K2, 0, 0};
+  meta.r[0] = InReq{0, 0, 0, 0, K1, 0, K2, 0, 0};
   gm.njobs = 0;
   fill_compaction(gm, meta, hidden, hidden_row_stride, d_model, hidden_out, hidden_out_row_stride, Kc, Vc,
                   kv_head_stride, kv_tok_stride, Hkv, K_out, V_out, out_head_stride, out_tok_stride, kept_local, K2);
@@ -750,12 +789,13 @@ size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
 
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
-  long long l = 0, k1 = 0;
+  long long l = 0, k1 = 0, lk1 = 0;
   for (int b = 0; b < batch->B; ++b) {
-    l += batch->reqs[b].l > 0 ? batch->reqs[b].l : 0;
-    k1 += batch->reqs[b].k1 > 0 ? batch->reqs[b].k1 : 0;
+    const long long lb = batch->reqs[b].l > 0 ? batch->reqs[b].l : 0;
+    const long long kb = batch->reqs[b].k1 > 0 ? batch->reqs[b].k1 : 0;
+    l += lb; k1 += kb; lk1 += lb * kb;
   }
-  return in_ws(l, k1, batch->Hq > 0 ? batch->Hq : 0, batch->B).end;
+  return in_ws(l, k1, lk1, batch->Hq > 0 ? batch->Hq : 0, batch->B).end;
 }
 
 size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in) {
@@ -783,7 +823,7 @@ trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch, void* workspace, s
   InTotals t;
   trevs_status s = validate_in_batch(batch, t);
   if (s != TREVS_OK || batch->B == 0) return s;
-  const InWs L = in_ws(t.l, t.k1, batch->Hq, batch->B);
+  const InWs L = in_ws(t.l, t.k1, t.lk1, batch->Hq, batch->B);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_in_batch(batch, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -803,18 +843,28 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   const PreWs LP = pre_ws(tp.n);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
-  const InWs LI = in_ws(ti.l, ti.k1, in->B > 0 ? in->Hq : 0, in->B);
+  const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);
   s = check_ws(workspace, workspace_bytes, need);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
   const cudaStream_t st = (cudaStream_t)stream;
   if (pre->B > 0 && in->B > 0 && pre->B <= kMaxChunk && in->B <= kMaxChunk) {
-    // one chunk each: stage 2 overlaps the tail of stage 1, one gather launch for both
+    // one chunk each: the stages are independent, so stage 2 runs as a parallel branch on
+    // an auxiliary stream; one gather launch then serves both
+    AuxStream* aux = nullptr;
+    TREVS_TRY_CUDA(aux_stream(aux), "auxiliary stream");
+    TREVS_TRY_CUDA(cudaEventRecord(aux->fork, st), "fork");
+    TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
     static thread_local GatherMeta gm;
     s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, &gm);
     if (s != TREVS_OK) return s;
-    return run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, true, &gm);
+    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, &gm, false);
+    if (s != TREVS_OK) return s;
+    TREVS_TRY_CUDA(cudaEventRecord(aux->join, aux->stream), "join");
+    TREVS_TRY_CUDA(cudaStreamWaitEvent(st, aux->join, 0), "join");
+    if (gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, false)), "gather launch");
+    return TREVS_OK;
   }
   if (pre->B > 0) {
     s = run_pre_batch(pre, prm, ws, LP, st);

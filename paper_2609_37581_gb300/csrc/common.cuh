@@ -29,11 +29,12 @@ struct PreMeta {
 };
 
 struct InReq {
-  int l_off, l;     // text rows of Q and of the row statistics
-  int k1_off, k1;   // visual rows of K, V, hidden, p
-  int k2_off, k2;   // kept rows of kept_local and of the compacted outputs
-  int hs_off;       // first head-statistics block (Hq * ceil(l / 16) blocks)
-  int ts_off;       // first token-score block (ceil(l / 16) * ceil(k1 / 64) blocks)
+  long long attn_off;  // first attention probability of this request ([Hq][l][k1] fp32)
+  int l_off, l;        // text rows of Q and of the row variances
+  int k1_off, k1;      // visual rows of K, V, hidden, p
+  int k2_off, k2;      // kept rows of kept_local and of the compacted outputs
+  int hs_off;          // first head-statistics block
+  int ts_off;          // first token-score block
 };
 
 struct InMeta {
@@ -239,6 +240,24 @@ __device__ inline void block_kth_largest(const uint32_t* keys, int n, int k, Sel
     sh -= nbits;
     nb = 1u << nbits;
   }
+}
+
+// flags[i] = 1 (other flags untouched) for the k largest non-zero keys of keys[0..n) (ties to
+// the lower index), for n <= blockDim.x: thread i ranks key i against every key
+// (shared-memory broadcast reads).
+__device__ inline void block_mark_topk_small(const uint32_t* keys, int n, int k, uint8_t* flags) {
+  const int i = threadIdx.x;
+  if (i < n) {
+    const uint32_t mine = keys[i];
+    int rank = 0;
+#pragma unroll 4
+    for (int j = 0; j < n; ++j) {
+      const uint32_t o = keys[j];
+      rank += (o > mine) || (o == mine && j < i);
+    }
+    if (mine != 0u && rank < k) flags[i] = 1;
+  }
+  __syncthreads();
 }
 
 // flags[i] |= 1 for the entries of the top k described by (tau, need, n_eq). When every

@@ -1,10 +1,13 @@
 // Stage 2 (in-LLM at layer l*, Sec. 4.2): text-to-vision attention statistics, head
 // variance (Eq. 8), high-variance head set H*, token scores (Eq. 9), TopK and compaction.
+#include <cooperative_groups.h>
+
 #include "in_llm.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace trevs {
 
-constexpr int kQB = kTextBlockRows;
 constexpr int kKB = kKeyBlock;
 constexpr int kDh = 128;       // head width
 constexpr int kRowBytes = kDh * 2;
@@ -24,39 +27,50 @@ __device__ __forceinline__ void load_rows(uint32_t dst, const __nv_bfloat16* bas
   }
 }
 
-// A fragments of a 16 x 128 tile for all 8 k-steps.
-__device__ __forceinline__ void load_afrag(uint32_t qs, int lane, uint32_t (&af)[8][4]) {
+// A fragments of the 16 x 128 m-tile starting at `row0` of a tile, for all 8 k-steps.
+__device__ __forceinline__ void load_afrag(uint32_t qs, int row0, int lane, uint32_t (&af)[8][4]) {
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks)
-    ldmatrix_x4(tile_addr(qs, lane & 15, 2 * ks + (lane >> 4)), af[ks][0], af[ks][1], af[ks][2], af[ks][3]);
+    ldmatrix_x4(tile_addr(qs, row0 + (lane & 15), 2 * ks + (lane >> 4)), af[ks][0], af[ks][1], af[ks][2],
+                af[ks][3]);
 }
 
-// acc[2][4] = Q_tile(16 x 128) . K_rows(key0 .. key0+15)^T
-__device__ __forceinline__ void qk_16x16(const uint32_t (&af)[8][4], uint32_t ks_base, int key0, int lane,
-                                         float (&acc)[2][4]) {
+// acc[NT][4] = Q m-tile (16 x 128) . K_rows(key0 .. key0 + 8*NT - 1)^T, NT even.
+template <int NT>
+__device__ __forceinline__ void qk_tile(const uint32_t (&af)[8][4], uint32_t ks_base, int key0, int lane,
+                                        float (&acc)[NT][4]) {
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
+  for (int i = 0; i < NT; ++i)
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
-    const int mi = lane >> 3;
-    const int rr = key0 + 8 * (mi >> 1) + (lane & 7), c = 2 * ks + (mi & 1);
-    uint32_t b0, b1, b2, b3;
-    ldmatrix_x4(tile_addr(ks_base, rr, c), b0, b1, b2, b3);
-    mma_bf16_16816(acc[0], af[ks], b0, b1);
-    mma_bf16_16816(acc[1], af[ks], b2, b3);
+#pragma unroll
+    for (int p = 0; p < NT / 2; ++p) {
+      const int mi = lane >> 3;
+      const int rr = key0 + 16 * p + 8 * (mi >> 1) + (lane & 7), c = 2 * ks + (mi & 1);
+      uint32_t b0, b1, b2, b3;
+      ldmatrix_x4(tile_addr(ks_base, rr, c), b0, b1, b2, b3);
+      mma_bf16_16816(acc[2 * p], af[ks], b0, b1);
+      mma_bf16_16816(acc[2 * p + 1], af[ks], b2, b3);
+    }
   }
 }
 
 // ------------------------------------------------------------------ attention statistics
 //
-// Block (request, head h, 16-row block of text queries): logits Q_h . K_g^T * scale for all
-// K1 keys into shared memory (tensor cores), then per row the max, the sum of exp and the
-// two-pass variance of the softmax row about its mean 1/K1 (Eq. 8). The last block of a
-// request averages the row variances into u_h.
+// Block (request, head h, chunk of QC = 16*MT text rows): logits Q_h . K_g^T * scale for all
+// K1 keys into shared memory (tensor cores; K streamed once in 64-key chunks through a
+// two-buffer cp.async ring), then per row the max, the sum of exp and the two-pass
+// variance of the softmax row about its mean 1/K1 (Eq. 8). The last block of a request
+// averages the row variances into u_h and clears p for the token-score pass.
+// Warp w computes m-tile (w % MT) against key slice (w / MT) of each chunk.
+template <int MT>
 __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constant__ InMeta meta,
                                                             const InArgs a, int k1_ld) {
+  constexpr int QC = 16 * MT;
+  constexpr int KW = 16 * MT;          // keys per warp in a 64-key chunk
+  constexpr int NT = KW / 8;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_last;
   if (!a.overlap) pdl_wait();   // Q, K may come from the preceding grid
@@ -64,22 +78,24 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
   const InReq r = meta.r[b];
-  const int nqb = (r.l + kQB - 1) / kQB;
+  const int nqc = (r.l + QC - 1) / QC;
   const int t = blockIdx.x - r.hs_off;
-  const int h = t / nqb, qb = t - h * nqb;
+  const int h = t / nqc, qc = t - h * nqc;
   const int g = (h * a.Hkv) / a.Hq;
-  const int q0 = qb * kQB;
+  const int q0 = qc * QC;
 
-  uint8_t* qs = smem;                              // 16 x 256 B
-  uint8_t* kbuf = smem + kQB * kRowBytes;          // 2 x 64 x 256 B
-  float* lg = reinterpret_cast<float*>(kbuf + 2 * kKB * kRowBytes);   // [16][k1_ld]
+  uint8_t* qs = smem;                              // QC x 256 B
+  uint8_t* kbuf = smem + QC * kRowBytes;           // 2 x 64 x 256 B
+  float* lg = reinterpret_cast<float*>(kbuf + 2 * kKB * kRowBytes);   // [QC][k1_ld]
   const uint32_t qs_a = smem_u32(qs), kb_a = smem_u32(kbuf);
 
   const __nv_bfloat16* Qb = a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs;
   const __nv_bfloat16* Kb = a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs;
   const int nkc = (r.k1 + kKB - 1) / kKB;
+  const int mt = warp % MT, kslice = warp / MT;
+  const float sc = a.scale * 1.4426950408889634f;   // logits in log2 units: exp(x) = exp2(x * log2 e)
 
-  load_rows(qs_a, Qb, a.q_ts, q0, kQB, r.l, tid, 128);
+  load_rows(qs_a, Qb, a.q_ts, q0, QC, r.l, tid, 128);
   load_rows(kb_a, Kb, a.k_ts, 0, kKB, r.k1, tid, 128);
   cp_async_commit();
   uint32_t af[8][4];
@@ -88,49 +104,64 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
     cp_async_commit();
     cp_async_wait<1>();
     __syncthreads();
-    if (kc == 0) load_afrag(qs_a, lane, af);
-    float acc[2][4];
-    qk_16x16(af, kb_a + (kc & 1) * kKB * kRowBytes, 16 * warp, lane, acc);
+    if (kc == 0) load_afrag(qs_a, 16 * mt, lane, af);
+    float acc[NT][4];
+    qk_tile<NT>(af, kb_a + (kc & 1) * kKB * kRowBytes, kslice * KW, lane, acc);
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      const int key = kc * kKB + 16 * warp + 8 * nt + 2 * (lane & 3);
-      const int row = lane >> 2;
-      *reinterpret_cast<float2*>(lg + row * k1_ld + key) = make_float2(acc[nt][0] * a.scale, acc[nt][1] * a.scale);
-      *reinterpret_cast<float2*>(lg + (row + 8) * k1_ld + key) = make_float2(acc[nt][2] * a.scale, acc[nt][3] * a.scale);
+    for (int nt = 0; nt < NT; ++nt) {
+      const int key = kc * kKB + kslice * KW + 8 * nt + 2 * (lane & 3);
+      const int row = 16 * mt + (lane >> 2);
+      *reinterpret_cast<float2*>(lg + row * k1_ld + key) = make_float2(acc[nt][0] * sc, acc[nt][1] * sc);
+      *reinterpret_cast<float2*>(lg + (row + 8) * k1_ld + key) = make_float2(acc[nt][2] * sc, acc[nt][3] * sc);
     }
     __syncthreads();
   }
 
+  // row statistics, TPR threads per row (all rows of the chunk in parallel)
+  constexpr int TPR = 128 / QC;
+  __shared__ float s_inv[64];
   const int k1 = r.k1;
   const float mean = 1.0f / (float)k1;
-  for (int rr = warp; rr < kQB; rr += 4) {
-    const int q = q0 + rr;
-    if (q >= r.l) break;
+  {
+    const int rr = tid / TPR, sub = tid % TPR;
     float* row = lg + rr * k1_ld;
     float mx = -INFINITY;
-    for (int i = lane; i < k1; i += 32) mx = fmaxf(mx, row[i]);
+#pragma unroll 4
+    for (int i = sub; i < k1; i += TPR) mx = fmaxf(mx, row[i]);
 #pragma unroll
-    for (int o = 16; o; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    for (int o = 1; o < TPR; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     float sum = 0.f;
-    for (int i = lane; i < k1; i += 32) {
-      const float e = expf(row[i] - mx);
+#pragma unroll 4
+    for (int i = sub; i < k1; i += TPR) {
+      const float e = exp2f(row[i] - mx);
       row[i] = e;
       sum += e;
     }
 #pragma unroll
-    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    const float inv = 1.0f / sum;
-    float v = 0.f;
-    for (int i = lane; i < k1; i += 32) {
-      const float dlt = row[i] * inv - mean;
-      v = fmaf(dlt, dlt, v);
-    }
+    for (int o = 1; o < TPR; o <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (sub == 0) s_inv[rr] = 1.0f / sum;
+  }
+  __syncthreads();
+  // A[h][q][i] = e / sum, written along i by whole warps, and the two-pass variance of the
+  // row about its mean 1/K1 (Eq. 8)
+  {
+    const int rows = min(QC, r.l - q0);
+    float* A = a.attn + r.attn_off + ((long long)h * r.l + q0) * k1;
+    for (int rr = warp; rr < rows; rr += 4) {
+      const float inv = s_inv[rr];
+      const float* row = lg + rr * k1_ld;
+      float* out = A + (long long)rr * k1;
+      float v = 0.f;
+#pragma unroll 2
+      for (int i = lane; i < k1; i += 32) {
+        const float p = row[i] * inv;
+        out[i] = p;
+        const float dlt = p - mean;
+        v = fmaf(dlt, dlt, v);
+      }
 #pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) {
-      const long long o = (long long)h * a.stats_ld + r.l_off + q;
-      a.row_stats[o] = make_float2(mx, inv);
-      a.row_var[o] = v / (float)k1;
+      for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == 0) a.row_var[(long long)h * a.stats_ld + r.l_off + q0 + rr] = v / (float)k1;
     }
   }
 
@@ -141,17 +172,20 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
   __syncthreads();
   if (tid == 0) {
     const unsigned prev = atomicAdd(&a.cnt_hs[b], 1u);
-    s_last = (prev == (unsigned)(a.Hq * nqb) - 1);
+    s_last = (prev == (unsigned)(a.Hq * nqc) - 1);
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
   if (tid == 0) a.cnt_hs[b] = 0u;
-  for (int hh = tid; hh < a.Hq; hh += 128) {
+  // u_h = mean over text rows of the row variances: one warp per head, lanes over rows
+  for (int hh = warp; hh < a.Hq; hh += 4) {
     const float* rv = a.row_var + (long long)hh * a.stats_ld + r.l_off;
     float s = 0.f;
-    for (int q = 0; q < r.l; ++q) s += __ldcg(rv + q);
-    a.u[(long long)b * a.u_ld + hh] = s / (float)r.l;
+    for (int q = lane; q < r.l; q += 32) s += __ldcg(rv + q);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) a.u[(long long)b * a.u_ld + hh] = s / (float)r.l;
   }
   if (a.zero_p)
     for (int i = tid; i < r.k1; i += 128) a.p_bits[r.k1_off + i] = 0u;
@@ -159,36 +193,42 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
 
 // ------------------------------------------------------------------ token scores
 //
-// Block (request, 16-row text block, 64-key block): for each head of H* in ascending order
-// recompute the logits on the tensor cores, turn them into attention with the row
-// statistics, and accumulate the head sum; the max over the block's text rows of the head
-// mean (Eq. 9) is merged across text blocks with an integer atomicMax on the (non-negative)
-// float bits, which is exact and order independent. The last block of a request selects
-// TopK(p, K2) and writes H*.
+// Block (request, 16-row text chunk, 64-key block): for each head of H* in ascending order
+// sum the stored attention probabilities (Eq. 9, head mean), then take the max over the
+// chunk's text rows; chunks merge with an integer atomicMax on the (non-negative) float
+// bits, which is exact and order independent. Thread t owns key t % 64 and rows
+// t / 64, t / 64 + 2, ...; every load is a 256-byte row segment. The last block of a
+// request selects TopK(p, K2) and writes H*.
 __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_constant__ InMeta meta,
                                                              const InArgs a, int smem_bytes) {
+  constexpr int QC = kScoreTextRows;
+  constexpr int RPT = QC / 2;         // rows per thread
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ SelShared ss;
   __shared__ int s_heads[kMaxHeads];
   __shared__ int s_sel[kMaxHeads];
+  __shared__ float s_half[kKB];
   __shared__ int s_nh, s_last;
-  pdl_wait();   // u, row statistics and the cleared p come from the preceding grid
+  pdl_wait();   // u, the attention probabilities and the cleared p come from the preceding grid
   pdl_launch_dependents();
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].ts_off; });
   const InReq r = meta.r[b];
   const int nib = (r.k1 + kKB - 1) / kKB;
   const int t = blockIdx.x - r.ts_off;
-  const int qb = t / nib, ib = t - qb * nib;
-  const int q0 = qb * kQB, i0 = ib * kKB;
+  const int qc = t / nib, ib = t - qc * nib;
+  const int q0 = qc * QC, i0 = ib * kKB;
 
   // H*: the n_keep heads of largest u, ties to the lower head
+  __shared__ float s_u[kMaxHeads];
   const float* u = a.u + (long long)b * a.u_ld;
+  for (int hh = tid; hh < a.Hq; hh += 128) s_u[hh] = __ldcg(u + hh);
+  __syncthreads();
   for (int hh = tid; hh < a.Hq; hh += 128) {
-    const float uh = __ldcg(u + hh);
+    const float uh = s_u[hh];
     int rank = 0;
     for (int x = 0; x < a.Hq; ++x) {
-      const float ux = __ldcg(u + x);
+      const float ux = s_u[x];
       rank += (ux > uh) || (ux == uh && x < hh);
     }
     s_sel[hh] = rank < a.n_keep;
@@ -201,74 +241,58 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
     s_nh = cnt;
   }
   __syncthreads();
+  const int nh = s_nh;
 
-  uint8_t* qs = smem;
-  uint8_t* ks = smem + kQB * kRowBytes;
-  const uint32_t qs_a = smem_u32(qs), ks_a = smem_u32(ks);
-  float psum[2][4];
+  const int key = i0 + (tid & (kKB - 1));
+  const int rbase = tid / kKB;
+  float psum[RPT];
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
+  for (int j = 0; j < RPT; ++j) psum[j] = 0.f;
+  if (key < r.k1) {
+    // four heads' rows in flight at a time; heads are still summed in ascending order
+    const float* A0 = a.attn + r.attn_off + key;
+    const long long hstride = (long long)r.l * r.k1;
+    for (int h0 = 0; h0 < nh; h0 += 4) {
+      float v[4][RPT];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) psum[i][j] = 0.f;
-  const int ra = q0 + (lane >> 2), rb = ra + 8;
-  int g_loaded = -1;
-  for (int hi = 0; hi < s_nh; ++hi) {
-    const int h = s_heads[hi];
-    const int g = (h * a.Hkv) / a.Hq;
-    load_rows(qs_a, a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs, a.q_ts, q0, kQB, r.l, tid, 128);
-    if (g != g_loaded)
-      load_rows(ks_a, a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs, a.k_ts, i0, kKB, r.k1, tid, 128);
-    g_loaded = g;
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-    uint32_t af[8][4];
-    load_afrag(qs_a, lane, af);
-    float acc[2][4];
-    qk_16x16(af, ks_a, 16 * warp, lane, acc);
-    const long long so = (long long)h * a.stats_ld + r.l_off;
-    const float2 sa = ra < r.l ? __ldcg(a.row_stats + so + ra) : make_float2(0.f, 0.f);
-    const float2 sb = rb < r.l ? __ldcg(a.row_stats + so + rb) : make_float2(0.f, 0.f);
+      for (int x = 0; x < 4; ++x) {
+        const float* A = A0 + (long long)s_heads[min(h0 + x, nh - 1)] * hstride;
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      psum[nt][0] += expf(acc[nt][0] * a.scale - sa.x) * sa.y;
-      psum[nt][1] += expf(acc[nt][1] * a.scale - sa.x) * sa.y;
-      psum[nt][2] += expf(acc[nt][2] * a.scale - sb.x) * sb.y;
-      psum[nt][3] += expf(acc[nt][3] * a.scale - sb.x) * sb.y;
+        for (int j = 0; j < RPT; ++j) {
+          const int q = q0 + rbase + 2 * j;
+          v[x][j] = (h0 + x < nh && q < r.l) ? __ldcg(A + (long long)q * r.k1) : 0.f;
+        }
+      }
+#pragma unroll
+      for (int x = 0; x < 4; ++x)
+#pragma unroll
+        for (int j = 0; j < RPT; ++j) psum[j] += v[x][j];
     }
-    __syncthreads();
   }
   // rows past L contribute nothing; attention is positive, so 0 never wins the max
-  const float inv_nh = s_nh > 0 ? 1.0f / (float)s_nh : 0.f;
+  float m = 0.f;
 #pragma unroll
-  for (int nt = 0; nt < 2; ++nt) {
-    float m0 = fmaxf(ra < r.l ? psum[nt][0] : 0.f, rb < r.l ? psum[nt][2] : 0.f);
-    float m1 = fmaxf(ra < r.l ? psum[nt][1] : 0.f, rb < r.l ? psum[nt][3] : 0.f);
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-      m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
-      m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, o));
-    }
-    if (lane < 4) {
-      const int i = i0 + 16 * warp + 8 * nt + 2 * lane;
-      if (i < r.k1) atomicMax(a.p_bits + r.k1_off + i, __float_as_uint(m0 * inv_nh));
-      if (i + 1 < r.k1) atomicMax(a.p_bits + r.k1_off + i + 1, __float_as_uint(m1 * inv_nh));
-    }
+  for (int j = 0; j < RPT; ++j) m = fmaxf(m, psum[j]);
+  if (rbase == 1) s_half[tid & (kKB - 1)] = m;
+  __syncthreads();
+  if (rbase == 0 && key < r.k1) {
+    const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
+    atomicMax(a.p_bits + r.k1_off + key, __float_as_uint(fmaxf(m, s_half[tid]) * inv_nh));
   }
 
   __threadfence();
   __syncthreads();
   if (tid == 0) {
-    const int nqb = (r.l + kQB - 1) / kQB;
+    const int nqc = (r.l + QC - 1) / QC;
     const unsigned prev = atomicAdd(&a.cnt_ts[b], 1u);
-    s_last = (prev == (unsigned)(nqb * nib) - 1);
+    s_last = (prev == (unsigned)(nqc * nib) - 1);
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
   if (tid == 0) a.cnt_ts[b] = 0u;
   if (a.heads_out)
-    for (int x = tid; x < s_nh; x += 128) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
+    for (int x = tid; x < nh; x += 128) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
   if (r.k2 <= 0) return;
   const int n = r.k1;
   const bool in_smem = (size_t)n * 5 <= (size_t)smem_bytes;
@@ -280,28 +304,322 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
   int need, n_eq;
   block_fill_keys(keys, reinterpret_cast<const float*>(a.p_bits + r.k1_off), n,
                   [&](float x, int) { return score_key(x); }, ss, lo, hi);
-  block_kth_largest(keys, n, r.k2, ss, lo, hi, tau, need, n_eq);
-  block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+  if (n <= 128) {
+    block_mark_topk_small(keys, n, r.k2, flags);
+  } else {
+    block_kth_largest(keys, n, r.k2, ss, lo, hi, tau, need, n_eq);
+    block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+  }
   block_compact_flags(flags, n, a.kept_local + r.k2_off, ss);
+}
+
+// ------------------------------------------------------------------ fused stage 2 for small requests
+//
+// One cluster of 8 CTAs per request (text rows L <= 64, visual tokens K1 <= 128). CTA c owns
+// heads c, c + 8, ... (at most 8). Phase 1: for each of its heads, the logits on the tensor
+// cores and the softmax statistics and Eq. 8 row variances in registers (a quad of lanes
+// holds all keys of two text rows). The CTAs then read each other's u_h through distributed
+// shared memory and agree on H*. Phase 2: each CTA recomputes the logits of its selected
+// heads (ascending) and accumulates their attention probabilities in registers. Phase 3:
+// the keys are split among the CTAs for Eq. 9 (partials summed in CTA order, max over the
+// text rows), CTA 0 collects p and selects TopK(p, K2). Only the results reach global
+// memory; the cluster barriers are hardware barriers of co-resident CTAs.
+template <int NCH>   // 64-key chunks: K1 <= 64 * NCH
+__global__ void __launch_bounds__(128) in_cluster_kernel(const __grid_constant__ InMeta meta, const InArgs a,
+                                                         int a_ld) {
+  constexpr int QR = 64;              // text rows (four m16 tiles, one per warp)
+  constexpr int NT = 8;               // n-tiles of a 64-key chunk
+  cg::cluster_group cluster = cg::this_cluster();
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ float s_u[8];
+  __shared__ float s_upart[8][4];
+  __shared__ float2 s_stat[8][QR];    // per own head and row: (max in log2 units, 1 / sum)
+  __shared__ float s_uall[kMaxHeads];
+  __shared__ int s_sel[kMaxHeads];
+  __shared__ int s_heads[kMaxHeads];
+  __shared__ int s_nh;
+  __shared__ uint32_t s_pmax[16];
+  __shared__ float s_p[128];
+  __shared__ uint32_t s_keys[128];
+  __shared__ uint8_t s_flags[128];
+  __shared__ SelShared ss;
+  pdl_wait();                         // Q, K may come from the preceding grid
+  pdl_launch_dependents();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c = (int)cluster.block_rank();
+  const int b = blockIdx.x / kClusterCtas;
+  const InReq r = meta.r[b];
+  const int L = r.l, K1 = r.k1, Hq = a.Hq;
+  const int nmine = c < Hq ? (Hq - c + kClusterCtas - 1) / kClusterCtas : 0;
+
+  uint8_t* qs = smem;                                   // QR x 256 B
+  uint8_t* ks = smem + QR * kRowBytes;                  // 64 * NCH x 256 B
+  float* pbuf = reinterpret_cast<float*>(smem);         // [QR][a_ld] after phase 2
+  const uint32_t qs_a = smem_u32(qs), ks_a = smem_u32(ks);
+  const float sc = a.scale * 1.4426950408889634f;       // logits in log2 units
+  const float mean = 1.0f / (float)K1;
+  const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
+
+  auto issue = [&](int j) {
+    const int h = c + kClusterCtas * j;
+    const int g = (h * a.Hkv) / Hq;
+    load_rows(qs_a, a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs, a.q_ts, 0, QR, L, tid, 128);
+    load_rows(ks_a, a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs, a.k_ts, 0, 64 * NCH, K1, tid, 128);
+  };
+  float acc[NCH][NT][4];
+  // logits of the staged head into acc; the stage is free (and refilled with head `next`) after
+  auto logits = [&](int next) {
+    cp_async_wait<0>();
+    __syncthreads();
+    uint32_t af[8][4];
+    load_afrag(qs_a, 16 * warp, lane, af);
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch) qk_tile<NT>(af, ks_a + ch * 64 * kRowBytes, 0, lane, acc[ch]);
+    __syncthreads();
+    if (next >= 0) issue(next);
+    cp_async_commit();
+  };
+
+  // ---- phase 1: statistics and row variances of this CTA's heads
+  if (nmine > 0) issue(0);
+  cp_async_commit();
+  for (int j = 0; j < nmine; ++j) {
+    logits(j + 1 < nmine ? j + 1 : -1);
+    float mxa = -INFINITY, mxb = -INFINITY;
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
+          if (key < K1) {
+            mxa = fmaxf(mxa, acc[ch][nt][e] * sc);
+            mxb = fmaxf(mxb, acc[ch][nt][2 + e] * sc);
+          }
+        }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, o));
+      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, o));
+    }
+    float sa = 0.f, sb = 0.f;
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
+          const float ea = key < K1 ? exp2f(acc[ch][nt][e] * sc - mxa) : 0.f;
+          const float eb = key < K1 ? exp2f(acc[ch][nt][2 + e] * sc - mxb) : 0.f;
+          acc[ch][nt][e] = ea;
+          acc[ch][nt][2 + e] = eb;
+          sa += ea;
+          sb += eb;
+        }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      sa += __shfl_xor_sync(0xffffffffu, sa, o);
+      sb += __shfl_xor_sync(0xffffffffu, sb, o);
+    }
+    const float ia = 1.0f / sa, ib = 1.0f / sb;
+    float va = 0.f, vb = 0.f;
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
+          if (key < K1) {
+            const float da = acc[ch][nt][e] * ia - mean, db = acc[ch][nt][2 + e] * ib - mean;
+            va = fmaf(da, da, va);
+            vb = fmaf(db, db, vb);
+          }
+        }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      va += __shfl_xor_sync(0xffffffffu, va, o);
+      vb += __shfl_xor_sync(0xffffffffu, vb, o);
+    }
+    if ((lane & 3) == 0) {
+      s_stat[j][ra] = make_float2(mxa, ia);
+      s_stat[j][rb] = make_float2(mxb, ib);
+    }
+    // Eq. 8 numerator: sum over this warp's valid rows of Var_i A[q, i]
+    float vs = ((lane & 3) == 0) ? ((ra < L ? va : 0.f) + (rb < L ? vb : 0.f)) / (float)K1 : 0.f;
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) vs += __shfl_xor_sync(0xffffffffu, vs, o);
+    if (lane == 0) s_upart[j][warp] = vs;
+  }
+  __syncthreads();
+  if (tid < nmine) s_u[tid] = (((s_upart[tid][0] + s_upart[tid][1]) + s_upart[tid][2]) + s_upart[tid][3]) / (float)L;
+  cluster.sync();
+
+  // every CTA gathers all u_h and ranks the heads: H* is the n_keep largest, ties to lower h
+  for (int h = tid; h < Hq; h += 128) s_uall[h] = *cluster.map_shared_rank(&s_u[h / kClusterCtas], h % kClusterCtas);
+  __syncthreads();
+  for (int h = tid; h < Hq; h += 128) {
+    const float uh = s_uall[h];
+    int rank = 0;
+    for (int x = 0; x < Hq; ++x) rank += (s_uall[x] > uh) || (s_uall[x] == uh && x < h);
+    s_sel[h] = rank < a.n_keep;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int cnt = 0;
+    for (int h = 0; h < Hq && cnt < a.n_keep; ++h)
+      if (s_sel[h]) s_heads[cnt++] = h;
+    s_nh = cnt;
+  }
+  __syncthreads();
+  const int nh = s_nh;
+  if (c == 0) {
+    for (int h = tid; h < Hq; h += 128) a.u[(long long)b * a.u_ld + h] = s_uall[h];
+    if (a.heads_out)
+      for (int x = tid; x < nh; x += 128) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
+  }
+
+  // ---- phase 2: sum of the attention probabilities of this CTA's selected heads
+  int sel[8];
+  int nsel = 0;
+  for (int j = 0; j < nmine; ++j)
+    if (s_sel[c + kClusterCtas * j]) sel[nsel++] = j;
+  float psum[NCH][NT][4];
+#pragma unroll
+  for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) psum[ch][nt][e] = 0.f;
+  if (nsel > 0) issue(sel[0]);
+  cp_async_commit();
+  for (int x = 0; x < nsel; ++x) {
+    logits(x + 1 < nsel ? sel[x + 1] : -1);
+    const float2 ta = s_stat[sel[x]][ra], tb = s_stat[sel[x]][rb];
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          psum[ch][nt][e] += exp2f(acc[ch][nt][e] * sc - ta.x) * ta.y;
+          psum[ch][nt][2 + e] += exp2f(acc[ch][nt][2 + e] * sc - tb.x) * tb.y;
+        }
+  }
+  cp_async_wait<0>();
+  __syncthreads();                                      // the stage is free: it becomes pbuf
+#pragma unroll
+  for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int key = 64 * ch + 8 * nt + 2 * (lane & 3);
+      *reinterpret_cast<float2*>(pbuf + ra * a_ld + key) = make_float2(psum[ch][nt][0], psum[ch][nt][1]);
+      *reinterpret_cast<float2*>(pbuf + rb * a_ld + key) = make_float2(psum[ch][nt][2], psum[ch][nt][3]);
+    }
+  if (tid < 16) s_pmax[tid] = 0u;
+  cluster.sync();
+
+  // ---- phase 3: Eq. 9 for keys i = c + 8m: partials summed in CTA order, max over text rows
+  const int kc = K1 > c ? (K1 - c + kClusterCtas - 1) / kClusterCtas : 0;
+  for (int pair = tid; pair < kc * L; pair += 128) {
+    const int m = pair % kc, q = pair / kc;
+    const int i = c + kClusterCtas * m;
+    float v[kClusterCtas];
+#pragma unroll
+    for (int cc = 0; cc < kClusterCtas; ++cc) v[cc] = *cluster.map_shared_rank(pbuf + q * a_ld + i, cc);
+    float t = 0.f;
+#pragma unroll
+    for (int cc = 0; cc < kClusterCtas; ++cc) t += v[cc];
+    atomicMax(&s_pmax[m], __float_as_uint(t));
+  }
+  __syncthreads();
+  if (tid < kc) {
+    const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
+    *cluster.map_shared_rank(&s_p[c + kClusterCtas * tid], 0) = __uint_as_float(s_pmax[tid]) * inv_nh;
+  }
+  cluster.sync();
+
+  if (c == 0) {
+    for (int i = tid; i < K1; i += 128) {
+      a.p_bits[r.k1_off + i] = __float_as_uint(s_p[i]);
+      s_keys[i] = score_key(s_p[i]);
+      s_flags[i] = 0;
+    }
+    __syncthreads();
+    if (r.k2 > 0) {
+      block_mark_topk_small(s_keys, K1, r.k2, s_flags);
+      block_compact_flags(s_flags, K1, a.kept_local + r.k2_off, ss);
+    }
+  }
 }
 
 // ------------------------------------------------------------------ host-side launchers
 
-int in_head_stats_ld(int max_k1) { return ((max_k1 + kKB - 1) / kKB) * kKB + 8; }
+// Row stride of the logits tile: 2 mod 32 words keeps the row-parallel passes conflict-free.
+int in_head_stats_ld(int max_k1) { return ((max_k1 + kKB - 1) / kKB) * kKB + 2; }
 
 cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
   if (meta.total_hs == 0) return cudaSuccess;
   const int ld = in_head_stats_ld(max_k1);
-  const int smem = kQB * kRowBytes + 2 * kKB * kRowBytes + kQB * ld * 4;
-  cudaError_t e = ensure_dynamic_smem(in_head_stats_kernel, smem);
+  const int qc = stats_text_rows(max_k1);
+  const int smem = qc * kRowBytes + 2 * kKB * kRowBytes + qc * ld * 4;   // two K chunk buffers
+  cudaError_t e;
+  switch (qc) {
+    case 64:
+      e = ensure_dynamic_smem(in_head_stats_kernel<4>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<4>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+    case 32:
+      e = ensure_dynamic_smem(in_head_stats_kernel<2>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<2>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+    default:
+      e = ensure_dynamic_smem(in_head_stats_kernel<1>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<1>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+  }
+}
+
+// Fused stage 2 on 8-CTA clusters when every request has L <= 64 and K1 <= 128.
+bool in_cluster_fits(int Hq, int max_l, int max_k1) {
+  if (max_l > 64 || max_k1 > 128 || Hq > 64) return false;
+  return true;
+}
+
+cudaError_t launch_in_cluster(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
+  if (meta.B == 0) return cudaSuccess;
+  const int nch = max_k1 <= 64 ? 1 : 2;
+  const int a_ld = 64 * nch + 8;
+  int smem = 64 * kRowBytes + 64 * nch * kRowBytes;     // one Q / K stage, later the partial sums
+  if (64 * a_ld * 4 > smem) smem = 64 * a_ld * 4;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(meta.B * kClusterCtas);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kClusterCtas;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e;
+  if (nch == 1) {
+    e = ensure_dynamic_smem(in_cluster_kernel<1>, smem);
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, in_cluster_kernel<1>, meta, a, a_ld);
+  }
+  e = ensure_dynamic_smem(in_cluster_kernel<2>, smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(in_head_stats_kernel, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+  return cudaLaunchKernelEx(&cfg, in_cluster_kernel<2>, meta, a, a_ld);
 }
 
 cudaError_t launch_in_token_score(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
   if (meta.total_ts == 0) return cudaSuccess;
-  int smem = kQB * kRowBytes + kKB * kRowBytes;
-  if (max_k1 * 5 > smem) smem = max_k1 * 5;
+  const int smem = max_k1 * 5 + 16;
   cudaError_t e = ensure_dynamic_smem(in_token_score_kernel, smem);
   if (e != cudaSuccess) return e;
   return launch_kernel(in_token_score_kernel, dim3(meta.total_ts), dim3(128), smem, st, true, meta, a, smem);

@@ -6,8 +6,12 @@
 namespace trevs {
 
 constexpr int kMaxHeads = 128;
-constexpr int kTextBlockRows = 16;   // text rows per stage-2 block (one m16 tile)
 constexpr int kKeyBlock = 64;        // visual keys per stage-2 block / shared-memory chunk
+constexpr int kScoreTextRows = 16;   // text rows per token-score block
+constexpr int kClusterCtas = 8;      // CTAs per request of the fused small-request stage 2
+
+// Text rows per head-statistics block: the block keeps rows x K1 fp32 logits on chip.
+inline int stats_text_rows(int max_k1) { return max_k1 <= 128 ? 64 : (max_k1 <= 512 ? 32 : 16); }
 
 struct InArgs {
   const __nv_bfloat16* Q;
@@ -16,7 +20,7 @@ struct InArgs {
   long long k_hs, k_ts;
   int Hq, Hkv, n_keep;
   float scale;
-  float2* row_stats;        // [Hq][stats_ld]: (row max of scaled logits, 1 / row sum of exp)
+  float* attn;              // attention probabilities, request b at attn_off: [Hq][l][k1]
   float* row_var;           // [Hq][stats_ld]: Var_i A[q, i]
   long long stats_ld;       // total text rows of the launch
   float* u;                 // [B][u_ld] head variances (Eq. 8)

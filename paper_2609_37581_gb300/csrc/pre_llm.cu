@@ -253,7 +253,7 @@ __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant
 // ------------------------------------------------------------------ row gather
 //
 // One warp per destination row: dst[row] = src[off + idx[row]] for every head segment,
-// 16-byte vector loads with four in flight per lane.
+// 16-byte vector loads with eight in flight per lane.
 __global__ void __launch_bounds__(256) gather_rows_kernel(const __grid_constant__ GatherMeta gm) {
   pdl_wait();   // the indices come from the preceding grids
   const GatherJob& j = gm.job[blockIdx.y];
@@ -269,10 +269,10 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const __grid_constant_
   const int total = U * j.heads;
   const uint8_t* src = j.src + srow * j.src_tok;
   uint8_t* dst = j.dst + (long long)row * j.dst_tok;
-  for (int x0 = lane; x0 < total; x0 += 128) {
-    uint4 v[4];
+  for (int x0 = lane; x0 < total; x0 += 256) {
+    uint4 v[8];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < 8; ++q) {
       const int x = x0 + 32 * q;
       if (x < total) {
         const int h = x / U, u = x - h * U;
@@ -280,7 +280,7 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const __grid_constant_
       }
     }
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < 8; ++q) {
       const int x = x0 + 32 * q;
       if (x < total) {
         const int h = x / U, u = x - h * U;

@@ -107,7 +107,9 @@ __device__ inline void select_request(const PreArgs& a, const PreReq& r, int b, 
       flags[i] = in_v ? 1 : 0;
       return in_v ? 0u : score_key(x);
     }, ss, lo, hi);
-    if (r.kt > 0) {
+    if (r.kt > 0 && n <= nthr) {
+      block_mark_topk_small(keys, n, r.kt, flags);
+    } else if (r.kt > 0) {
       block_kth_largest(keys, n, r.kt, ss, lo, hi, tau, need, n_eq);
       block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
     }
@@ -137,8 +139,12 @@ __device__ inline void select_request(const PreArgs& a, const PreReq& r, int b, 
   if (do_select && r.k1 > 0) {
     for (int i = tid; i < n; i += nthr) flags[i] = 0;
     block_fill_keys(keys, sf, n, [&](float x, int) { return score_key(x); }, ss, lo, hi);
-    block_kth_largest(keys, n, r.k1, ss, lo, hi, tau, need, n_eq);
-    block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+    if (n <= nthr) {
+      block_mark_topk_small(keys, n, r.k1, flags);
+    } else {
+      block_kth_largest(keys, n, r.k1, ss, lo, hi, tau, need, n_eq);
+      block_mark_selected(keys, n, tau, need, n_eq, flags, ss);
+    }
     block_compact_flags(flags, n, out, ss);
   }
 }

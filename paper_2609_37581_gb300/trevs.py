@@ -83,8 +83,7 @@ _SIGS = {
     "trevs_in_llm_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
     "trevs_in_llm_head_scores": (_c_i32, [_vp, _c_i64, _c_i64, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
                                           _c_i32, _c_i32, _c_i32, _c_f32, _vp, _vp, _vp, _c_sz, _vp]),
-    "trevs_in_llm_select": (_c_i32, [_vp, _c_i64, _c_i64, _vp, _c_i64, _c_i64, _c_i32, _c_i32, _c_i32,
-                                     _c_i32, _c_i32, _c_f32, _vp, _vp, _c_i32, _c_i32, _vp, _vp, _vp,
+    "trevs_in_llm_select": (_c_i32, [_vp, _vp, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp,
                                      _vp, _c_sz, _vp]),
     "trevs_in_llm_compact": (_c_i32, [_vp, _c_i64, _c_i32, _vp, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
                                       _c_i32, _vp, _c_i32, _vp, _c_i64, _vp, _vp, _c_i64, _c_i64, _vp]),
@@ -200,20 +199,19 @@ def trevs_pre_llm_gather(Z, kept_idx, Z_out, stream=None):
                                       _ptr(Z_out), Z_out.stride(0), _stream(stream)))
 
 
-def trevs_in_llm_head_scores(Q, K, Hq, Hkv, L, K1, u_out, row_stats_out, q_strides, k_strides,
+def trevs_in_llm_head_scores(Q, K, Hq, Hkv, L, K1, u_out, attn_out, q_strides, k_strides,
                              scale=0.0, ws=None, stream=None):
     w, nb = _ws_args(ws)
     check(load().trevs_in_llm_head_scores(_ptr(Q), q_strides[0], q_strides[1], _ptr(K), k_strides[0],
                                           k_strides[1], Hq, Hkv, L, K1, HEAD_DIM, scale, _ptr(u_out),
-                                          _ptr(row_stats_out), w, nb, _stream(stream)))
+                                          _ptr(attn_out), w, nb, _stream(stream)))
 
 
-def trevs_in_llm_select(Q, K, Hq, Hkv, L, K1, u, row_stats, n_keep, K2, kept_local, q_strides, k_strides,
-                        heads_out=None, p_out=None, scale=0.0, ws=None, stream=None):
+def trevs_in_llm_select(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=None, p_out=None, ws=None,
+                        stream=None):
     w, nb = _ws_args(ws)
-    check(load().trevs_in_llm_select(_ptr(Q), q_strides[0], q_strides[1], _ptr(K), k_strides[0], k_strides[1],
-                                     Hq, Hkv, L, K1, HEAD_DIM, scale, _ptr(u), _ptr(row_stats), n_keep, K2,
-                                     _ptr(heads_out), _ptr(p_out), _ptr(kept_local), w, nb, _stream(stream)))
+    check(load().trevs_in_llm_select(_ptr(u), _ptr(attn), Hq, L, K1, n_keep, K2, _ptr(heads_out), _ptr(p_out),
+                                     _ptr(kept_local), w, nb, _stream(stream)))
 
 
 def trevs_in_llm_compact(hidden, Kc, Vc, kept_local, hidden_out, K_out, V_out, Hkv, K1,

@@ -94,8 +94,8 @@ def test_stage2_validation(lib):
     assert hs(32, 32, 32, 4096, 128) == t.TREVS_ERR_UNSUPPORTED        # K1 beyond the limit
     assert hs(32, 32, 0, 64, 128) == t.TREVS_ERR_INVALID_ARGUMENT      # no text rows
     assert hs(256, 32, 32, 64, 128) == t.TREVS_ERR_UNSUPPORTED         # Hq
-    sel = lambda nk, K2: lib.trevs_in_llm_select(FAKE, 4096, 128, FAKE, 8192, 128, 32, 32, 32, 64, 128, 0.0,
-                                                 FAKE, FAKE, nk, K2, None, None, FAKE, FAKE, 1 << 24, None)
+    sel = lambda nk, K2: lib.trevs_in_llm_select(FAKE, FAKE, 32, 32, 64, nk, K2, None, None, FAKE, FAKE, 1 << 24,
+                                                 None)
     assert sel(0, 32) == t.TREVS_ERR_INVALID_ARGUMENT
     assert sel(33, 32) == t.TREVS_ERR_INVALID_ARGUMENT
     assert sel(8, 65) == t.TREVS_ERR_INVALID_ARGUMENT

@@ -103,21 +103,16 @@ def test_single_request_stage2_entry_points_head_major_layout():
     qs, ks = (r.l * 128, 128), (r.k1 * 128, 128)
     ws = T.workspace(T.load().trevs_in_llm_workspace_size(w.hq, r.l, r.k1))
     u = torch.zeros(w.hq, dtype=torch.float32, device="cuda")
-    stats = torch.zeros((w.hq, r.l, 2), dtype=torch.float32, device="cuda")
-    T.trevs_in_llm_head_scores(Q, K, w.hq, w.hkv, r.l, r.k1, u, stats, qs, ks, ws=ws)
+    attn = torch.zeros((w.hq, r.l, r.k1), dtype=torch.float32, device="cuda")
+    T.trevs_in_llm_head_scores(Q, K, w.hq, w.hkv, r.l, r.k1, u, attn, qs, ks, ws=ws)
     ref = O.in_llm_request(w.Q, w.K, w.V, w.hidden, w.n_keep_heads, r.k2)
     H.assert_close(u.cpu().numpy(), ref["u"], H.RTOL, 1e-9, "u")
-    # row statistics: max of the scaled logits and 1 / sum of exp
-    Qf, Kf = O.bf16_bits_to_f64(w.Q), O.bf16_bits_to_f64(w.K)
-    lg = np.einsum("lhd,khd->hlk", Qf, Kf) / math.sqrt(128)
-    mx = lg.max(axis=2)
-    H.assert_close(stats[..., 0].cpu().numpy(), mx, 1e-5, 1e-5, "row max")
-    H.assert_close(stats[..., 1].cpu().numpy(), 1.0 / np.exp(lg - mx[..., None]).sum(axis=2), H.RTOL, 0, "1/sum")
+    A = O.text_to_vision_attention(O.bf16_bits_to_f64(w.Q), O.bf16_bits_to_f64(w.K))
+    H.assert_close(attn.cpu().numpy(), A, H.RTOL, H.ATOL_P, "attention")
     heads = torch.full((w.n_keep_heads,), -1, dtype=torch.int32, device="cuda")
     p = torch.zeros(r.k1, dtype=torch.float32, device="cuda")
     kept = torch.full((r.k2,), -1, dtype=torch.int32, device="cuda")
-    T.trevs_in_llm_select(Q, K, w.hq, w.hkv, r.l, r.k1, u, stats, w.n_keep_heads, r.k2, kept, qs, ks,
-                          heads_out=heads, p_out=p, ws=ws)
+    T.trevs_in_llm_select(u, attn, w.hq, r.l, r.k1, w.n_keep_heads, r.k2, kept, heads_out=heads, p_out=p, ws=ws)
     np.testing.assert_array_equal(heads.cpu().numpy(), ref["heads"])
     H.assert_close(p.cpu().numpy(), ref["p"], H.RTOL, H.ATOL_P, "p")
     if H.boundary_gap(ref["p"], r.k2) >= H.NEAR_TIE:
@@ -134,6 +129,27 @@ def test_single_request_stage2_entry_points_head_major_layout():
     np.testing.assert_array_equal(H.host_u16(hid_out), w.hidden[kk])
     np.testing.assert_array_equal(H.host_u16(K_out), Kh[:, kk])
     np.testing.assert_array_equal(H.host_u16(V_out), Vh[:, kk])
+
+
+def test_stage2_select_exact_on_given_attention():
+    # identical fp32 attention on both sides: H* and the kept set are exact (ties included)
+    rng = np.random.default_rng(5)
+    Hq, L, K1 = 6, 21, 130
+    A = rng.integers(0, 3, size=(Hq, L, K1)).astype(np.float32) / 8
+    u = np.array([0.5, 0.25, 0.5, 0.125, 0.25, 0.5], np.float32)
+    ws = T.workspace(T.load().trevs_in_llm_workspace_size(Hq, L, K1))
+    for nk, K2 in ((3, 40), (2, 130), (6, 1)):
+        kept = torch.full((K2,), -1, dtype=torch.int32, device="cuda")
+        heads = torch.full((nk,), -1, dtype=torch.int32, device="cuda")
+        p = torch.zeros(K1, dtype=torch.float32, device="cuda")
+        T.trevs_in_llm_select(H.dev_f32(u), H.dev_f32(A), Hq, L, K1, nk, K2, kept, heads_out=heads, p_out=p, ws=ws)
+        want_h = O.select_heads(u.astype(np.float64), nk)
+        np.testing.assert_array_equal(heads.cpu().numpy(), want_h)
+        want_p = O.token_scores(A.astype(np.float64), want_h)
+        H.assert_close(p.cpu().numpy(), want_p, 1e-6, 1e-7, "p")
+        # fp32 sums of multiples of 1/8 are exact: the ranking is unique
+        np.testing.assert_array_equal(kept.cpu().numpy(), O.top_k(p.cpu().numpy().astype(np.float64), K2))
+        np.testing.assert_array_equal(kept.cpu().numpy(), O.top_k(want_p, K2))
 
 
 def test_gather_skips_out_of_range_indices():
