@@ -173,6 +173,29 @@ TREVS_API trevs_status trevs_in_llm_select(const float* u, const float* attn, in
                                  float* p_out, int32_t* kept_local,
                                  void* workspace, size_t workspace_bytes, void* stream);
 
+/* Allocation-free form of trevs_in_llm_select: the same H*, Eq. 9 scores and TopK(p, K2),
+ * with the same arguments except the workspace. The paper has no counterpart; this is for
+ * callers that cannot hand the library device memory at the time of the call (a memory
+ * budget fixed at start-up, an allocator closed after warm-up, glue code without a device
+ * allocator). Its scratch is a fixed array inside the library's device image (about 20 KB
+ * per GPU, held until the process exits), sized for K1 <= TREVS_MAX_STAGE2_TOKENS (2048);
+ * a larger K1 returns TREVS_ERR_UNSUPPORTED and launches nothing. The call allocates no
+ * device memory; it clears the part of the array that must start at zero (and p_out when
+ * given) with stream-ordered memsets before its one kernel.
+ * - The first call on each device resolves the array's address on the current device
+ *   (cudaGetSymbolAddress; this also loads the module). Make that first call, on every
+ *   device it will be used on, before capturing the call into a CUDA graph.
+ * - Every call on a device shares the one array: calls that can overlap (on different
+ *   streams without ordering, from several host threads, or several instances of a graph
+ *   running at once) race on it and give wrong results. Order them on one stream.
+ * - Errors: TREVS_ERR_INVALID_ARGUMENT / TREVS_ERR_UNSUPPORTED before any CUDA call,
+ *   TREVS_ERR_CUDA when resolving the array or enqueuing fails; message in
+ *   trevs_last_error_string(). */
+TREVS_API trevs_status trevs_in_llm_select_noalloc(const float* u, const float* attn, int32_t Hq, int32_t L,
+                                         int32_t K1, int32_t n_keep_heads, int32_t K2,
+                                         int32_t* heads_out, float* p_out, int32_t* kept_local,
+                                         void* stream);
+
 /* Compaction at l* (Sec. 4.2): for k < K2 and i = kept_local[k],
  *   hidden_out[k] = hidden[i]                       (d_model bf16 per row)
  *   K_out(g, k, :) = Kc(g, i, :), V_out(g, k, :) = Vc(g, i, :) for g < Hkv (d_h bf16 each).

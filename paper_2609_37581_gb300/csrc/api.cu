@@ -513,6 +513,13 @@ const trevs_pre_params kDefaults = {1.4f, 1.0f, 1.0f, 1e-6f, TREVS_SELECT_RATIO}
 
 }  // namespace
 
+namespace trevs {
+// Lets the other translation units of the library report through trevs_last_error_string
+// and trevs_last_launch_count.
+trevs_status record_error(trevs_status s, const char* msg) { return fail(s, "%s", msg); }
+void record_launches(int n) { g_launches = n; }
+}  // namespace trevs
+
 // ======================================================================== C ABI
 
 extern "C" {

@@ -85,6 +85,8 @@ _SIGS = {
                                           _c_i32, _c_i32, _c_i32, _c_f32, _vp, _vp, _vp, _c_sz, _vp]),
     "trevs_in_llm_select": (_c_i32, [_vp, _vp, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp,
                                      _vp, _c_sz, _vp]),
+    "trevs_in_llm_select_noalloc": (_c_i32, [_vp, _vp, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp,
+                                             _vp]),
     "trevs_in_llm_compact": (_c_i32, [_vp, _c_i64, _c_i32, _vp, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
                                       _c_i32, _vp, _c_i32, _vp, _c_i64, _vp, _vp, _c_i64, _c_i64, _vp]),
     "trevs_pre_llm_varlen_workspace_size": (_c_sz, [ctypes.POINTER(PreBatchC)]),
@@ -212,6 +214,13 @@ def trevs_in_llm_select(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=No
     w, nb = _ws_args(ws)
     check(load().trevs_in_llm_select(_ptr(u), _ptr(attn), Hq, L, K1, n_keep, K2, _ptr(heads_out), _ptr(p_out),
                                      _ptr(kept_local), w, nb, _stream(stream)))
+
+
+def trevs_in_llm_select_noalloc(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=None, p_out=None,
+                                stream=None):
+    """trevs_in_llm_select without a workspace: the library's fixed device scratch is used."""
+    check(load().trevs_in_llm_select_noalloc(_ptr(u), _ptr(attn), Hq, L, K1, n_keep, K2, _ptr(heads_out),
+                                             _ptr(p_out), _ptr(kept_local), _stream(stream)))
 
 
 def trevs_in_llm_compact(hidden, Kc, Vc, kept_local, hidden_out, K_out, V_out, Hkv, K1,

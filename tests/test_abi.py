@@ -99,6 +99,13 @@ def test_stage2_validation(lib):
     assert sel(0, 32) == t.TREVS_ERR_INVALID_ARGUMENT
     assert sel(33, 32) == t.TREVS_ERR_INVALID_ARGUMENT
     assert sel(8, 65) == t.TREVS_ERR_INVALID_ARGUMENT
+    na = lambda K1, nk, K2: lib.trevs_in_llm_select_noalloc(FAKE, FAKE, 32, 32, K1, nk, K2, None, None, FAKE, None)
+    assert na(t.MAX_STAGE2_TOKENS + 1, 8, 8) == t.TREVS_ERR_UNSUPPORTED    # beyond the fixed scratch
+    assert "K1" in _err(lib)
+    assert na(64, 0, 8) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert na(64, 8, 65) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert lib.trevs_in_llm_select_noalloc(FAKE, None, 32, 32, 64, 8, 8, None, None, FAKE,
+                                           None) == t.TREVS_ERR_INVALID_ARGUMENT
     assert lib.trevs_in_llm_compact(FAKE, 4096, 4096, None, None, 0, 0, 1, 128, 64, FAKE, 65, FAKE, 4096,
                                     None, None, 0, 0, None) == t.TREVS_ERR_INVALID_ARGUMENT
     assert lib.trevs_in_llm_compact(FAKE, 4096, 4096, FAKE, None, 0, 0, 1, 128, 64, FAKE, 32, FAKE, 4096,
