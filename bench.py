@@ -326,7 +326,9 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         "roofline": {"bound": "hbm", "kernel": DOMINANT, "achieved": round(achieved, 1), "peak": peak,
                      "peak_source": src, "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "traffic": committed_traffic(), "algorithmic_bytes": nbytes["score_kernel"],
-                     "kernel_us": round(kernel_ms * 1e3, 2)},
+                     "kernel_us": round(kernel_ms * 1e3, 2),
+                     "timed": "CUDA events around a graph of pre_saliency_kernel -> pre_score_kernel "
+                              "(PDL); the saliency kernel reads s_v only"},
         "step_roofline": {"algorithmic_bytes": nbytes["step"],
                           "achieved_gbs": round(nbytes["step"] / (ms * 1e-3) / 1e9, 1),
                           "frac": round(nbytes["step"] / (ms * 1e-3) / 1e9 / peak, 4), "peak_source": src},
