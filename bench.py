@@ -199,6 +199,22 @@ class ClockSampler:
 # ------------------------------------------------------------------ GPU arm
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest of every rank's x (the slowest rank sets the job's time)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(max_elapsed_ms: float, steps: int, tokens_per_rank_step: int, world: int):
+    """(ms per step, whole-job tokens/s) for `world` replicas that each prune their own batch,
+    timed by the slowest rank."""
+    ms = max_elapsed_ms / steps
+    return ms, tokens_per_rank_step * world / (ms * 1e-3)
+
+
 def gpu_arm(args, rank, world, w, cpu_baseline):
     import torch
     from paper_2609_37581_gb300 import trevs as T
@@ -275,9 +291,7 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         kernel_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
 
     if distributed:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+        elapsed_ms = max_over_ranks(elapsed_ms, dev)
 
     # end to end through the public call with host buffers
     e2e = None
@@ -311,14 +325,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
 
     if rank != 0:
         return None
-    ms = elapsed_ms / args.steps
-    tokens_per_step = w.visual_tokens() * world
+    ms, value = replica_throughput(elapsed_ms, args.steps, w.visual_tokens(), world)
     nbytes = algorithmic_bytes(w)
     peak, src = peaks()
     achieved = nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9
     clk = sampler.summary()
     return {
-        "metric": METRIC, "value": tokens_per_step / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
         "us_per_prune": round(ms * 1e3, 2), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic (seeded, LLaVA-1.5-shaped; no dataset)",
