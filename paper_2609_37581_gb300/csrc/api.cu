@@ -12,10 +12,11 @@
 #include "trevs.h"
 
 namespace trevs {
-cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, int max_n, long long z_rows,
-                             long long t_rows, cudaStream_t);
-cudaError_t launch_pre_select(const PreMeta&, const PreArgs&, int max_n, cudaStream_t);
-cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, cudaStream_t);
+cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, long long z_rows, cudaStream_t, bool pdl);
+size_t pre_score_part_bytes(int max_m);
+cudaError_t launch_pre_fixup(const PreMeta&, const PreArgs&, int max_m, cudaStream_t);
+cudaError_t launch_pre_select(const PreMeta&, const PreArgs&, int max_n, cudaStream_t, bool pdl);
+cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
@@ -26,8 +27,10 @@ cudaError_t launch_in_cluster(const InMeta&, const InArgs&, int max_k1, cudaStre
 namespace trevs {
 
 cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes) {
-  // the default limit is 48 KB minus the kernel's static shared memory: always opt in
-  if (bytes <= 0) return cudaSuccess;
+  // Every kernel of the library prefers the largest shared-memory carveout, so that an SM
+  // never has to drain and re-split L1 / shared memory between two of its grids (the scoring
+  // grid needs the largest split and follows the pre-pass closely). The default dynamic limit
+  // is 48 KB minus the kernel's static shared memory: opt in to what a launch asks for.
   struct Entry {
     const void* kernel;
     int device;
@@ -39,16 +42,21 @@ cudaError_t ensure_dynamic_smem_impl(const void* kernel, int bytes) {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lock(mu);
-  for (Entry& x : granted)
-    if (x.kernel == kernel && x.device == dev) {
-      if (x.bytes >= bytes) return cudaSuccess;
-      e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-      if (e == cudaSuccess) x.bytes = bytes;
-      return e;
-    }
-  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e == cudaSuccess) granted.push_back(Entry{kernel, dev, bytes});
-  return e;
+  Entry* x = nullptr;
+  for (Entry& g : granted)
+    if (g.kernel == kernel && g.device == dev) x = &g;
+  if (!x) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    granted.push_back(Entry{kernel, dev, 0});
+    x = &granted.back();
+  }
+  if (bytes > x->bytes) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    x->bytes = bytes;
+  }
+  return cudaSuccess;
 }
 
 // A second stream with fork / join events, created once per (host thread, device), so that
@@ -130,16 +138,20 @@ inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 constexpr size_t kStatusBytes = 256;
 
 struct PreWs {
-  size_t counters, sal, s_t, s_fused, keys, flags, end;
+  size_t counters, sal, t_rinv, part, s_t, s_fused, keys, flags, end;
 };
 
-// Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request.
-PreWs pre_ws(long long total_n) {
+// Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request;
+// t_rinv holds 1 / ||t_j|| of the text rows; part the partial sums of the scoring tiles
+// that two or more scoring CTAs share (up to max_m text rows).
+PreWs pre_ws(long long total_n, long long total_m, int max_m) {
   PreWs w;
   const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
   size_t o = kStatusBytes;
   w.counters = o; o = al256(o + 4 * (size_t)kMaxChunk);
   w.sal = o;      o = al256(o + 16 * (size_t)kMaxChunk);
+  w.t_rinv = o;   o = al256(o + 4 * (size_t)(total_m > 0 ? total_m : 0));
+  w.part = o;     o = al256(o + (total_n > 0 ? pre_score_part_bytes(max_m > 0 ? max_m : 1) : 0));
   w.s_t = o;      o = al256(o + 4 * (size_t)total_n);
   w.s_fused = o;  o = al256(o + 4 * (size_t)total_n);
   w.keys = o;     o = al256(o + 4 * padded);
@@ -210,7 +222,7 @@ trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
     }
     t.n += r.n; t.m += r.m; t.k1 += r.k1;
     t.max_n = r.n > t.max_n ? r.n : t.max_n;
-    t.max_m = r.m > t.max_m ? r.m : t.max_m;
+    if (r.n > 0) t.max_m = r.m > t.max_m ? r.m : t.max_m;   // requests without visual rows score nothing
   }
   TREVS_CHECK(t.n < (1ll << 31) && t.m < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
   if (t.n > 0) {
@@ -258,7 +270,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     tiles += (q.n + kScoreTileRows - 1) / kScoreTileRows;
     no += q.n; mo += q.m; ko += q.k1;
     max_n = q.n > max_n ? q.n : max_n;
-    max_m = q.m > max_m ? q.m : max_m;
+    if (q.n > 0) max_m = q.m > max_m ? q.m : max_m;
   }
   meta.total_tiles = tiles;
   PreArgs a;
@@ -276,13 +288,18 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
   a.sal = reinterpret_cast<int4*>(ws + L.sal);
   a.sal_ready = 1;
+  a.t_rinv = reinterpret_cast<float*>(ws + L.t_rinv);   // chunks run one after the other: rows from 0
+  a.total_m = mo;
+  a.part = reinterpret_cast<float*>(ws + L.part);
   a.err = reinterpret_cast<uint32_t*>(ws);
   a.d = bt->d;
   a.mode = prm.select_mode == TREVS_SELECT_FUSED ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
-  TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, st)), "saliency launch");
-  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, max_n, no, mo, st)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_fixup(meta, a, max_m, st)), "fixup launch");
+  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, max_n, st, true)), "pre_select launch");
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
   if (bt->Z_out && ko > 0) {
@@ -552,7 +569,9 @@ trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream) {
   return TREVS_OK;
 }
 
-size_t trevs_pre_llm_workspace_size(int32_t N) { return N < 0 ? 0 : pre_ws(N).end; }
+size_t trevs_pre_llm_workspace_size(int32_t N) {
+  return N < 0 ? 0 : pre_ws(N, TREVS_MAX_TEXT_TOKENS, TREVS_MAX_TEXT_TOKENS).end;
+}
 
 trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
                                   const uint16_t* T, int64_t t_row_stride, int32_t M, const float* s_v,
@@ -574,7 +593,7 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   PreTotals tot;
   s = validate_pre_batch(&bt, tot);
   if (s != TREVS_OK) return s;
-  const PreWs L = pre_ws(N);
+  const PreWs L = pre_ws(N, TREVS_MAX_TEXT_TOKENS, TREVS_MAX_TEXT_TOKENS);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
@@ -591,11 +610,18 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   a.flags = ws + L.flags; a.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
   a.counters = reinterpret_cast<uint32_t*>(ws + L.counters);
   a.sal = reinterpret_cast<int4*>(ws + L.sal);
+  a.t_rinv = reinterpret_cast<float*>(ws + L.t_rinv);
+  a.total_m = M;
+  a.part = reinterpret_cast<float*>(ws + L.part);
   a.err = reinterpret_cast<uint32_t*>(ws);
   a.d = d; a.mode = s_fused_out ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = s_fused_out ? kActScoresFused : kActScores;
-  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, N, M, (cudaStream_t)stream)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, (cudaStream_t)stream)), "pre-pass launch");
+  TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream, true)), "pre_score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_fixup(meta, a, M, (cudaStream_t)stream)), "fixup launch");
+  if (s_fused_out)
+    TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream, true)), "fused-score launch");
   return TREVS_OK;
 }
 
@@ -614,7 +640,7 @@ trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const floa
   const bool fused = prm.select_mode == TREVS_SELECT_FUSED;
   if (fused && !s_fused) TREVS_CHECK(s_v && s_t, "fused mode needs s_fused or both s_v and s_t");
   if (!fused) TREVS_CHECK(s_v && s_t, "ratio mode needs s_v and s_t");
-  const PreWs L = pre_ws(N);
+  const PreWs L = pre_ws(N, TREVS_MAX_TEXT_TOKENS, TREVS_MAX_TEXT_TOKENS);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
@@ -635,7 +661,7 @@ trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const floa
   a.mode = fused ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
-  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream)), "pre_select launch");
+  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream, false)), "pre_select launch");
   return TREVS_OK;
 }
 
@@ -789,9 +815,15 @@ trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_str
 
 size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
-  long long n = 0;
-  for (int b = 0; b < batch->B; ++b) n += batch->reqs[b].n > 0 ? batch->reqs[b].n : 0;
-  return pre_ws(n).end;
+  long long n = 0, m = 0;
+  int max_m = 0;
+  for (int b = 0; b < batch->B; ++b) {
+    const trevs_pre_request& r = batch->reqs[b];
+    n += r.n > 0 ? r.n : 0;
+    m += r.m > 0 ? r.m : 0;
+    if (r.n > 0 && r.m > max_m) max_m = r.m;
+  }
+  return pre_ws(n, m, max_m).end;
 }
 
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
@@ -818,7 +850,7 @@ trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_
   PreTotals t;
   s = validate_pre_batch(batch, t);
   if (s != TREVS_OK || batch->B == 0) return s;
-  const PreWs L = pre_ws(t.n);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -848,7 +880,7 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   s = validate_in_batch(in, ti);
   if (s != TREVS_OK) return s;
-  const PreWs LP = pre_ws(tp.n);
+  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
   const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);

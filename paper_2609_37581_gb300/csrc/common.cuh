@@ -19,12 +19,12 @@ struct PreReq {
   int m_off, m;     // text rows of T
   int k1_off, k1;   // kept rows of kept_idx / Z_out
   int kt;           // textual share K_t of the keep budget (Sec. 3.1)
-  int tile_off;     // first score tile of this request
+  int tile_off;     // first 128-row scoring tile of this request
 };
 
 struct PreMeta {
   int B;
-  int total_tiles;
+  int total_tiles;  // 128-row scoring tiles over all requests (the last of a request may be short)
   PreReq r[kMaxChunk];
 };
 
@@ -387,6 +387,8 @@ __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepc
 template <class... KArgs, class... Args>
 inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                                  bool pdl, Args... args) {
+  const cudaError_t e = ensure_dynamic_smem(kernel, (int)smem);   // carveout, dynamic limit
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;

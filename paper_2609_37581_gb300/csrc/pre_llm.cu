@@ -7,240 +7,499 @@ namespace trevs {
 
 // ------------------------------------------------------------------ scoring contraction
 //
-// One CTA scores a tile of 128 visual rows of one request against the M text rows of that
-// request. G = Z_tile . T^T runs on the 5th-generation tensor cores: TMA streams 64-column
-// chunks of Z and T into a ring of 128-byte-swizzled shared-memory stages, one thread
-// issues UMMA (M = 128, N = M rounded up to 16, K = 16 per instruction) into a TMEM
-// accumulator, and four warps compute the fp32 squared norms ||z_i||^2, ||t_j||^2 from the
-// same stages. The epilogue reads the accumulator row by row from TMEM and forms
-// m_ji = max(G_ji / (||t_j|| ||z_i||), 0) and s^t_i = sqrt(sum_j m_ji^2 / M); the [M, N]
-// similarity never reaches memory. The last tile of a request to finish (ticket counter,
-// no waiting) runs that request's selection.
+// A persistent grid, one CTA per SM, scores the visual rows of every request against the M
+// text rows of that request. Each request is cut into tiles of 128 rows (its last tile may
+// be shorter), and each tile into Z stages of 256 columns. Work is counted in (tile, stage)
+// units, tile by tile; CTA c takes the contiguous units [W c / P, W (c + 1) / P), so that
+// every CTA streams the same number of stages. A tile whose stages are split between CTAs
+// leaves partial sums of G and ||z||^2 in the workspace (at most two per CTA: where its
+// range starts and where it ends), and pre_fixup_kernel adds them up in stage order.
 //
-// Warp roles: 0 = TMA producer, 1 = TMEM owner and MMA issuer, 2..7 = squared norms of the
-// 128 Z rows and the M T rows of every stage (row units spread over 192 threads, four
-// independent accumulators each); 2..5 then run the epilogue (warp w reads TMEM lanes
-// 32*(w%4) .. 32*(w%4)+31, i.e. those tile rows). All eight warps run the selection.
+// For each sub-tile the 5th-generation tensor cores compute G = Z_sub . T^T (UMMA M = 128,
+// N = M_b rounded up to 16) into one of two TMEM accumulators, while eight warps sum the
+// squares ||z_i||^2 from the same shared-memory stages. Four epilogue warps read a finished
+// accumulator while the next sub-tile streams into the other, and form
+// m_ji = max(G_ji / (||t_j|| ||z_i||), 0) and s^t_i = sqrt(sum_j m_ji^2 / M) with 1 / ||t_j||
+// from the pre-pass; the [M, N] similarity never reaches memory. Selection runs in the next
+// grid of the stream.
+//
+// Operands. Z arrives in stages of 128 rows x 256 columns: one 3D TMA box per 8 rows covers
+// four 64-column slices (512 contiguous bytes of each row, 4 KB per copy), which streams HBM
+// at full rate; in shared memory the 1 KB swizzle atoms of one slice lie 4 KB apart, which
+// the UMMA descriptor states as its stride between 8-row groups. The SM's TMA engine is
+// left to Z alone: T (hot in L2) is copied by two warps with cp.async into its own ring, in
+// the same 128-byte swizzled layout, each slot holding 1, 2 or 4 consecutive slices (as many
+// as fit), so that the MMA issuer synchronises once per slot rather than once per slice.
+//
+// Warp roles: 0 = TMA producer (Z), 1 = TMEM owner and MMA issuer, 2..3 = T copies,
+// 4..7 = epilogue (warp w reads TMEM lanes 32*(w%4) .. +31), 8..15 = Z norms (two threads
+// per row, two slices each).
 
 constexpr int kTileRows = kScoreTileRows;
-constexpr int kChunk = 64;                     // d' columns per stage (one 128-byte swizzle row)
-constexpr int kMaxStages = 8;
-constexpr int kZBoxRows = 64;
-constexpr int kTBoxRows = 32;
-constexpr int kZStageBytes = kTileRows * kChunk * 2;
-constexpr int kScoreThreads = 256;
+constexpr int kChunk = 64;                     // d' columns per slice (one 128-byte swizzle row)
+constexpr int kZSlices = 4;                    // slices per Z stage
+constexpr int kZBoxRows = 8;                   // rows per Z copy (one swizzle atom per slice)
+constexpr int kZBoxBytes = kZBoxRows * kZSlices * 128;
+constexpr int kZStageBytes = kTileRows * kZSlices * 128;
+constexpr int kMaxZStages = 4;
+constexpr int kMaxTSlots = 8;
+constexpr int kScoreThreads = 512;
+constexpr int kZNormWarps = 8;
+constexpr int kTCopyThreads = 64;
+constexpr int kRingBudget = 200 * 1024;
 
 struct ScoreLaunch {
-  int stages;
-  int stage_bytes;
-  int tmem_cols;
-  int smem_bytes;   // dynamic shared memory actually requested (for the selection)
+  int z_stages;
+  int t_slots;
+  int t_slot_slices;  // 64-column slices per T slot (1, 2 or 4)
+  int t_slice_bytes;  // bytes of one slice of T in a slot (M rounded up to 16 rows x 128)
+  int acc_cols;       // TMEM columns of one accumulator (power of two >= 32)
+  int mld;            // row length of a partial G (max M rounded up to 4)
 };
 
+// Floats of one partial-sum slot: G [128][mld], then ||z||^2 [128].
+__host__ __device__ inline long long score_slot_floats(int mld) { return (long long)kTileRows * mld + kTileRows; }
+
+struct SubTile {
+  int b, row0, h;   // request, its first row, rows (1..128)
+  int tile;         // tile index over the launch
+  int zs0, zs1;     // Z stages [zs0, zs1) of the tile
+  int slot;         // -1: the whole tile; 0 / 1: partial sums of the range's first / last tile
+};
+
+// Scoring CTA whose stage units [W c / P, W (c + 1) / P) contain unit u (32-bit arithmetic:
+// W * P < 2^31 by construction).
+__host__ __device__ inline int score_cta_of(int u, int W, int P) { return (int)(((long long)(u + 1) * P - 1) / W); }
+
+// Calls f(segment) for the tiles of stage units [u0, u1) in order; f returns false to stop.
+template <class F>
+__device__ __forceinline__ void for_each_subtile(const PreMeta& meta, int nzs, long long u0, long long u1, F f) {
+  if (u0 >= u1) return;
+  int b = find_request(meta.B, (int)(u0 / nzs), [&](int i) { return meta.r[i].tile_off; });
+  for (long long u = u0; u < u1;) {
+    const int t = (int)(u / nzs);
+    const int zs0 = (int)(u - (long long)t * nzs);
+    const int zs1 = (int)min((long long)nzs, zs0 + (u1 - u));
+    while (b + 1 < meta.B && meta.r[b + 1].tile_off <= t) ++b;
+    const PreReq& r = meta.r[b];
+    const int row0 = (t - r.tile_off) * kTileRows;
+    const int slot = (zs0 == 0 && zs1 == nzs) ? -1 : (u == u0 ? 0 : 1);
+    if (!f(SubTile{b, row0, min(kTileRows, r.n - row0), t, zs0, zs1, slot})) return;
+    u += zs1 - zs0;
+  }
+}
+
 __global__ void __launch_bounds__(kScoreThreads, 1)
-    pre_score_kernel(const __grid_constant__ CUtensorMap tmZ, const __grid_constant__ CUtensorMap tmT,
+    pre_score_kernel(const __grid_constant__ CUtensorMap tmZ3, const __grid_constant__ CUtensorMap tmZ2,
                      const __grid_constant__ PreMeta meta, const PreArgs a, const ScoreLaunch L) {
   using namespace sm100;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t acc_bar;
+  __shared__ __align__(8) uint64_t zfull[kMaxZStages], zempty[kMaxZStages];
+  __shared__ __align__(8) uint64_t tfull[kMaxTSlots], tempty[kMaxTSlots];
+  __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], norm_full[2], norm_empty[2];
   __shared__ uint32_t tmem_base_s;
-  __shared__ float rinv_t[256];
-  __shared__ float zsq_s[kTileRows];
-  __shared__ SelShared ss;
-  __shared__ int s_last;
+  __shared__ float rinv_s[4][256];   // one row per epilogue warp (no cross-warp barrier)
+  __shared__ float zsq_s[2][2][kTileRows];   // [buffer][half of the columns][row]
   __shared__ volatile int s_abort;
-  __shared__ volatile int s_issued;
+  __shared__ volatile int s_zissued;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int sel_bytes = L.smem_bytes - (int)(smem - smem_raw);
-  const uint32_t sbase = smem_u32(smem);
+  const uint32_t zbase = smem_u32(smem);
+  const uint32_t tbase = zbase + L.z_stages * kZStageBytes;   // after the Z stages
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int tile = blockIdx.x;
-  const int b = find_request(meta.B, tile, [&](int i) { return meta.r[i].tile_off; });
-  const PreReq r = meta.r[b];
-  const int row0 = (tile - r.tile_off) * kTileRows;
-  const int m = r.m;
-  const int nk = (a.d + kChunk - 1) / kChunk;
-  const int S = L.stages;
-  const int nz_box = (row0 + kZBoxRows < r.n) ? 2 : 1;
-  const int nt_box = (m + kTBoxRows - 1) / kTBoxRows;
-  const int n_mma = (m + 15) & ~15;
-  const uint32_t stage_tx = (uint32_t)(nz_box * kZBoxRows + nt_box * kTBoxRows) * kChunk * 2;
+  const int d = a.d;
+  const int nk = (d + kChunk - 1) / kChunk;                 // 64-column slices
+  const int nzs = (nk + kZSlices - 1) / kZSlices;           // Z stages per tile
+  const long long W = (long long)meta.total_tiles * nzs, P = gridDim.x;
+  const long long u0 = W * blockIdx.x / P, u1 = W * (blockIdx.x + 1) / P;
+  const bool ragged = (d % (kChunk * kZSlices)) != 0;       // last Z stage copied slice by slice
+  const int SZ = L.z_stages, ST = L.t_slots, TS = L.t_slot_slices;
+  const int t_slot_bytes = TS * L.t_slice_bytes;
 
   if (tid == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(smem_u32(&full_bar[s]), 1);
-      mbar_init(smem_u32(&empty_bar[s]), 1 + 6);   // MMA commit + six norm warps
+    for (int s = 0; s < SZ; ++s) {
+      mbar_init(smem_u32(&zfull[s]), 1);
+      mbar_init(smem_u32(&zempty[s]), 1 + kZNormWarps);   // MMA commit + the Z-norm warps
     }
-    mbar_init(smem_u32(&acc_bar), 1);
+    for (int s = 0; s < ST; ++s) {
+      mbar_init(smem_u32(&tfull[s]), kTCopyThreads);      // the copy lanes, once their copies land
+      mbar_init(smem_u32(&tempty[s]), 1);                 // MMA commit
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&acc_full[i]), 1);
+      mbar_init(smem_u32(&acc_empty[i]), 4);              // the epilogue warps
+      mbar_init(smem_u32(&norm_full[i]), kZNormWarps);
+      mbar_init(smem_u32(&norm_empty[i]), 4);
+    }
     s_abort = 0;
-    s_issued = 0;
+    s_zissued = 0;
     mbar_fence_init();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&tmem_base_s), (uint32_t)L.tmem_cols);
+    tmem_alloc(smem_u32(&tmem_base_s), (uint32_t)(2 * L.acc_cols));
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
-  pdl_launch_dependents();   // later grids of the stream may start launching
+  pdl_launch_dependents();   // the selection grid may start launching
 
   if (warp == 0) {
     if (lane == 0) {
-      tma_prefetch_desc(&tmZ);
-      tma_prefetch_desc(&tmT);
+      tma_prefetch_desc(&tmZ3);
+      tma_prefetch_desc(&tmZ2);
       const uint64_t pz = l2_policy_evict_first();   // Z is streamed once
-      const uint64_t pt = l2_policy_evict_last();    // T is re-read by every tile of the request
-      for (int kc = 0; kc < nk; ++kc) {
-        const int s = kc % S, it = kc / S;
-        if (kc >= S && !mbar_wait(smem_u32(&empty_bar[s]), (it - 1) & 1, &s_abort)) {
-          s_abort = 1;
-          break;
+      int gz = 0;
+      for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& t) {
+        const PreReq& r = meta.r[t.b];
+        const int nzb = (t.h + kZBoxRows - 1) / kZBoxRows;
+        const int y0 = r.n_off + t.row0;
+        for (int zs = t.zs0; zs < t.zs1; ++zs, ++gz) {
+          const int s = gz % SZ, it = gz / SZ;
+          if (gz >= SZ && !mbar_wait(smem_u32(&zempty[s]), (it - 1) & 1, &s_abort)) {
+            s_abort = 1;
+            return false;
+          }
+          const uint32_t A = zbase + s * kZStageBytes;
+          const uint32_t fb = smem_u32(&zfull[s]);
+          const int k0 = zs * kZSlices;
+          const int ns = min(kZSlices, nk - k0);
+          if (!(ragged && zs == nzs - 1)) {
+            mbar_arrive_expect_tx(fb, (uint32_t)(nzb * kZBoxBytes));
+            for (int zb = 0; zb < nzb; ++zb) tma_load_3d(A + zb * kZBoxBytes, &tmZ3, 0, y0 + zb * kZBoxRows, k0, fb, pz);
+          } else {
+            // last, partial stage: slice by slice from the 2D map (zero fill beyond d')
+            mbar_arrive_expect_tx(fb, (uint32_t)(nzb * ns * kZBoxRows * 128));
+            for (int zb = 0; zb < nzb; ++zb)
+              for (int c = 0; c < ns; ++c)
+                tma_load_2d(A + zb * kZBoxBytes + c * 1024, &tmZ2, (k0 + c) * kChunk, y0 + zb * kZBoxRows, fb, pz);
+          }
+          s_zissued = gz + 1;
         }
-        const uint32_t A = sbase + s * L.stage_bytes, B = A + kZStageBytes;
-        const uint32_t fb = smem_u32(&full_bar[s]);
-        mbar_arrive_expect_tx(fb, stage_tx);
-        const int x = kc * kChunk;
-        tma_load_2d(A, &tmZ, x, r.n_off + row0, fb, pz);
-        if (nz_box == 2) tma_load_2d(A + kZBoxRows * 128, &tmZ, x, r.n_off + row0 + kZBoxRows, fb, pz);
-        for (int tb = 0; tb < nt_box; ++tb) tma_load_2d(B + tb * kTBoxRows * 128, &tmT, x, r.m_off + tb * kTBoxRows, fb, pt);
-        s_issued = kc + 1;
-      }
+        return true;
+      });
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(kTileRows, n_mma);
-      for (int kc = 0; kc < nk; ++kc) {
-        const int s = kc % S, it = kc / S;
-        if (!mbar_wait(smem_u32(&full_bar[s]), it & 1, &s_abort)) {
+      int gz = 0, gt = 0, j = 0;
+      for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& t) {
+        const int buf = j & 1, use = j >> 1;
+        if (j >= 2 && !mbar_wait(smem_u32(&acc_empty[buf]), (use - 1) & 1, &s_abort)) {
           s_abort = 1;
-          break;
+          return false;
         }
         tc_fence_after();
-        const uint32_t A = sbase + s * L.stage_bytes, B = A + kZStageBytes;
+        const uint32_t dg = tmem + (uint32_t)(buf * L.acc_cols);
+        const uint32_t idesc = umma_idesc_bf16(kTileRows, (meta.r[t.b].m + 15) & ~15);
+        int kc = 0;   // slice index within the sub-tile
+        for (int zs = t.zs0; zs < t.zs1; ++zs, ++gz) {
+          const int s = gz % SZ, it = gz / SZ;
+          if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort)) {
+            s_abort = 1;
+            return false;
+          }
+          const uint32_t A = zbase + s * kZStageBytes;
+          const int ns = min(kZSlices, nk - zs * kZSlices);
+          for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
+            const int ts = gt % ST, tit = gt / ST;
+            if (!mbar_wait(smem_u32(&tfull[ts]), tit & 1, &s_abort)) {
+              s_abort = 1;
+              return false;
+            }
+            fence_proxy_async_smem();   // the slot was written by cp.async (generic proxy)
+            tc_fence_after();
+            const uint32_t B = tbase + ts * t_slot_bytes;
+            const int nsl = min(TS, ns - c0);
+            for (int c = 0; c < nsl; ++c, ++kc) {
 #pragma unroll
-        for (int k = 0; k < kChunk / 16; ++k)
-          umma_bf16(tmem, umma_desc_sw128(A + 32 * k), umma_desc_sw128(B + 32 * k), idesc, (kc | k) != 0);
-        umma_commit(smem_u32(&empty_bar[s]));   // frees the stage once these MMAs have read it
-      }
-      umma_commit(smem_u32(&acc_bar));          // accumulator complete (also on abort)
+              for (int k = 0; k < kChunk / 16; ++k)
+                umma_bf16(dg, umma_desc_sw128(A + (c0 + c) * 1024 + 32 * k, kZSlices * 1024),
+                          umma_desc_sw128(B + c * L.t_slice_bytes + 32 * k), idesc, (kc | k) != 0);
+            }
+            umma_commit(smem_u32(&tempty[ts]));   // frees the T slot once these MMAs have read it
+          }
+          umma_commit(smem_u32(&zempty[s]));      // and the Z stage
+        }
+        umma_commit(smem_u32(&acc_full[buf]));    // this sub-tile's accumulator is complete
+        ++j;
+        return true;
+      });
     }
-  } else {
-    // row units u = t, t + 192 (t = tid - 64; 128 + M <= 384): u < 128 is Z row u, else T row u - 128
-    const int t = tid - 64;
-    const int units = kTileRows + m;
-    float acc[2][4];
-#pragma unroll
-    for (int x = 0; x < 2; ++x)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) acc[x][j] = 0.f;
-    for (int kc = 0; kc < nk; ++kc) {
-      const int s = kc % S, it = kc / S;
-      if (!mbar_wait(smem_u32(&full_bar[s]), it & 1, &s_abort)) {
-        s_abort = 1;
-        break;
-      }
-      const uint8_t* A = smem + s * L.stage_bytes;
-#pragma unroll
-      for (int x = 0; x < 2; ++x) {
-        const int u = t + 192 * x;
-        if (u < units) {
-          // T row u - 128 sits right after the 128 Z rows of the stage
-          const uint8_t* rowp = A + u * 128;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) bf16_sq_acc8(*reinterpret_cast<const uint4*>(rowp + (swz(u, j) << 4)), acc[x]);
+  } else if (warp < 4) {
+    // T copies: the slices of the next slot from the request's M text rows, piece p = 16
+    // bytes (row p / 8, 16-byte column p % 8 of a slice), swizzled like a TMA
+    // 128-byte-swizzle box; slice c of a slot lies t_slice_bytes after slice c - 1
+    const int ct = tid - 64;
+    int gt = 0;
+    for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
+      const PreReq& r = meta.r[st.b];
+      const int pieces = r.m * 8;
+      const uint8_t* tsrc = reinterpret_cast<const uint8_t*>(a.T + (long long)r.m_off * a.t_stride);
+      for (int zs = st.zs0; zs < st.zs1; ++zs) {
+        const int ns = min(kZSlices, nk - zs * kZSlices);
+        for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
+          const int ts = gt % ST, tit = gt / ST;
+          if (gt >= ST && !mbar_wait(smem_u32(&tempty[ts]), (tit - 1) & 1, &s_abort)) {
+            s_abort = 1;
+            return false;
+          }
+          const uint32_t B = tbase + ts * t_slot_bytes;
+          const int nsl = min(TS, ns - c0);
+          for (int c = 0; c < nsl; ++c) {
+            const int kc = zs * kZSlices + c0 + c;
+            const uint32_t Bc = B + c * L.t_slice_bytes;
+            for (int p = ct; p < pieces; p += kTCopyThreads) {
+              const int row = p >> 3, q = p & 7;
+              const int col = kc * kChunk + q * 8;
+              const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
+              cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, col < d ? 16 : 0);   // zero past d'
+            }
+          }
+          cp_async_arrive_noinc(smem_u32(&tfull[ts]));
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&empty_bar[s]));
-    }
+      return true;
+    });
+    cp_async_wait_all();
+  } else if (warp >= 8) {
+    // Z norms: thread zt owns row zt % 128 of every sub-tile, slices 2 (zt / 128) and + 1 of
+    // every stage
+    const int zt = tid - 256;
+    const int row = zt & (kTileRows - 1), half = zt >> 7;
+    int gz = 0, j = 0;
+    for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
+      const int buf = j & 1, use = j >> 1;
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      const bool mine = row < st.h;
+      for (int zs = st.zs0; zs < st.zs1; ++zs, ++gz) {
+        const int s = gz % SZ, it = gz / SZ;
+        if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort)) {
+          s_abort = 1;
+          return false;
+        }
+        if (mine) {
+          const uint8_t* rowp = smem + s * kZStageBytes + (row >> 3) * kZBoxBytes + (row & 7) * 128;
+          const int ncols = min(kZSlices * kChunk, d - zs * kZSlices * kChunk);   // columns of this stage
 #pragma unroll
-    for (int x = 0; x < 2; ++x) {
-      const int u = t + 192 * x;
-      const float sq = (acc[x][0] + acc[x][1]) + (acc[x][2] + acc[x][3]);
-      if (u < kTileRows) zsq_s[u] = sq;
-      else if (u < units) rinv_t[u - kTileRows] = sq > 0.f ? 1.0f / sqrtf(sq) : 0.f;
-    }
-    asm volatile("bar.sync 1, 192;" ::: "memory");   // the six norm warps
-  }
-  if (warp >= 2 && warp < 6) {
-    const int q = warp & 3;             // TMEM lane quarter of this warp
-    const int row = 32 * q + lane;      // tile row owned by this thread
-    const float zacc = zsq_s[row];
-    bool ok = mbar_wait(smem_u32(&acc_bar), 0, &s_abort);
-    ok = __all_sync(0xffffffffu, ok && !s_abort);
-    tc_fence_after();
-    if (ok) {
-      const float rz = zacc > 0.f ? 1.0f / sqrtf(zacc) : 0.f;
-      float sum = 0.f;
-      for (int c0 = 0; c0 < m; c0 += 32) {
-        float v[32];
-        tmem_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0, v);
+          for (int c = 2 * half; c < 2 * half + 2; ++c) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          if (c0 + j < m) {
-            const float x = fmaxf(v[j] * rinv_t[c0 + j] * rz, 0.f);
-            sum = fmaf(x, x, sum);
+            for (int qq = 0; qq < 8; ++qq) {
+              if (c * kChunk + qq * 8 < ncols)   // d' is a multiple of 8: whole 16-byte pieces
+                bf16_sq_acc8(*reinterpret_cast<const uint4*>(rowp + c * 1024 + (swz(row, qq) << 4)), acc);
+            }
           }
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&zempty[s]));
       }
-      if (row0 + row < r.n) a.s_t[r.n_off + row0 + row] = sqrtf(sum / (float)m);
-    }
-    tc_fence_before();
+      if (j >= 2 && !mbar_wait(smem_u32(&norm_empty[buf]), (use - 1) & 1, &s_abort)) {
+        s_abort = 1;
+        return false;
+      }
+      zsq_s[buf][half][row] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&norm_full[buf]));
+      ++j;
+      return true;
+    });
+  } else {
+    const int q = warp & 3;             // TMEM lane quarter of this warp
+    const int row = 32 * q + lane;      // sub-tile row owned by this thread
+    float* rt = rinv_s[q];
+    pdl_wait();                         // 1 / ||t|| come from the pre-pass
+    int j = 0;
+    for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
+      const PreReq& r = meta.r[st.b];
+      const int m = r.m;
+      const int buf = j & 1, use = j >> 1;
+      __syncwarp();
+      for (int c = lane; c < m; c += 32) rt[c] = __ldcg(a.t_rinv + r.m_off + c);
+      __syncwarp();
+      bool ok = mbar_wait(smem_u32(&acc_full[buf]), use & 1, &s_abort);
+      ok = ok && mbar_wait(smem_u32(&norm_full[buf]), use & 1, &s_abort);
+      ok = __all_sync(0xffffffffu, ok && !s_abort);
+      if (!ok) {
+        s_abort = 1;
+        return false;
+      }
+      tc_fence_after();
+      const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * L.acc_cols);
+      const float zsq = zsq_s[buf][0][row] + zsq_s[buf][1][row];
+      const float rz = zsq > 0.f ? 1.0f / sqrtf(zsq) : 0.f;
+      float sum = 0.f;
+      if (st.slot < 0) {
+        for (int c0 = 0; c0 < m; c0 += 32) {
+          float v[32];
+          tmem_ld_32x32b_x32(lane_base + (uint32_t)c0, v);
+#pragma unroll
+          for (int jj = 0; jj < 32; ++jj) {
+            if (c0 + jj < m) {
+              const float x = fmaxf(v[jj] * rt[c0 + jj] * rz, 0.f);
+              sum = fmaf(x, x, sum);
+            }
+          }
+        }
+      } else {
+        // A tile split between CTAs: leave this CTA's partial sums (G row, columns
+        // 0 .. round_up(m, 4), and ||z||^2) in its slot for pre_fixup_kernel.
+        const long long sf = score_slot_floats(L.mld);
+        float* own = a.part + (2 * (long long)blockIdx.x + st.slot) * sf;
+        float* g = own + (long long)row * L.mld;
+        for (int c0 = 0; c0 < m; c0 += 32) {
+          float v[32];
+          tmem_ld_32x32b_x32(lane_base + (uint32_t)c0, v);
+#pragma unroll
+          for (int jj = 0; jj < 32; jj += 4)
+            if (c0 + jj < m) *reinterpret_cast<float4*>(g + c0 + jj) = make_float4(v[jj], v[jj + 1], v[jj + 2], v[jj + 3]);
+        }
+        own[(long long)kTileRows * L.mld + row] = zsq;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(smem_u32(&acc_empty[buf]));
+        mbar_arrive(smem_u32(&norm_empty[buf]));
+      }
+      if (st.slot < 0 && row < st.h) a.s_t[r.n_off + st.row0 + row] = sqrtf(sum / (float)m);
+      ++j;
+      return true;
+    });
   }
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, (uint32_t)L.tmem_cols);
+    tmem_dealloc(tmem, (uint32_t)(2 * L.acc_cols));
   }
   if (s_abort) {
     // let the copies already issued land before the block's shared memory is released
     if (tid == 0) {
-      const int issued = s_issued;
       const volatile int no_abort = 0;
-      for (int kc = issued - S > 0 ? issued - S : 0; kc < issued; ++kc)
-        mbar_wait(smem_u32(&full_bar[kc % S]), (kc / S) & 1, &no_abort, 500000000ull);
+      const int zi = s_zissued;
+      for (int g = zi - SZ > 0 ? zi - SZ : 0; g < zi; ++g)
+        mbar_wait(smem_u32(&zfull[g % SZ]), (g / SZ) & 1, &no_abort, 500000000ull);
       atomicOr(a.err, 1u);
     }
     return;
   }
-
-  if (a.action == kActScores) return;
-  // last finished tile of this request runs its selection
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    const unsigned ntiles = (unsigned)((r.n + kTileRows - 1) / kTileRows);
-    const unsigned prev = atomicAdd(&a.counters[b], 1u);
-    s_last = (prev == ntiles - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (tid == 0) a.counters[b] = 0u;
-  select_request(a, r, b, smem, sel_bytes, ss, a.mode == kModeFused, a.action == kActSelect);
 }
 
-// One CTA per request: selection from scores already in memory.
+// One CTA per tile split between scoring CTAs: s^t of its rows from the partial sums its
+// contributors left, added in stage order. The host lists the split tiles (tile, request,
+// first contributor, contributor count, slot of the first contributor). Thread (row, q)
+// adds column groups q, q + 4, ... of one row with all of a pass's loads in flight (the data
+// sit in L2; dependent round trips would dominate), and the four partial row sums meet in
+// shared memory.
+constexpr int kFixupThreads = 4 * kTileRows;
+struct FixJob {
+  int tile, b, c0, nc, slot0;
+};
+struct FixMeta {
+  int njobs, mld;
+  FixJob job[kMaxScoreCtas];
+};
+__global__ void __launch_bounds__(kFixupThreads, 1) pre_fixup_kernel(const __grid_constant__ PreMeta meta,
+                                                                     const __grid_constant__ FixMeta fm,
+                                                                     const PreArgs a) {
+  __shared__ float red[4][kTileRows];
+  __shared__ float rt[256];
+  const FixJob& jb = fm.job[blockIdx.x];
+  const PreReq& r = meta.r[jb.b];
+  const int mld = fm.mld;
+  const int row0 = (jb.tile - r.tile_off) * kTileRows;
+  const int h = min(kTileRows, r.n - row0);
+  const int m = r.m;
+  const int row = threadIdx.x & (kTileRows - 1), q = threadIdx.x >> 7;
+  const long long sf = score_slot_floats(mld);
+  const float* p0 = a.part + (2 * (long long)jb.c0 + jb.slot0) * sf;
+  pdl_wait();   // the partial sums come from the scoring grid (1 / ||t|| from before it)
+  for (int j = threadIdx.x; j < m; j += kFixupThreads) rt[j] = __ldcg(a.t_rinv + r.m_off + j);
+  __syncthreads();
+  const int ng = (m + 3) >> 2;
+  float sum = 0.f;
+  for (int g0 = q; g0 < ng; g0 += 16) {            // up to four groups of this thread per pass
+    float4 acc[4];
+    float zsq = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k0 = 0; k0 < jb.nc; k0 += 2) {         // two contributors' loads in flight at a time
+      float4 v[2][4];
+      float zv[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int x = k0 + k;
+        const float* base = x == 0 ? p0 : a.part + 2 * (long long)(jb.c0 + x) * sf;
+        const bool live = x < jb.nc;
+        zv[k] = live ? __ldcg(base + (long long)kTileRows * mld + row) : 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int g = g0 + 4 * i;
+          v[k][i] = (live && g < ng) ? __ldcg(reinterpret_cast<const float4*>(base + (long long)row * mld + 4 * g))
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {                 // stage order: contributor c0 first
+        zsq += zv[k];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          acc[i].x += v[k][i].x; acc[i].y += v[k][i].y; acc[i].z += v[k][i].z; acc[i].w += v[k][i].w;
+        }
+      }
+    }
+    const float rz = zsq > 0.f ? 1.0f / sqrtf(zsq) : 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int g = g0 + 4 * i;
+      const float gv[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (4 * g + e < m) {
+          const float xx = fmaxf(gv[e] * rt[4 * g + e] * rz, 0.f);
+          sum = fmaf(xx, xx, sum);
+        }
+      }
+    }
+  }
+  red[q][row] = sum;
+  __syncthreads();
+  if (q == 0 && row < h)
+    a.s_t[r.n_off + row0 + row] = sqrtf(((red[0][row] + red[1][row]) + (red[2][row] + red[3][row])) / (float)m);
+}
+
+// One CTA per request: selection from scores already in memory (action kActSelect), or only
+// the Eq. 6-7 fused scores (kActScoresFused).
 __global__ void __launch_bounds__(512) pre_select_kernel(const __grid_constant__ PreMeta meta,
                                                          const PreArgs a, int smem_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ SelShared ss;
+  pdl_wait();   // the scores come from the preceding grid
   const PreReq r = meta.r[blockIdx.x];
-  select_request(a, r, blockIdx.x, smem, smem_bytes, ss, a.mode == kModeFused && !a.s_fused_given, true);
+  select_request(a, r, blockIdx.x, smem, smem_bytes, ss, a.mode == kModeFused && !a.s_fused_given,
+                 a.action == kActSelect);
 }
 
-// One CTA per request: the saliency side of the selection (inputs only), run ahead of the
-// scoring grid so that the last tile of a request only ranks textual relevance.
+// Pre-pass, run ahead of the scoring grid. Blocks [0, n_sal): the saliency side of the
+// selection of request b = blockIdx.x (inputs only), so that the selection grid only ranks
+// textual relevance. Remaining blocks: 1 / ||t_j|| of the text rows, one warp per row.
 __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant__ PreMeta meta,
-                                                           const PreArgs a, int smem_bytes) {
+                                                           const PreArgs a, int smem_bytes, int n_sal) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ SelShared ss;
   pdl_launch_dependents();
+  if ((int)blockIdx.x >= n_sal) {
+    const long long row = (long long)(blockIdx.x - n_sal) * 16 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= a.total_m) return;
+    const uint4* t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int p = lane; p < a.d / 8; p += 32) bf16_sq_acc8(__ldg(t + p), acc);
+    float sq = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    if (lane == 0) a.t_rinv[row] = sq > 0.f ? 1.0f / sqrtf(sq) : 0.f;
+    return;
+  }
   const int b = blockIdx.x;
   const PreReq r = meta.r[b];
   const bool in_smem = (size_t)r.n * 4 + 16 <= (size_t)smem_bytes;
@@ -325,51 +584,129 @@ static cudaError_t make_tmap(CUtensorMap* tm, const void* base, long long rows, 
   return res == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, int max_n, long long z_rows,
-                             long long t_rows_total, cudaStream_t st) {
+// The same matrix seen as [cols / 64][rows][64] (only whole 64-column slices): a box of
+// box_rows rows x `slices` consecutive slices lands as `slices` swizzle atoms, 1 KB apart.
+static cudaError_t make_tmap_sliced(CUtensorMap* tm, const void* base, long long rows, int cols, long long stride,
+                                    int box_rows, int slices) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return cudaErrorNotSupported;
+  const int full = cols / kChunk;
+  const cuuint64_t dims[3] = {(cuuint64_t)kChunk, (cuuint64_t)(rows > 0 ? rows : 1), (cuuint64_t)(full > 0 ? full : 1)};
+  const cuuint64_t strides[2] = {(cuuint64_t)stride * 2, (cuuint64_t)kChunk * 2};
+  const cuuint32_t box[3] = {(cuuint32_t)kChunk, (cuuint32_t)box_rows, (cuuint32_t)slices};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult res = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+static int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+// Persistent scoring grid: one CTA per SM, but at least four stage units per CTA.
+static int score_grid(const PreMeta& meta, int d) {
+  const long long nzs = ((d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
+  const long long W = (long long)meta.total_tiles * nzs;
+  long long P = sm_count();
+  if (P > kMaxScoreCtas) P = kMaxScoreCtas;
+  if (P > W / 4) P = W / 4;
+  return P < 1 ? 1 : (int)P;
+}
+
+// pdl: the preceding grid of the stream is the pre-pass, which this grid may overlap.
+cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, long long z_rows, cudaStream_t st,
+                             bool pdl) {
   if (meta.total_tiles == 0) return cudaSuccess;
-  const int t_rows = ((max_m + kTBoxRows - 1) / kTBoxRows) * kTBoxRows;
   ScoreLaunch L;
-  L.stage_bytes = kZStageBytes + t_rows * 128;
-  int stages = (106 * 1024 - 1024) / L.stage_bytes;   // two CTAs per SM
-  if (stages < 3) stages = (200 * 1024) / L.stage_bytes;   // one CTA per SM, deeper ring
-  L.stages = stages > kMaxStages ? kMaxStages : (stages < 2 ? 2 : stages);
+  const int tn = (max_m + 15) & ~15;                 // the MMA reads M rounded up to 16 rows
+  L.t_slice_bytes = tn * 128;
+  L.t_slot_slices = tn <= 64 ? 4 : (tn <= 128 ? 2 : 1);
+  L.z_stages = 2;
+  const int slot_bytes = L.t_slot_slices * L.t_slice_bytes;
+  const int slots = (kRingBudget - L.z_stages * kZStageBytes) / slot_bytes;
+  L.t_slots = slots > kMaxTSlots ? kMaxTSlots : slots;   // >= 2 for every M <= 256
   int cols = 32;
-  while (cols < ((max_m + 15) & ~15)) cols <<= 1;
-  L.tmem_cols = cols;
-  int smem = L.stages * L.stage_bytes + 1024;
-  const int sel = (int)((size_t)max_n * 5 + 16) + 1024;
-  if (a.action != kActScores && sel > smem && sel <= 200 * 1024) smem = sel;
-  L.smem_bytes = smem;
-  CUtensorMap tmZ, tmT;
-  cudaError_t e = make_tmap(&tmZ, a.Z, z_rows, a.d, a.z_stride, kZBoxRows);
+  while (cols < tn) cols <<= 1;
+  L.acc_cols = cols;
+  L.mld = (max_m + 3) & ~3;
+  const int smem = L.z_stages * kZStageBytes + L.t_slots * slot_bytes + 1024;
+  CUtensorMap tmZ3, tmZ2;
+  cudaError_t e = make_tmap_sliced(&tmZ3, a.Z, z_rows, a.d, a.z_stride, kZBoxRows, kZSlices);
   if (e != cudaSuccess) return e;
-  e = make_tmap(&tmT, a.T, t_rows_total, a.d, a.t_stride, kTBoxRows);
+  e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, kZBoxRows);
   if (e != cudaSuccess) return e;
   e = ensure_dynamic_smem(pre_score_kernel, smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(pre_score_kernel, dim3(meta.total_tiles), dim3(kScoreThreads), smem, st, a.sal_ready != 0,
-                       tmZ, tmT, meta, a, L);
+  return launch_kernel(pre_score_kernel, dim3(score_grid(meta, a.d)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
+                       tmZ2, meta, a, L);
 }
 
-cudaError_t launch_pre_saliency(const PreMeta& meta, const PreArgs& a, int max_n, cudaStream_t st) {
-  if (meta.B == 0) return cudaSuccess;
-  int smem = (int)((size_t)max_n * 4 + 16);
-  if (smem > 160 * 1024) smem = 0;   // keys stay in the global scratch
+// Partial sums of the scoring grid launched just before (same meta, d' and max M): the
+// split tiles are listed here, on the host, from the same partition the grid uses.
+cudaError_t launch_pre_fixup(const PreMeta& meta, const PreArgs& a, int max_m, cudaStream_t st) {
+  if (meta.total_tiles == 0) return cudaSuccess;
+  static thread_local FixMeta fm;
+  const int nzs = ((a.d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
+  const int P = score_grid(meta, a.d);
+  const int W = meta.total_tiles * nzs;
+  fm.njobs = 0;
+  fm.mld = (max_m + 3) & ~3;
+  int b = 0;
+  for (int c = 1; c < P; ++c) {
+    const int bc = (int)((long long)W * c / P);
+    if (bc % nzs == 0) continue;
+    const int t = bc / nzs, t_start = t * nzs;
+    const int c0 = score_cta_of(t_start, W, P);
+    if (c0 != c - 1) continue;                       // the tile's first boundary lists it
+    while (b + 1 < meta.B && meta.r[b + 1].tile_off <= t) ++b;
+    FixJob& j = fm.job[fm.njobs++];
+    j.tile = t;
+    j.b = b;
+    j.c0 = c0;
+    j.nc = score_cta_of(t_start + nzs - 1, W, P) - c0 + 1;
+    j.slot0 = (int)((long long)W * c0 / P) < t_start ? 1 : 0;
+  }
+  if (fm.njobs == 0) return cudaSuccess;
+  return launch_kernel(pre_fixup_kernel, dim3(fm.njobs), dim3(kFixupThreads), 0, st, true, meta, fm, a);
+}
+
+// Workspace bytes of the partial sums for up to max_m text rows.
+size_t pre_score_part_bytes(int max_m) {
+  return (size_t)2 * kMaxScoreCtas * (size_t)score_slot_floats((max_m + 3) & ~3) * sizeof(float);
+}
+
+// Pre-pass: the saliency rules of the B requests (when `saliency`) and 1 / ||t_j|| of the
+// launch's text rows.
+cudaError_t launch_pre_saliency(const PreMeta& meta, const PreArgs& a, int max_n, bool saliency, cudaStream_t st) {
+  const int n_sal = saliency ? meta.B : 0;
+  const long long tn_blocks = (a.total_m + 15) / 16;
+  if (n_sal + tn_blocks == 0) return cudaSuccess;
+  int smem = saliency ? (int)((size_t)max_n * 4 + 16) : 0;
+  if (smem > 24 * 1024) smem = 0;   // keys in the global scratch: leave the SM to the scoring grid
   cudaError_t e = ensure_dynamic_smem(pre_saliency_kernel, smem);
   if (e != cudaSuccess) return e;
-  pre_saliency_kernel<<<meta.B, 512, smem, st>>>(meta, a, smem);
+  pre_saliency_kernel<<<(unsigned)(n_sal + tn_blocks), 512, smem, st>>>(meta, a, smem, n_sal);
   return cudaGetLastError();
 }
 
-cudaError_t launch_pre_select(const PreMeta& meta, const PreArgs& a, int max_n, cudaStream_t st) {
+// pdl: the preceding grid of the stream is the scoring grid (the kernel waits for it).
+cudaError_t launch_pre_select(const PreMeta& meta, const PreArgs& a, int max_n, cudaStream_t st, bool pdl) {
   if (meta.B == 0) return cudaSuccess;
   int smem = (int)((size_t)max_n * 5 + 16);
   if (smem > 160 * 1024) smem = 0;   // keys stay in the global scratch
   cudaError_t e = ensure_dynamic_smem(pre_select_kernel, smem);
   if (e != cudaSuccess) return e;
-  pre_select_kernel<<<meta.B, 512, smem, st>>>(meta, a, smem);
-  return cudaGetLastError();
+  return launch_kernel(pre_select_kernel, dim3(meta.B), dim3(512), smem, st, pdl, meta, a, smem);
 }
 
 cudaError_t launch_gather(const GatherMeta& gm, cudaStream_t st, bool pdl) {

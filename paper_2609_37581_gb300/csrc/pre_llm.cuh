@@ -8,7 +8,8 @@ namespace trevs {
 
 enum { kModeRatio = 0, kModeFused = 1 };
 
-constexpr int kScoreTileRows = 128;   // visual rows per scoring CTA (UMMA M)
+constexpr int kScoreTileRows = 128;   // visual rows per scoring tile (UMMA M)
+constexpr int kMaxScoreCtas = 256;    // CTAs of the persistent scoring grid, at most
 enum { kActScores = 0, kActScoresFused = 1, kActSelect = 2 };
 
 struct PreArgs {
@@ -19,6 +20,9 @@ struct PreArgs {
   const float* s_v;
   float* s_t;          // [sum n]
   float* s_fused;      // [sum n] (fused mode)
+  float* t_rinv;       // [sum m] 1 / ||t_j|| (0 for a zero row), from the pre-pass
+  long long total_m;   // text rows of the launch
+  float* part;         // [2 per scoring CTA] partial sums of tiles split between CTAs
   int* kept;           // [sum k1]
   uint8_t* flags;      // [sum n] scratch
   uint32_t* keys;      // [sum n] scratch (used when shared memory is too small)
