@@ -20,8 +20,8 @@ cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool 
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
-bool in_cluster_fits(int Hq, int max_l, int max_k1);
-cudaError_t launch_in_cluster(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+bool in_small_fits(int Hq, int max_l, int max_k1);
+cudaError_t launch_in_small(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
 
 namespace trevs {
@@ -492,8 +492,9 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.hs_finalize = 1;
   a.zero_p = 1;
   a.overlap = overlap ? 1 : 0;
-  if (in_cluster_fits(bt->Hq, max_l, max_k1)) {
-    TREVS_TRY_CUDA(counted(launch_in_cluster(meta, a, max_k1, st)), "fused stage-2 launch");
+  if (in_small_fits(bt->Hq, max_l, max_k1)) {
+    TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
+    ++g_launches;   // two grids
   } else {
     TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
     TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");

@@ -1,10 +1,6 @@
 // Stage 2 (in-LLM at layer l*, Sec. 4.2): text-to-vision attention statistics, head
 // variance (Eq. 8), high-variance head set H*, token scores (Eq. 9), TopK and compaction.
-#include <cooperative_groups.h>
-
 #include "in_llm.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace trevs {
 
@@ -313,245 +309,212 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
   block_compact_flags(flags, n, a.kept_local + r.k2_off, ss);
 }
 
-// ------------------------------------------------------------------ fused stage 2 for small requests
+// ------------------------------------------------------------------ stage 2 for small requests
 //
-// One cluster of 8 CTAs per request (text rows L <= 64, visual tokens K1 <= 128). CTA c owns
-// heads c, c + 8, ... (at most 8). Phase 1: for each of its heads, the logits on the tensor
-// cores and the softmax statistics and Eq. 8 row variances in registers (a quad of lanes
-// holds all keys of two text rows). The CTAs then read each other's u_h through distributed
-// shared memory and agree on H*. Phase 2: each CTA recomputes the logits of its selected
-// heads (ascending) and accumulates their attention probabilities in registers. Phase 3:
-// the keys are split among the CTAs for Eq. 9 (partials summed in CTA order, max over the
-// text rows), CTA 0 collects p and selects TopK(p, K2). Only the results reach global
-// memory; the cluster barriers are hardware barriers of co-resident CTAs.
+// Requests with L <= 64 text rows and K1 <= 128 visual tokens take two grids.
+//
+// in_attn_small_kernel: one block per (request, head). Q_h (64 rows) and K_g (K1 rows) are
+// copied into shared memory once; each warp computes the logits of 16 text rows against all
+// keys on the tensor cores and keeps them in registers (a quad of lanes holds two rows), so
+// the softmax max and sum and the two-pass Eq. 8 row variance need only quad shuffles. The
+// block writes the attention probabilities A_h[q][i] and u_h.
+//
+// in_select_small_kernel: one block per request. H* from u; Eq. 9 p_i = max_q of the mean
+// over H* (heads summed in ascending order) with thread (key i, row group) and every load of
+// a batch in flight; then TopK(p, K2) in shared memory.
 template <int NCH>   // 64-key chunks: K1 <= 64 * NCH
-__global__ void __launch_bounds__(128) in_cluster_kernel(const __grid_constant__ InMeta meta, const InArgs a,
-                                                         int a_ld) {
+__global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constant__ InMeta meta, const InArgs a) {
   constexpr int QR = 64;              // text rows (four m16 tiles, one per warp)
   constexpr int NT = 8;               // n-tiles of a 64-key chunk
-  cg::cluster_group cluster = cg::this_cluster();
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ float s_u[8];
-  __shared__ float s_upart[8][4];
-  __shared__ float2 s_stat[8][QR];    // per own head and row: (max in log2 units, 1 / sum)
-  __shared__ float s_uall[kMaxHeads];
-  __shared__ int s_sel[kMaxHeads];
-  __shared__ int s_heads[kMaxHeads];
-  __shared__ int s_nh;
-  __shared__ uint32_t s_pmax[16];
-  __shared__ float s_p[128];
-  __shared__ uint32_t s_keys[128];
-  __shared__ uint8_t s_flags[128];
-  __shared__ SelShared ss;
+  __shared__ float s_upart[4];
   pdl_wait();                         // Q, K may come from the preceding grid
   pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int c = (int)cluster.block_rank();
-  const int b = blockIdx.x / kClusterCtas;
+  const int b = blockIdx.x / a.Hq, h = blockIdx.x - b * a.Hq;
+  const int g = (h * a.Hkv) / a.Hq;
   const InReq r = meta.r[b];
-  const int L = r.l, K1 = r.k1, Hq = a.Hq;
-  const int nmine = c < Hq ? (Hq - c + kClusterCtas - 1) / kClusterCtas : 0;
-
-  uint8_t* qs = smem;                                   // QR x 256 B
-  uint8_t* ks = smem + QR * kRowBytes;                  // 64 * NCH x 256 B
-  float* pbuf = reinterpret_cast<float*>(smem);         // [QR][a_ld] after phase 2
-  const uint32_t qs_a = smem_u32(qs), ks_a = smem_u32(ks);
-  const float sc = a.scale * 1.4426950408889634f;       // logits in log2 units
-  const float mean = 1.0f / (float)K1;
-  const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
-
-  auto issue = [&](int j) {
-    const int h = c + kClusterCtas * j;
-    const int g = (h * a.Hkv) / Hq;
-    load_rows(qs_a, a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs, a.q_ts, 0, QR, L, tid, 128);
-    load_rows(ks_a, a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs, a.k_ts, 0, 64 * NCH, K1, tid, 128);
-  };
+  const int L = r.l, K1 = r.k1;
+  const uint32_t qs_a = smem_u32(smem), ks_a = qs_a + QR * kRowBytes;
+  load_rows(qs_a, a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs, a.q_ts, 0, QR, L, tid, 128);
+  load_rows(ks_a, a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs, a.k_ts, 0, 64 * NCH, K1, tid, 128);
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
   float acc[NCH][NT][4];
-  // logits of the staged head into acc; the stage is free (and refilled with head `next`) after
-  auto logits = [&](int next) {
-    cp_async_wait<0>();
-    __syncthreads();
+  {
     uint32_t af[8][4];
     load_afrag(qs_a, 16 * warp, lane, af);
 #pragma unroll
     for (int ch = 0; ch < NCH; ++ch) qk_tile<NT>(af, ks_a + ch * 64 * kRowBytes, 0, lane, acc[ch]);
-    __syncthreads();
-    if (next >= 0) issue(next);
-    cp_async_commit();
-  };
-
-  // ---- phase 1: statistics and row variances of this CTA's heads
-  if (nmine > 0) issue(0);
-  cp_async_commit();
-  for (int j = 0; j < nmine; ++j) {
-    logits(j + 1 < nmine ? j + 1 : -1);
-    float mxa = -INFINITY, mxb = -INFINITY;
-#pragma unroll
-    for (int ch = 0; ch < NCH; ++ch)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
-          if (key < K1) {
-            mxa = fmaxf(mxa, acc[ch][nt][e] * sc);
-            mxb = fmaxf(mxb, acc[ch][nt][2 + e] * sc);
-          }
-        }
-#pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
-      mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, o));
-      mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, o));
-    }
-    float sa = 0.f, sb = 0.f;
-#pragma unroll
-    for (int ch = 0; ch < NCH; ++ch)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
-          const float ea = key < K1 ? exp2f(acc[ch][nt][e] * sc - mxa) : 0.f;
-          const float eb = key < K1 ? exp2f(acc[ch][nt][2 + e] * sc - mxb) : 0.f;
-          acc[ch][nt][e] = ea;
-          acc[ch][nt][2 + e] = eb;
-          sa += ea;
-          sb += eb;
-        }
-#pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
-      sa += __shfl_xor_sync(0xffffffffu, sa, o);
-      sb += __shfl_xor_sync(0xffffffffu, sb, o);
-    }
-    const float ia = 1.0f / sa, ib = 1.0f / sb;
-    float va = 0.f, vb = 0.f;
-#pragma unroll
-    for (int ch = 0; ch < NCH; ++ch)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
-          if (key < K1) {
-            const float da = acc[ch][nt][e] * ia - mean, db = acc[ch][nt][2 + e] * ib - mean;
-            va = fmaf(da, da, va);
-            vb = fmaf(db, db, vb);
-          }
-        }
-#pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
-      va += __shfl_xor_sync(0xffffffffu, va, o);
-      vb += __shfl_xor_sync(0xffffffffu, vb, o);
-    }
-    if ((lane & 3) == 0) {
-      s_stat[j][ra] = make_float2(mxa, ia);
-      s_stat[j][rb] = make_float2(mxb, ib);
-    }
-    // Eq. 8 numerator: sum over this warp's valid rows of Var_i A[q, i]
-    float vs = ((lane & 3) == 0) ? ((ra < L ? va : 0.f) + (rb < L ? vb : 0.f)) / (float)K1 : 0.f;
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) vs += __shfl_xor_sync(0xffffffffu, vs, o);
-    if (lane == 0) s_upart[j][warp] = vs;
   }
-  __syncthreads();
-  if (tid < nmine) s_u[tid] = (((s_upart[tid][0] + s_upart[tid][1]) + s_upart[tid][2]) + s_upart[tid][3]) / (float)L;
-  cluster.sync();
-
-  // every CTA gathers all u_h and ranks the heads: H* is the n_keep largest, ties to lower h
-  for (int h = tid; h < Hq; h += 128) s_uall[h] = *cluster.map_shared_rank(&s_u[h / kClusterCtas], h % kClusterCtas);
-  __syncthreads();
-  for (int h = tid; h < Hq; h += 128) {
-    const float uh = s_uall[h];
-    int rank = 0;
-    for (int x = 0; x < Hq; ++x) rank += (s_uall[x] > uh) || (s_uall[x] == uh && x < h);
-    s_sel[h] = rank < a.n_keep;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    int cnt = 0;
-    for (int h = 0; h < Hq && cnt < a.n_keep; ++h)
-      if (s_sel[h]) s_heads[cnt++] = h;
-    s_nh = cnt;
-  }
-  __syncthreads();
-  const int nh = s_nh;
-  if (c == 0) {
-    for (int h = tid; h < Hq; h += 128) a.u[(long long)b * a.u_ld + h] = s_uall[h];
-    if (a.heads_out)
-      for (int x = tid; x < nh; x += 128) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
-  }
-
-  // ---- phase 2: sum of the attention probabilities of this CTA's selected heads
-  int sel[8];
-  int nsel = 0;
-  for (int j = 0; j < nmine; ++j)
-    if (s_sel[c + kClusterCtas * j]) sel[nsel++] = j;
-  float psum[NCH][NT][4];
+  const float sc = a.scale * 1.4426950408889634f;       // logits in log2 units
+  const float mean = 1.0f / (float)K1;
+  const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
+  float mxa = -INFINITY, mxb = -INFINITY;
 #pragma unroll
   for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) psum[ch][nt][e] = 0.f;
-  if (nsel > 0) issue(sel[0]);
-  cp_async_commit();
-  for (int x = 0; x < nsel; ++x) {
-    logits(x + 1 < nsel ? sel[x + 1] : -1);
-    const float2 ta = s_stat[sel[x]][ra], tb = s_stat[sel[x]][rb];
-#pragma unroll
-    for (int ch = 0; ch < NCH; ++ch)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          psum[ch][nt][e] += exp2f(acc[ch][nt][e] * sc - ta.x) * ta.y;
-          psum[ch][nt][2 + e] += exp2f(acc[ch][nt][2 + e] * sc - tb.x) * tb.y;
+      for (int e = 0; e < 2; ++e) {
+        const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
+        if (key < K1) {
+          mxa = fmaxf(mxa, acc[ch][nt][e] * sc);
+          mxb = fmaxf(mxb, acc[ch][nt][2 + e] * sc);
         }
+      }
+#pragma unroll
+  for (int o = 1; o < 4; o <<= 1) {
+    mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, o));
+    mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, o));
   }
-  cp_async_wait<0>();
-  __syncthreads();                                      // the stage is free: it becomes pbuf
+  float sa = 0.f, sb = 0.f;
+#pragma unroll
+  for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int key = 64 * ch + 8 * nt + 2 * (lane & 3) + e;
+        const float ea = key < K1 ? exp2f(acc[ch][nt][e] * sc - mxa) : 0.f;
+        const float eb = key < K1 ? exp2f(acc[ch][nt][2 + e] * sc - mxb) : 0.f;
+        acc[ch][nt][e] = ea;
+        acc[ch][nt][2 + e] = eb;
+        sa += ea;
+        sb += eb;
+      }
+#pragma unroll
+  for (int o = 1; o < 4; o <<= 1) {
+    sa += __shfl_xor_sync(0xffffffffu, sa, o);
+    sb += __shfl_xor_sync(0xffffffffu, sb, o);
+  }
+  const float ia = 1.0f / sa, ib = 1.0f / sb;
+  float* A = a.attn + r.attn_off + (long long)h * L * K1;
+  float va = 0.f, vb = 0.f;
 #pragma unroll
   for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
       const int key = 64 * ch + 8 * nt + 2 * (lane & 3);
-      *reinterpret_cast<float2*>(pbuf + ra * a_ld + key) = make_float2(psum[ch][nt][0], psum[ch][nt][1]);
-      *reinterpret_cast<float2*>(pbuf + rb * a_ld + key) = make_float2(psum[ch][nt][2], psum[ch][nt][3]);
+      const float pa0 = acc[ch][nt][0] * ia, pa1 = acc[ch][nt][1] * ia;
+      const float pb0 = acc[ch][nt][2] * ib, pb1 = acc[ch][nt][3] * ib;
+      if (key < K1) {
+        va = fmaf(pa0 - mean, pa0 - mean, va);
+        vb = fmaf(pb0 - mean, pb0 - mean, vb);
+      }
+      if (key + 1 < K1) {
+        va = fmaf(pa1 - mean, pa1 - mean, va);
+        vb = fmaf(pb1 - mean, pb1 - mean, vb);
+      }
+      if (key < K1) {
+        if (ra < L) {
+          A[(long long)ra * K1 + key] = pa0;
+          if (key + 1 < K1) A[(long long)ra * K1 + key + 1] = pa1;
+        }
+        if (rb < L) {
+          A[(long long)rb * K1 + key] = pb0;
+          if (key + 1 < K1) A[(long long)rb * K1 + key + 1] = pb1;
+        }
+      }
     }
-  if (tid < 16) s_pmax[tid] = 0u;
-  cluster.sync();
+#pragma unroll
+  for (int o = 1; o < 4; o <<= 1) {
+    va += __shfl_xor_sync(0xffffffffu, va, o);
+    vb += __shfl_xor_sync(0xffffffffu, vb, o);
+  }
+  // Eq. 8 numerator: sum over this warp's valid rows of Var_i A[q, i]
+  float vs = ((lane & 3) == 0) ? ((ra < L ? va : 0.f) + (rb < L ? vb : 0.f)) / (float)K1 : 0.f;
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) vs += __shfl_xor_sync(0xffffffffu, vs, o);
+  if (lane == 0) s_upart[warp] = vs;
+  __syncthreads();
+  if (tid == 0) a.u[(long long)b * a.u_ld + h] = (((s_upart[0] + s_upart[1]) + s_upart[2]) + s_upart[3]) / (float)L;
+}
 
-  // ---- phase 3: Eq. 9 for keys i = c + 8m: partials summed in CTA order, max over text rows
-  const int kc = K1 > c ? (K1 - c + kClusterCtas - 1) / kClusterCtas : 0;
-  for (int pair = tid; pair < kc * L; pair += 128) {
-    const int m = pair % kc, q = pair / kc;
-    const int i = c + kClusterCtas * m;
-    float v[kClusterCtas];
-#pragma unroll
-    for (int cc = 0; cc < kClusterCtas; ++cc) v[cc] = *cluster.map_shared_rank(pbuf + q * a_ld + i, cc);
-    float t = 0.f;
-#pragma unroll
-    for (int cc = 0; cc < kClusterCtas; ++cc) t += v[cc];
-    atomicMax(&s_pmax[m], __float_as_uint(t));
+constexpr int kSelThreads = 512;
+__global__ void __launch_bounds__(kSelThreads) in_select_small_kernel(const __grid_constant__ InMeta meta,
+                                                                       const InArgs a) {
+  __shared__ float s_u[kMaxHeads];
+  __shared__ int s_sel[kMaxHeads];
+  __shared__ int s_heads[kMaxHeads];
+  __shared__ int s_nh;
+  __shared__ float s_red[kSelThreads];
+  __shared__ uint32_t s_keys[128];
+  __shared__ uint8_t s_flags[128];
+  __shared__ SelShared ss;
+  pdl_wait();                         // u and the attention probabilities come from the preceding grid
+  pdl_launch_dependents();
+  const int tid = threadIdx.x;
+  const int b = blockIdx.x;
+  const InReq r = meta.r[b];
+  const int L = r.l, K1 = r.k1, Hq = a.Hq;
+  const float* u = a.u + (long long)b * a.u_ld;
+  for (int hh = tid; hh < Hq; hh += kSelThreads) s_u[hh] = __ldcg(u + hh);
+  __syncthreads();
+  for (int hh = tid; hh < Hq; hh += kSelThreads) {   // H*: the n_keep largest u, ties to the lower head
+    const float uh = s_u[hh];
+    int rank = 0;
+    for (int x = 0; x < Hq; ++x) rank += (s_u[x] > uh) || (s_u[x] == uh && x < hh);
+    s_sel[hh] = rank < a.n_keep;
   }
   __syncthreads();
-  if (tid < kc) {
-    const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
-    *cluster.map_shared_rank(&s_p[c + kClusterCtas * tid], 0) = __uint_as_float(s_pmax[tid]) * inv_nh;
+  if (tid == 0) {
+    int cnt = 0;
+    for (int hh = 0; hh < Hq && cnt < a.n_keep; ++hh)
+      if (s_sel[hh]) s_heads[cnt++] = hh;
+    s_nh = cnt;
   }
-  cluster.sync();
-
-  if (c == 0) {
-    for (int i = tid; i < K1; i += 128) {
-      a.p_bits[r.k1_off + i] = __float_as_uint(s_p[i]);
-      s_keys[i] = score_key(s_p[i]);
-      s_flags[i] = 0;
+  __syncthreads();
+  const int nh = s_nh;
+  // thread (key i, row group rg): rows rg, rg + NG, ...; heads four at a time, all loads in flight
+  const int kp = K1 <= 64 ? 64 : 128;
+  const int NG = kSelThreads / kp;
+  const int i = tid % kp, rg = tid / kp;
+  const float* A = a.attn + r.attn_off + i;
+  const long long hstride = (long long)L * K1;
+  float m = 0.f;                      // probabilities are positive: 0 never wins the max
+  if (i < K1) {
+    constexpr int RPT = 16;           // rows per thread at most (L <= 64, NG >= 4)
+    float psum[RPT];
+#pragma unroll
+    for (int j = 0; j < RPT; ++j) psum[j] = 0.f;
+    for (int h0 = 0; h0 < nh; h0 += 4) {
+      float v[4][RPT];
+#pragma unroll
+      for (int x = 0; x < 4; ++x) {
+        const float* Ah = A + (long long)s_heads[min(h0 + x, nh - 1)] * hstride;
+#pragma unroll
+        for (int j = 0; j < RPT; ++j) {
+          const int q = rg + NG * j;
+          v[x][j] = (h0 + x < nh && q < L) ? __ldcg(Ah + (long long)q * K1) : 0.f;
+        }
+      }
+#pragma unroll
+      for (int x = 0; x < 4; ++x)
+#pragma unroll
+        for (int j = 0; j < RPT; ++j) psum[j] += v[x][j];
     }
-    __syncthreads();
-    if (r.k2 > 0) {
-      block_mark_topk_small(s_keys, K1, r.k2, s_flags);
-      block_compact_flags(s_flags, K1, a.kept_local + r.k2_off, ss);
-    }
+#pragma unroll
+    for (int j = 0; j < RPT; ++j) m = fmaxf(m, psum[j]);
+  }
+  s_red[tid] = m;
+  __syncthreads();
+  const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
+  if (tid < K1) {
+    float mx = 0.f;
+    for (int x = 0; x < NG; ++x) mx = fmaxf(mx, s_red[x * kp + tid]);
+    const float p = mx * inv_nh;
+    a.p_bits[r.k1_off + tid] = __float_as_uint(p);
+    s_keys[tid] = score_key(p);
+    s_flags[tid] = 0;
+  }
+  if (a.heads_out)
+    for (int x = tid; x < nh; x += kSelThreads) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
+  __syncthreads();
+  if (r.k2 > 0) {
+    block_mark_topk_small(s_keys, K1, r.k2, s_flags);
+    block_compact_flags(s_flags, K1, a.kept_local + r.k2_off, ss);
   }
 }
 
@@ -582,39 +545,18 @@ cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_k1
   }
 }
 
-// Fused stage 2 on 8-CTA clusters when every request has L <= 64 and K1 <= 128.
-bool in_cluster_fits(int Hq, int max_l, int max_k1) {
-  if (max_l > 64 || max_k1 > 128 || Hq > 64) return false;
-  return true;
-}
+// The two-grid small path when every request has L <= 64 and K1 <= 128.
+bool in_small_fits(int Hq, int max_l, int max_k1) { return max_l <= 64 && max_k1 <= 128 && Hq <= kMaxHeads; }
 
-cudaError_t launch_in_cluster(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
+cudaError_t launch_in_small(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
   if (meta.B == 0) return cudaSuccess;
   const int nch = max_k1 <= 64 ? 1 : 2;
-  const int a_ld = 64 * nch + 8;
-  int smem = 64 * kRowBytes + 64 * nch * kRowBytes;     // one Q / K stage, later the partial sums
-  if (64 * a_ld * 4 > smem) smem = 64 * a_ld * 4;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(meta.B * kClusterCtas);
-  cfg.blockDim = dim3(128);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kClusterCtas;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e;
-  if (nch == 1) {
-    e = ensure_dynamic_smem(in_cluster_kernel<1>, smem);
-    if (e != cudaSuccess) return e;
-    return cudaLaunchKernelEx(&cfg, in_cluster_kernel<1>, meta, a, a_ld);
-  }
-  e = ensure_dynamic_smem(in_cluster_kernel<2>, smem);
+  const int smem = 64 * kRowBytes + 64 * nch * kRowBytes;
+  const dim3 grid((unsigned)(meta.B * a.Hq));
+  cudaError_t e = nch == 1 ? launch_kernel(in_attn_small_kernel<1>, grid, dim3(128), smem, st, true, meta, a)
+                           : launch_kernel(in_attn_small_kernel<2>, grid, dim3(128), smem, st, true, meta, a);
   if (e != cudaSuccess) return e;
-  return cudaLaunchKernelEx(&cfg, in_cluster_kernel<2>, meta, a, a_ld);
+  return launch_kernel(in_select_small_kernel, dim3(meta.B), dim3(kSelThreads), 0, st, true, meta, a);
 }
 
 cudaError_t launch_in_token_score(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {

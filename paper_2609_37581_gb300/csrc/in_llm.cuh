@@ -8,7 +8,6 @@ namespace trevs {
 constexpr int kMaxHeads = 128;
 constexpr int kKeyBlock = 64;        // visual keys per stage-2 block / shared-memory chunk
 constexpr int kScoreTextRows = 16;   // text rows per token-score block
-constexpr int kClusterCtas = 8;      // CTAs per request of the fused small-request stage 2
 
 // Text rows per head-statistics block: the block keeps rows x K1 fp32 logits on chip.
 inline int stats_text_rows(int max_k1) { return max_k1 <= 128 ? 64 : (max_k1 <= 512 ? 32 : 16); }
