@@ -253,9 +253,10 @@ trevs_status validate_params(const trevs_pre_params* p) {
 
 // Runs stage 1 for requests [b0, b1) of the batch; offsets are relative to the chunk. When
 // `gm_out` is given the gather job is left to the caller (to share one launch with stage 2).
+// after_score (may be null) is recorded on `st` right after the scoring grid is enqueued.
 trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
                            long long n_base, long long m_base, long long k1_base, uint8_t* ws,
-                           const PreWs& L, cudaStream_t st, GatherMeta* gm_out) {
+                           const PreWs& L, cudaStream_t st, GatherMeta* gm_out, cudaEvent_t after_score = nullptr) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
   meta.B = b1 - b0;
@@ -298,6 +299,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.action = kActSelect;
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
+  if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "fork after scoring");
   TREVS_TRY_CUDA(counted(launch_pre_fixup(meta, a, max_m, st)), "fixup launch");
   TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, max_n, st, true)), "pre_select launch");
   GatherMeta& g = gm_out ? *gm_out : gm;
@@ -890,20 +892,19 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
   const cudaStream_t st = (cudaStream_t)stream;
   if (pre->B > 0 && in->B > 0 && pre->B <= kMaxChunk && in->B <= kMaxChunk) {
-    // one chunk each: the stages are independent, so stage 2 runs as a parallel branch on
-    // an auxiliary stream; one gather launch then serves both
+    // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
+    // 2 (with its own compaction) forks once that grid is enqueued, so it waits for it to
+    // finish and then runs beside the fixup, selection and gather of stage 1, which occupy
+    // few SMs.
     AuxStream* aux = nullptr;
     TREVS_TRY_CUDA(aux_stream(aux), "auxiliary stream");
-    TREVS_TRY_CUDA(cudaEventRecord(aux->fork, st), "fork");
-    TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
-    static thread_local GatherMeta gm;
-    s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, &gm);
+    s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork);
     if (s != TREVS_OK) return s;
-    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, &gm, false);
+    TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
+    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true);
     if (s != TREVS_OK) return s;
     TREVS_TRY_CUDA(cudaEventRecord(aux->join, aux->stream), "join");
     TREVS_TRY_CUDA(cudaStreamWaitEvent(st, aux->join, 0), "join");
-    if (gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, false)), "gather launch");
     return TREVS_OK;
   }
   if (pre->B > 0) {
