@@ -232,7 +232,7 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         batches = [build_batches(w, T.SELECT_RATIO, dev=s) for s in sets]
         ws = T.workspace(max(T.trevs_prune_varlen_workspace_size(p, i) for p, i in batches))
         calls = [T.PreparedCall(p, i, ws, params) for p, i in batches]
-        # the dominant kernel's chain: stage-1 pre-pass, scoring, fixup and selection (no gather)
+        # the dominant kernel's chain: stage-1 pre-pass, scoring, then the finishing grid (no gather)
         score_only = []
         for p, _ in batches:
             q = T.PreBatch(reqs=p.reqs, Z=p.Z, T=p.T, s_v=p.s_v, kept_idx=p.kept_idx, Z_out=None, s_t=p.s_t)
@@ -341,7 +341,8 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
                      "traffic": committed_traffic(), "algorithmic_bytes": nbytes["score_kernel"],
                      "kernel_us": round(kernel_ms * 1e3, 2),
                      "timed": "CUDA events around a graph of the stage-1 chain without the gather: "
-                              "pre-pass -> pre_score_kernel -> fixup -> selection (PDL-chained); "
+                              "pre-pass -> pre_score_kernel -> pre_finish_kernel (partial sums and "
+                              "selection; PDL-chained); "
                               "bytes are those of the scoring grid alone, so the fraction is a lower "
                               "bound for that grid"},
         "step_roofline": {"algorithmic_bytes": nbytes["step"],

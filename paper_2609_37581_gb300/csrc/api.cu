@@ -14,8 +14,8 @@
 namespace trevs {
 cudaError_t launch_pre_score(const PreMeta&, const PreArgs&, int max_m, long long z_rows, cudaStream_t, bool pdl);
 size_t pre_score_part_bytes(int max_m);
-cudaError_t launch_pre_fixup(const PreMeta&, const PreArgs&, int max_m, cudaStream_t);
-cudaError_t launch_pre_select(const PreMeta&, const PreArgs&, int max_n, cudaStream_t, bool pdl);
+cudaError_t launch_pre_finish(const PreMeta&, const PreArgs&, int max_m, int max_n, bool scored, cudaStream_t,
+                              bool pdl);
 cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
@@ -300,8 +300,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
   if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "fork after scoring");
-  TREVS_TRY_CUDA(counted(launch_pre_fixup(meta, a, max_m, st)), "fixup launch");
-  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, max_n, st, true)), "pre_select launch");
+  TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, st, true)), "finishing launch");
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
   if (bt->Z_out && ko > 0) {
@@ -622,9 +621,7 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   a.action = s_fused_out ? kActScoresFused : kActScores;
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, (cudaStream_t)stream)), "pre-pass launch");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream, true)), "pre_score launch");
-  TREVS_TRY_CUDA(counted(launch_pre_fixup(meta, a, M, (cudaStream_t)stream)), "fixup launch");
-  if (s_fused_out)
-    TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream, true)), "fused-score launch");
+  TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, M, N, true, (cudaStream_t)stream, true)), "finishing launch");
   return TREVS_OK;
 }
 
@@ -664,7 +661,7 @@ trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, const floa
   a.mode = fused ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
-  TREVS_TRY_CUDA(counted(launch_pre_select(meta, a, N, (cudaStream_t)stream, false)), "pre_select launch");
+  TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, 0, N, false, (cudaStream_t)stream, false)), "selection launch");
   return TREVS_OK;
 }
 

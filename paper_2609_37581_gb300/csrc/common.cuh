@@ -366,6 +366,225 @@ __device__ inline void block_mark_selected(const uint32_t* keys, int n, uint32_t
   block_emit_selected(keys, n, tau, need, s, [&](int i, int, bool sel) { if (sel) flags[i] = 1; });
 }
 
+// ------------------------------------------------------------------ register-resident selection
+//
+// Selection over up to E * blockDim.x entries held in registers, E per thread: thread t
+// holds entries i = e * blockDim.x + t (coalesced loads). Key 0 marks an excluded entry (no
+// float maps to it). The top k (ties to the lower index) are described by (tau, need):
+// entry i is selected iff key > tau, or key == tau and fewer than `need` entries equal to
+// tau precede it. Radix select on the offsets w = key - min(keys) with 8-bit digits, the
+// first digit taking the top bits of the occupied range; it stops as soon as every
+// candidate of the chosen digit belongs to the top k. Each pass costs three block
+// barriers. Requires blockDim.x >= 256, a multiple of 32, and E * blockDim.x / 32 <= 512.
+
+struct RegSelShared {
+  uint32_t hist[2][256];
+  uint32_t cell[512];     // per (element slot, warp) counts, then their prefix sums
+  uint32_t wred[3][32];
+  uint32_t res[4];
+};
+
+// Block-wide min of the non-zero keys, max of all keys and count of the non-zero keys;
+// also clears hist[0] for the first radix pass.
+template <int E>
+__device__ inline void block_reg_stats(const uint32_t (&key)[E], RegSelShared& s, uint32_t& lo, uint32_t& hi,
+                                       uint32_t& cnt) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  uint32_t l = 0xFFFFFFFFu, h = 0u, c = 0u;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    if (key[e] != 0u) { l = min(l, key[e]); ++c; }
+    h = max(h, key[e]);
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    l = min(l, __shfl_xor_sync(0xffffffffu, l, o));
+    h = max(h, __shfl_xor_sync(0xffffffffu, h, o));
+    c += __shfl_xor_sync(0xffffffffu, c, o);
+  }
+  if (lane == 0) { s.wred[0][warp] = l; s.wred[1][warp] = h; s.wred[2][warp] = c; }
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) s.hist[0][i] = 0u;
+  __syncthreads();
+  l = 0xFFFFFFFFu; h = 0u; c = 0u;
+  for (int w = 0; w < nwarps; ++w) { l = min(l, s.wred[0][w]); h = max(h, s.wred[1][w]); c += s.wred[2][w]; }
+  __syncthreads();   // wred is rewritten by the caller's next step
+  lo = l; hi = h; cnt = c;
+}
+
+// (tau, need) of the k largest non-zero keys; `lo`, `hi`, `cnt` as from block_reg_stats.
+template <int E>
+__device__ inline void block_reg_topk_ranged(const uint32_t (&key)[E], int k, uint32_t lo, uint32_t hi,
+                                             uint32_t cnt, RegSelShared& s, uint32_t& tau, int& need) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (k <= 0) { tau = 0xFFFFFFFFu; need = 0; return; }            // nothing
+  if ((uint32_t)k >= cnt) { tau = 0u; need = 0; return; }         // every non-zero key
+  if (lo == hi) { tau = lo; need = k; return; }                   // all equal: the first k
+  const int bits = 32 - __clz(hi - lo);
+  int sh = bits > 8 ? bits - 8 : 0;
+  uint32_t nb = 1u << (bits - sh);
+  uint32_t pm = 0u, pv = 0u, kk = (uint32_t)k;
+  int buf = 0;
+  while (true) {
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const uint32_t w = key[e] - lo;
+      if (key[e] != 0u && (w & pm) == pv) atomicAdd(&s.hist[buf][(w >> sh) & (nb - 1u)], 1u);
+    }
+    for (int i = tid; i < 256; i += blockDim.x) s.hist[buf ^ 1][i] = 0u;
+    __syncthreads();
+    // thread t < nb owns digit nb - 1 - t: counts from the top digit down
+    uint32_t c = 0u, incl = 0u;
+    if (tid < 256) {
+      c = tid < (int)nb ? s.hist[buf][nb - 1u - (uint32_t)tid] : 0u;
+      incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (lane == 31) s.wred[0][warp] = incl;
+    }
+    __syncthreads();
+    if (tid < 256 && c != 0u) {
+      uint32_t off = 0u;
+      for (int w = 0; w < warp; ++w) off += s.wred[0][w];
+      const uint32_t ex = incl - c + off;
+      if (ex < kk && kk <= ex + c) {
+        s.res[0] = nb - 1u - (uint32_t)tid;
+        s.res[1] = kk - ex;
+        s.res[2] = c;
+      }
+    }
+    __syncthreads();
+    const uint32_t dg = s.res[0], kn = s.res[1], cn = s.res[2];
+    pv |= dg << sh;
+    pm |= (nb - 1u) << sh;
+    buf ^= 1;
+    if (kn == cn) { tau = lo + pv - 1u; need = 0; return; }      // the whole digit is in: key >= lo + pv
+    if (sh == 0) { tau = lo + pv; need = (int)kn; return; }       // ties at one key value
+    kk = kn;
+    const int nbits = sh > 8 ? 8 : sh;
+    sh -= nbits;
+    nb = 1u << nbits;
+  }
+}
+
+template <int E>
+__device__ inline void block_reg_topk(const uint32_t (&key)[E], int k, RegSelShared& s, uint32_t& tau, int& need) {
+  uint32_t lo, hi, cnt;
+  block_reg_stats(key, s, lo, hi, cnt);
+  block_reg_topk_ranged(key, k, lo, hi, cnt, s, tau, need);
+}
+
+// The k-th largest key (1 <= k <= number of non-zero keys).
+template <int E>
+__device__ inline uint32_t block_reg_kth(const uint32_t (&key)[E], int k, RegSelShared& s) {
+  uint32_t tau;
+  int need;
+  block_reg_topk(key, k, s, tau, need);
+  if (need > 0) return tau;
+  // the top k are exactly the keys > tau: the k-th largest is their minimum
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  uint32_t m = 0xFFFFFFFFu;
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if (key[e] > tau) m = min(m, key[e]);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) m = min(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if (lane == 0) s.wred[0][warp] = m;
+  __syncthreads();
+  m = 0xFFFFFFFFu;
+  for (int w = 0; w < nwarps; ++w) m = min(m, s.wred[0][w]);
+  __syncthreads();
+  return m;
+}
+
+// Exclusive block-wide prefix sum of one value per thread (thread order).
+__device__ inline uint32_t block_excl_scan(uint32_t v, RegSelShared& s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) s.wred[1][warp] = incl;
+  __syncthreads();
+  uint32_t off = 0u;
+  for (int w = 0; w < warp; ++w) off += s.wred[1][w];
+  __syncthreads();
+  return incl - v + off;
+}
+
+// s.cell[e * nwarps + warp] = the number of entries before the 32-entry group (e, warp), in
+// index order, of each of the two per-group counts packed as lo16 | hi16 << 16.
+template <int E>
+__device__ inline void block_cell_offsets(const uint32_t (&packed)[E], RegSelShared& s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  if (lane == 0) {
+#pragma unroll
+    for (int e = 0; e < E; ++e) s.cell[e * nwarps + warp] = packed[e];
+  }
+  __syncthreads();
+  const int ncell = E * nwarps;
+  const uint32_t v = (int)threadIdx.x < ncell ? s.cell[threadIdx.x] : 0u;
+  const uint32_t ex = block_excl_scan(v, s);
+  if ((int)threadIdx.x < ncell) s.cell[threadIdx.x] = ex;
+  __syncthreads();
+}
+
+// Ordered output of a register-resident selection: out[pos] = i for every selected i,
+// ascending, where i = e * blockDim.x + t is selected iff bit e of `force` is set or
+// (tau, need) selects key[e]. Forced entries must carry key 0. Needs E * blockDim.x < 65536.
+template <int E>
+__device__ inline void block_reg_emit(const uint32_t (&key)[E], uint32_t force, uint32_t tau, int need, int* out,
+                                      RegSelShared& s) {
+  const int warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const uint32_t lt = lanemask_lt();
+  uint32_t packed[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const bool def = ((force >> e) & 1u) || key[e] > tau;
+    const bool eq = !def && need > 0 && key[e] == tau && key[e] != 0u;
+    packed[e] = (uint32_t)__popc(__ballot_sync(0xffffffffu, def)) |
+                ((uint32_t)__popc(__ballot_sync(0xffffffffu, eq)) << 16);
+  }
+  block_cell_offsets(packed, s);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const bool def = ((force >> e) & 1u) || key[e] > tau;
+    const bool eq = !def && need > 0 && key[e] == tau && key[e] != 0u;
+    const uint32_t bd = __ballot_sync(0xffffffffu, def), be = __ballot_sync(0xffffffffu, eq);
+    const uint32_t base = s.cell[e * nwarps + warp];
+    const uint32_t dbef = (base & 0xFFFFu) + __popc(bd & lt), ebef = (base >> 16) + __popc(be & lt);
+    const int i = e * blockDim.x + threadIdx.x;
+    if (def) out[dbef + min(ebef, (uint32_t)need)] = i;
+    else if (eq && ebef < (uint32_t)need) out[dbef + ebef] = i;
+  }
+}
+
+// Index of the need-th (1-based, index order) entry whose key equals tau; -1 if need <= 0.
+template <int E>
+__device__ inline int block_reg_nth_equal(const uint32_t (&key)[E], uint32_t tau, int need, RegSelShared& s) {
+  if (need <= 0) return -1;
+  const int warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  const uint32_t lt = lanemask_lt();
+  uint32_t packed[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) packed[e] = (uint32_t)__popc(__ballot_sync(0xffffffffu, key[e] == tau));
+  block_cell_offsets(packed, s);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const uint32_t be = __ballot_sync(0xffffffffu, key[e] == tau);
+    if (key[e] == tau && s.cell[e * nwarps + warp] + __popc(be & lt) + 1u == (uint32_t)need)
+      s.res[3] = (uint32_t)(e * blockDim.x + threadIdx.x);
+  }
+  __syncthreads();
+  const int cut = (int)s.res[3];
+  __syncthreads();
+  return cut;
+}
+
 // ------------------------------------------------------------------ launch helpers
 
 // Raises a kernel's dynamic shared-memory limit once per (kernel, device) and size, so

@@ -13,7 +13,7 @@ namespace trevs {
 // units, tile by tile; CTA c takes the contiguous units [W c / P, W (c + 1) / P), so that
 // every CTA streams the same number of stages. A tile whose stages are split between CTAs
 // leaves partial sums of G and ||z||^2 in the workspace (at most two per CTA: where its
-// range starts and where it ends), and pre_fixup_kernel adds them up in stage order.
+// range starts and where it ends), and pre_finish_kernel adds them up in stage order.
 //
 // For each sub-tile the 5th-generation tensor cores compute G = Z_sub . T^T (UMMA M = 128,
 // N = M_b rounded up to 16) into one of two TMEM accumulators, while eight warps sum the
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         }
       } else {
         // A tile split between CTAs: leave this CTA's partial sums (G row, columns
-        // 0 .. round_up(m, 4), and ||z||^2) in its slot for pre_fixup_kernel.
+        // 0 .. round_up(m, 4), and ||z||^2) in its slot for pre_finish_kernel.
         const long long sf = score_slot_floats(L.mld);
         float* own = a.part + (2 * (long long)blockIdx.x + st.slot) * sf;
         float* g = own + (long long)row * L.mld;
@@ -384,36 +384,33 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   }
 }
 
-// One CTA per tile split between scoring CTAs: s^t of its rows from the partial sums its
-// contributors left, added in stage order. The host lists the split tiles (tile, request,
-// first contributor, contributor count, slot of the first contributor). Thread (row, q)
-// adds column groups q, q + 4, ... of one row with all of a pass's loads in flight (the data
-// sit in L2; dependent round trips would dominate), and the four partial row sums meet in
-// shared memory.
-constexpr int kFixupThreads = 4 * kTileRows;
-struct FixJob {
-  int tile, b, c0, nc, slot0;
+// Finishing grid of stage 1, one CTA per job. A job with tile >= 0 is a tile split between
+// scoring CTAs: s^t of its rows from the partial sums its contributors left, added in stage
+// order. Thread (row, q) adds column groups q, q + 4, ... of one row with all of a pass's
+// loads in flight (the data sit in L2; dependent round trips would dominate), and the four
+// partial row sums meet in shared memory. The host lists the jobs (tile, request, first
+// contributor, contributor count, slot of the first contributor, jobs of the request);
+// requests without a split tile get one job with tile = -1. The last job of a request to
+// finish (a ticket per request, reset by that job) goes on with the request's selection
+// (Sec. 3.1) or fused scores (Eq. 6-7).
+constexpr int kFinishThreads = 4 * kTileRows;
+struct FinJob {
+  int tile, b, c0, nc, slot0, count;
 };
-struct FixMeta {
+struct FinMeta {
   int njobs, mld;
-  FixJob job[kMaxScoreCtas];
+  FinJob job[kMaxScoreCtas + kMaxChunk];
 };
-__global__ void __launch_bounds__(kFixupThreads, 1) pre_fixup_kernel(const __grid_constant__ PreMeta meta,
-                                                                     const __grid_constant__ FixMeta fm,
-                                                                     const PreArgs a) {
-  __shared__ float red[4][kTileRows];
-  __shared__ float rt[256];
-  const FixJob& jb = fm.job[blockIdx.x];
-  const PreReq& r = meta.r[jb.b];
-  const int mld = fm.mld;
+
+__device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, const PreArgs& a,
+                                  float (*red)[kTileRows], float* rt) {
   const int row0 = (jb.tile - r.tile_off) * kTileRows;
   const int h = min(kTileRows, r.n - row0);
   const int m = r.m;
   const int row = threadIdx.x & (kTileRows - 1), q = threadIdx.x >> 7;
   const long long sf = score_slot_floats(mld);
   const float* p0 = a.part + (2 * (long long)jb.c0 + jb.slot0) * sf;
-  pdl_wait();   // the partial sums come from the scoring grid (1 / ||t|| from before it)
-  for (int j = threadIdx.x; j < m; j += kFixupThreads) rt[j] = __ldcg(a.t_rinv + r.m_off + j);
+  for (int j = threadIdx.x; j < m; j += kFinishThreads) rt[j] = __ldcg(a.t_rinv + r.m_off + j);
   __syncthreads();
   const int ng = (m + 3) >> 2;
   float sum = 0.f;
@@ -467,33 +464,66 @@ __global__ void __launch_bounds__(kFixupThreads, 1) pre_fixup_kernel(const __gri
     a.s_t[r.n_off + row0 + row] = sqrtf(((red[0][row] + red[1][row]) + (red[2][row] + red[3][row])) / (float)m);
 }
 
-// One CTA per request: selection from scores already in memory (action kActSelect), or only
-// the Eq. 6-7 fused scores (kActScoresFused).
-__global__ void __launch_bounds__(512) pre_select_kernel(const __grid_constant__ PreMeta meta,
-                                                         const PreArgs a, int smem_bytes) {
+__global__ void __launch_bounds__(kFinishThreads, 1) pre_finish_kernel(const __grid_constant__ PreMeta meta,
+                                                                       const __grid_constant__ FinMeta fm,
+                                                                       const PreArgs a, int smem_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ SelShared ss;
-  pdl_wait();   // the scores come from the preceding grid
-  const PreReq r = meta.r[blockIdx.x];
-  select_request(a, r, blockIdx.x, smem, smem_bytes, ss, a.mode == kModeFused && !a.s_fused_given,
-                 a.action == kActSelect);
+  __shared__ union {
+    struct {
+      float red[4][kTileRows];
+      float rt[256];
+    } fx;
+    SelScratch sel;
+  } sh;
+  __shared__ int s_last;
+  pdl_launch_dependents();   // the next grid (the gather) waits for this one to complete
+  const FinJob& jb = fm.job[blockIdx.x];
+  const PreReq& r = meta.r[jb.b];
+  pdl_wait();   // partial sums and s^t come from the scoring grid (1 / ||t|| and rules from before it)
+  if (jb.tile >= 0) fixup_tile(jb, r, fm.mld, a, sh.fx.red, sh.fx.rt);
+  if (jb.count > 1) {
+    __threadfence();   // this job's s^t rows before its ticket
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const uint32_t done = atomicAdd(a.counters + jb.b, 1u) + 1u;
+      s_last = done == (uint32_t)jb.count;
+      if (s_last) a.counters[jb.b] = 0u;   // ready for the next launch
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();   // the other jobs' rows, read through L2
+  } else {
+    __syncthreads();
+  }
+  select_request_512(a, r, jb.b, smem, smem_bytes, sh.sel);
 }
 
 // Pre-pass, run ahead of the scoring grid. Blocks [0, n_sal): the saliency side of the
-// selection of request b = blockIdx.x (inputs only), so that the selection grid only ranks
-// textual relevance. Remaining blocks: 1 / ||t_j|| of the text rows, one warp per row.
+// selection of request b = blockIdx.x (inputs only), so that the finishing grid only ranks
+// textual relevance. Remaining blocks: 1 / ||t_j|| of the text rows, one warp per row with
+// all of a row's loads (up to d = 4096) in flight.
 __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant__ PreMeta meta,
                                                            const PreArgs a, int smem_bytes, int n_sal) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ SelShared ss;
+  __shared__ SelScratch sh;
   pdl_launch_dependents();
   if ((int)blockIdx.x >= n_sal) {
     const long long row = (long long)(blockIdx.x - n_sal) * 16 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= a.total_m) return;
     const uint4* t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
+    const int nv = a.d / 8;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int p = lane; p < a.d / 8; p += 32) bf16_sq_acc8(__ldg(t + p), acc);
+    for (int p0 = 0; p0 < nv; p0 += 16 * 32) {
+      uint4 v[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        const int p = p0 + 32 * q + lane;
+        v[q] = p < nv ? __ldg(t + p) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int q = 0; q < 16; ++q) bf16_sq_acc8(v[q], acc);
+    }
     float sq = (acc[0] + acc[1]) + (acc[2] + acc[3]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
@@ -505,7 +535,7 @@ __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant
   const bool in_smem = (size_t)r.n * 4 + 16 <= (size_t)smem_bytes;
   const size_t gbase = ((size_t)r.n_off + 4 * (size_t)b + 3) & ~(size_t)3;
   uint32_t* keys = in_smem ? reinterpret_cast<uint32_t*>(smem) : a.keys + gbase;
-  const int4 rule = saliency_prepare(a, r, keys, ss);
+  const int4 rule = saliency_rule_512(a, r, keys, sh);
   if (threadIdx.x == 0) a.sal[b] = rule;
 }
 
@@ -651,33 +681,50 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
                        tmZ2, meta, a, L);
 }
 
-// Partial sums of the scoring grid launched just before (same meta, d' and max M): the
-// split tiles are listed here, on the host, from the same partition the grid uses.
-cudaError_t launch_pre_fixup(const PreMeta& meta, const PreArgs& a, int max_m, cudaStream_t st) {
-  if (meta.total_tiles == 0) return cudaSuccess;
-  static thread_local FixMeta fm;
-  const int nzs = ((a.d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
-  const int P = score_grid(meta, a.d);
-  const int W = meta.total_tiles * nzs;
+// Finishing grid after the scoring grid launched just before it (same meta, d' and max M;
+// `scored` false: no scoring grid, selection only). The split tiles are listed here, on the
+// host, from the same partition the scoring grid uses.
+cudaError_t launch_pre_finish(const PreMeta& meta, const PreArgs& a, int max_m, int max_n, bool scored,
+                              cudaStream_t st, bool pdl) {
+  static thread_local FinMeta fm;
+  static thread_local int jobs_of[kMaxChunk];
   fm.njobs = 0;
   fm.mld = (max_m + 3) & ~3;
-  int b = 0;
-  for (int c = 1; c < P; ++c) {
-    const int bc = (int)((long long)W * c / P);
-    if (bc % nzs == 0) continue;
-    const int t = bc / nzs, t_start = t * nzs;
-    const int c0 = score_cta_of(t_start, W, P);
-    if (c0 != c - 1) continue;                       // the tile's first boundary lists it
-    while (b + 1 < meta.B && meta.r[b + 1].tile_off <= t) ++b;
-    FixJob& j = fm.job[fm.njobs++];
-    j.tile = t;
-    j.b = b;
-    j.c0 = c0;
-    j.nc = score_cta_of(t_start + nzs - 1, W, P) - c0 + 1;
-    j.slot0 = (int)((long long)W * c0 / P) < t_start ? 1 : 0;
+  for (int b = 0; b < meta.B; ++b) jobs_of[b] = 0;
+  if (scored && meta.total_tiles > 0) {
+    const int nzs = ((a.d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
+    const int P = score_grid(meta, a.d);
+    const int W = meta.total_tiles * nzs;
+    int b = 0;
+    for (int c = 1; c < P; ++c) {
+      const int bc = (int)((long long)W * c / P);
+      if (bc % nzs == 0) continue;
+      const int t = bc / nzs, t_start = t * nzs;
+      const int c0 = score_cta_of(t_start, W, P);
+      if (c0 != c - 1) continue;                     // the tile's first boundary lists it
+      while (b + 1 < meta.B && meta.r[b + 1].tile_off <= t) ++b;
+      FinJob& j = fm.job[fm.njobs++];
+      j.tile = t;
+      j.b = b;
+      j.c0 = c0;
+      j.nc = score_cta_of(t_start + nzs - 1, W, P) - c0 + 1;
+      j.slot0 = (int)((long long)W * c0 / P) < t_start ? 1 : 0;
+      ++jobs_of[b];
+    }
   }
+  const bool per_request = a.action != kActScores;
+  if (per_request)
+    for (int b = 0; b < meta.B; ++b)
+      if (jobs_of[b] == 0 && meta.r[b].n > 0) {
+        FinJob& j = fm.job[fm.njobs++];
+        j.tile = -1; j.b = b; j.c0 = 0; j.nc = 0; j.slot0 = 0;
+        jobs_of[b] = 1;
+      }
   if (fm.njobs == 0) return cudaSuccess;
-  return launch_kernel(pre_fixup_kernel, dim3(fm.njobs), dim3(kFixupThreads), 0, st, true, meta, fm, a);
+  for (int i = 0; i < fm.njobs; ++i) fm.job[i].count = per_request ? jobs_of[fm.job[i].b] : 1;
+  int smem = 0;   // keys and flags of the block-wide selection, for requests above kRegSelMaxN
+  if (per_request && max_n > kRegSelMaxN && (size_t)max_n * 5 + 16 <= (size_t)160 * 1024) smem = max_n * 5 + 16;
+  return launch_kernel(pre_finish_kernel, dim3(fm.njobs), dim3(kFinishThreads), smem, st, pdl, meta, fm, a, smem);
 }
 
 // Workspace bytes of the partial sums for up to max_m text rows.
@@ -691,22 +738,11 @@ cudaError_t launch_pre_saliency(const PreMeta& meta, const PreArgs& a, int max_n
   const int n_sal = saliency ? meta.B : 0;
   const long long tn_blocks = (a.total_m + 15) / 16;
   if (n_sal + tn_blocks == 0) return cudaSuccess;
-  int smem = saliency ? (int)((size_t)max_n * 4 + 16) : 0;
-  if (smem > 24 * 1024) smem = 0;   // keys in the global scratch: leave the SM to the scoring grid
-  cudaError_t e = ensure_dynamic_smem(pre_saliency_kernel, smem);
+  (void)max_n;   // requests above kRegSelMaxN keep their keys in the global scratch
+  cudaError_t e = ensure_dynamic_smem(pre_saliency_kernel, 0);   // the scoring grid's carveout
   if (e != cudaSuccess) return e;
-  pre_saliency_kernel<<<(unsigned)(n_sal + tn_blocks), 512, smem, st>>>(meta, a, smem, n_sal);
+  pre_saliency_kernel<<<(unsigned)(n_sal + tn_blocks), 512, 0, st>>>(meta, a, 0, n_sal);
   return cudaGetLastError();
-}
-
-// pdl: the preceding grid of the stream is the scoring grid (the kernel waits for it).
-cudaError_t launch_pre_select(const PreMeta& meta, const PreArgs& a, int max_n, cudaStream_t st, bool pdl) {
-  if (meta.B == 0) return cudaSuccess;
-  int smem = (int)((size_t)max_n * 5 + 16);
-  if (smem > 160 * 1024) smem = 0;   // keys stay in the global scratch
-  cudaError_t e = ensure_dynamic_smem(pre_select_kernel, smem);
-  if (e != cudaSuccess) return e;
-  return launch_kernel(pre_select_kernel, dim3(meta.B), dim3(512), smem, st, pdl, meta, a, smem);
 }
 
 cudaError_t launch_gather(const GatherMeta& gm, cudaStream_t st, bool pdl) {

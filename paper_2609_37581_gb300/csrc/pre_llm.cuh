@@ -153,6 +153,143 @@ __device__ inline void select_request(const PreArgs& a, const PreReq& r, int b, 
   }
 }
 
+// Register-resident forms of the two functions above for n <= E * blockDim.x (blockDim.x
+// a multiple of 32, at least 256): thread t holds entries e * blockDim.x + t.
+template <int E>
+__device__ inline int4 saliency_prepare_reg(const PreArgs& a, const PreReq& r, RegSelShared& rs) {
+  const int n = r.n;
+  const float* sv = a.s_v + r.n_off;
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  uint32_t key[E];
+  if (a.mode == kModeRatio) {
+    const int kv = r.k1 - r.kt;
+    if (kv <= 0 || n <= 0) return make_int4(-1, 0, 1, -1);   // empty: nothing passes the rule
+#pragma unroll
+    for (int e = 0; e < E; ++e) key[e] = e * nthr + tid < n ? score_key(__ldcg(sv + e * nthr + tid)) : 0u;
+    uint32_t tau;
+    int need;
+    block_reg_topk(key, kv, rs, tau, need);
+    // ties at tau: the first `need` of them in index order, i.e. up to the need-th one
+    const int cut = block_reg_nth_equal(key, tau, need, rs);
+    return make_int4((int)tau, 0, 1, cut);
+  }
+  if (n <= 0) return make_int4(0, 0, 0, 0);
+  const int kmed = n - (n - 1) / 2;  // lower median = kmed-th largest
+  float v[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    v[e] = e * nthr + tid < n ? __ldcg(sv + e * nthr + tid) : 0.f;
+    key[e] = e * nthr + tid < n ? score_key(v[e]) : 0u;
+  }
+  const float med = key_to_score(block_reg_kth(key, kmed, rs));
+#pragma unroll
+  for (int e = 0; e < E; ++e) key[e] = e * nthr + tid < n ? score_key(fabsf(v[e] - med)) : 0u;
+  const float mad = key_to_score(block_reg_kth(key, kmed, rs));
+  return make_int4(__float_as_int(med), __float_as_int(mad), 0, 0);
+}
+
+template <int E>
+__device__ inline void select_request_reg(const PreArgs& a, const PreReq& r, int b, RegSelShared& rs,
+                                          bool compute_fused, bool do_select) {
+  const int n = r.n;
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  const float* sv = a.s_v + r.n_off;
+  const float* st = a.s_t + r.n_off;
+  int4 rule = make_int4(-1, 0, 1, -1);
+  if (a.sal_ready) rule = __ldcg(a.sal + b);
+  else if (a.mode == kModeRatio ? do_select : compute_fused) rule = saliency_prepare_reg<E>(a, r, rs);
+  uint32_t key[E];
+  uint32_t tau;
+  int need;
+  if (a.mode == kModeRatio) {
+    if (!do_select || r.k1 <= 0) return;
+    // S_v from its rule (forced in); the textual keys exclude it (key 0)
+    uint32_t force = 0u;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const int i = e * nthr + tid;
+      key[e] = 0u;
+      if (i < n) {
+        if (in_saliency_set(__ldcg(sv + i), i, rule)) force |= 1u << e;
+        else key[e] = score_key(__ldcg(st + i));
+      }
+    }
+    block_reg_topk(key, r.kt, rs, tau, need);
+    block_reg_emit(key, force, tau, need, a.kept + r.k1_off, rs);
+    return;
+  }
+
+  // fused mode (Eq. 6-7)
+  float* sf = a.s_fused + r.n_off;
+  float f[E];
+  if (compute_fused) {
+    float t[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      t[e] = e * nthr + tid < n ? __ldcg(st + e * nthr + tid) : 0.f;
+      key[e] = e * nthr + tid < n ? score_key(t[e]) : 0u;
+    }
+    const int kmed = n - (n - 1) / 2;  // lower median = kmed-th largest
+    const float med_t = key_to_score(block_reg_kth(key, kmed, rs));
+#pragma unroll
+    for (int e = 0; e < E; ++e) key[e] = e * nthr + tid < n ? score_key(fabsf(t[e] - med_t)) : 0u;
+    const float mad_t = key_to_score(block_reg_kth(key, kmed, rs));
+    const float med_v = __int_as_float(rule.x), mad_v = __int_as_float(rule.y);
+    const float dv = mad_v + a.eps, dt = mad_t + a.eps;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const int i = e * nthr + tid;
+      f[e] = 0.f;
+      if (i < n) {
+        const float hv = fmaxf((__ldcg(sv + i) - med_v) / dv, 0.f) / a.tau_v;
+        const float ht = fmaxf((t[e] - med_t) / dt, 0.f) / a.tau_t;
+        f[e] = fmaxf(hv, ht) + a.lambda * sqrtf(hv * ht);
+        sf[i] = f[e];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < E; ++e) f[e] = e * nthr + tid < n ? __ldcg(sf + e * nthr + tid) : 0.f;
+  }
+  if (!do_select || r.k1 <= 0) return;
+#pragma unroll
+  for (int e = 0; e < E; ++e) key[e] = e * nthr + tid < n ? score_key(f[e]) : 0u;
+  block_reg_topk(key, r.k1, rs, tau, need);
+  block_reg_emit(key, 0u, tau, need, a.kept + r.k1_off, rs);
+}
+
+union SelScratch {
+  SelShared ss;
+  RegSelShared rs;
+};
+
+// Largest request the register-resident forms take with 512 threads (larger ones are
+// faster with the keys in memory).
+constexpr int kRegSelMaxN = 8 * 512;
+
+// Saliency rule of request r by a block of 512 threads; `keys` (n entries, 16-byte
+// aligned) is only touched for requests above kRegSelMaxN.
+__device__ inline int4 saliency_rule_512(const PreArgs& a, const PreReq& r, uint32_t* keys, SelScratch& sh) {
+  const int n = r.n;
+  if (n <= 512) return saliency_prepare_reg<1>(a, r, sh.rs);
+  if (n <= 1024) return saliency_prepare_reg<2>(a, r, sh.rs);
+  if (n <= kRegSelMaxN) return saliency_prepare_reg<8>(a, r, sh.rs);
+  return saliency_prepare(a, r, keys, sh.ss);
+}
+
+// Selection (or fused scores) of request r by a block of 512 threads.
+__device__ inline void select_request_512(const PreArgs& a, const PreReq& r, int b, uint8_t* smem, int smem_bytes,
+                                          SelScratch& sh) {
+  const int n = r.n;
+  if (n <= 0) return;
+  const bool compute_fused = a.mode == kModeFused && !a.s_fused_given;
+  const bool do_select = a.action == kActSelect;
+  if (n <= 512) select_request_reg<1>(a, r, b, sh.rs, compute_fused, do_select);
+  else if (n <= 1024) select_request_reg<2>(a, r, b, sh.rs, compute_fused, do_select);
+  else if (n <= kRegSelMaxN) select_request_reg<8>(a, r, b, sh.rs, compute_fused, do_select);
+  else select_request(a, r, b, smem, smem_bytes, sh.ss, compute_fused, do_select);
+}
+
 // ------------------------------------------------------------------ row gather
 
 struct GatherJob {
