@@ -279,6 +279,19 @@ TREVS_API size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, c
 TREVS_API trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_params* p,
                                   void* workspace, size_t workspace_bytes, void* stream);
 
+/* trevs_pre_llm_varlen that also times the scoring grid (Eq. 4-5) on `stream`. It has no
+ * counterpart in the paper: it is a measurement hook for the kernel that dominates stage 1.
+ * - ev_score_begin and ev_score_end are cudaEvent_t handles the caller created with timing
+ *   enabled. The call records ev_score_begin just before the scoring grid is enqueued and
+ *   ev_score_end just after it, so cudaEventElapsedTime(begin, end) spans the grid, from
+ *   the completion of the pre-pass before it to the grid's own completion.
+ * - Results are those of trevs_pre_llm_varlen.
+ * - Limits: 1 <= B <= 256 requests (one launch chunk); a larger B returns
+ *   TREVS_ERR_UNSUPPORTED, a NULL event TREVS_ERR_INVALID_ARGUMENT, before any CUDA call. */
+TREVS_API trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, const trevs_pre_params* p,
+                                        void* workspace, size_t workspace_bytes, void* stream,
+                                        void* ev_score_begin, void* ev_score_end);
+
 /* Stage 2 for a batch: attention statistics, Eq. 8 head variances, H*, Eq. 9 token scores,
  * TopK(p, k2) and compaction of hidden, K and V rows. */
 TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,

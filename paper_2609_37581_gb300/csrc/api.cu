@@ -256,7 +256,8 @@ trevs_status validate_params(const trevs_pre_params* p) {
 // after_score (may be null) is recorded on `st` right after the scoring grid is enqueued.
 trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
                            long long n_base, long long m_base, long long k1_base, uint8_t* ws,
-                           const PreWs& L, cudaStream_t st, GatherMeta* gm_out, cudaEvent_t after_score = nullptr) {
+                           const PreWs& L, cudaStream_t st, GatherMeta* gm_out, cudaEvent_t after_score = nullptr,
+                           cudaEvent_t before_score = nullptr) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
   meta.B = b1 - b0;
@@ -298,8 +299,9 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
+  if (before_score) TREVS_TRY_CUDA(cudaEventRecord(before_score, st), "event before scoring");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
-  if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "fork after scoring");
+  if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "event after scoring");
   TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, st, true)), "finishing launch");
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
@@ -854,6 +856,26 @@ trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
+}
+
+trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, const trevs_pre_params* p, void* workspace,
+                                        size_t workspace_bytes, void* stream, void* ev_score_begin,
+                                        void* ev_score_end) {
+  g_launches = 0;
+  const trevs_pre_params prm = p ? *p : kDefaults;
+  trevs_status s = validate_params(&prm);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(ev_score_begin != nullptr && ev_score_end != nullptr, "both events must be non-NULL");
+  PreTotals t;
+  s = validate_pre_batch(batch, t);
+  if (s != TREVS_OK) return s;
+  TREVS_CHECK(batch->B >= 1, "B = 0: nothing to time");
+  if (batch->B > kMaxChunk) return fail(TREVS_ERR_UNSUPPORTED, "B = %d > %d requests", batch->B, kMaxChunk);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m);
+  s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  return run_pre_chunk(batch, prm, 0, batch->B, 0, 0, 0, reinterpret_cast<uint8_t*>(workspace), L,
+                       (cudaStream_t)stream, nullptr, (cudaEvent_t)ev_score_end, (cudaEvent_t)ev_score_begin);
 }
 
 trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch, void* workspace, size_t workspace_bytes,

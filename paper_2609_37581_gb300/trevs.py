@@ -93,6 +93,8 @@ _SIGS = {
     "trevs_in_llm_varlen_workspace_size": (_c_sz, [ctypes.POINTER(InBatchC)]),
     "trevs_prune_varlen_workspace_size": (_c_sz, [ctypes.POINTER(PreBatchC), ctypes.POINTER(InBatchC)]),
     "trevs_pre_llm_varlen": (_c_i32, [ctypes.POINTER(PreBatchC), ctypes.POINTER(PreParams), _vp, _c_sz, _vp]),
+    "trevs_pre_llm_varlen_timed": (_c_i32, [ctypes.POINTER(PreBatchC), ctypes.POINTER(PreParams), _vp, _c_sz, _vp,
+                                            _vp, _vp]),
     "trevs_in_llm_varlen": (_c_i32, [ctypes.POINTER(InBatchC), _vp, _c_sz, _vp]),
     "trevs_prune_varlen": (_c_i32, [ctypes.POINTER(PreBatchC), ctypes.POINTER(PreParams),
                                     ctypes.POINTER(InBatchC), _vp, _c_sz, _vp]),
@@ -311,6 +313,16 @@ def trevs_pre_llm_varlen(pre: PreBatch, ws, params=None, stream=None):
     w, nb = _ws_args(ws)
     check(load().trevs_pre_llm_varlen(ctypes.byref(pre.c()),
                                       ctypes.byref(params) if params is not None else None, w, nb, _stream(stream)))
+
+
+def trevs_pre_llm_varlen_timed(pre: PreBatch, ws, ev_begin, ev_end, params=None, stream=None):
+    """trevs_pre_llm_varlen with the scoring grid bracketed by two timing events (torch.cuda.Event
+    objects that have been recorded once, or raw cudaEvent_t handles)."""
+    w, nb = _ws_args(ws)
+    h = lambda e: getattr(e, "cuda_event", e)
+    check(load().trevs_pre_llm_varlen_timed(ctypes.byref(pre.c()),
+                                            ctypes.byref(params) if params is not None else None, w, nb,
+                                            _stream(stream), h(ev_begin), h(ev_end)))
 
 
 def trevs_in_llm_varlen(inb: InBatch, ws, stream=None):

@@ -140,6 +140,20 @@ def test_varlen_validation(lib):
     assert lib.trevs_pre_llm_varlen(ctypes.byref(empty), None, None, 0, None) == 0
 
 
+def test_varlen_timed_validation(lib):
+    ok = _pre_batch([(576, 32, 64, 0.5), (1152, 8, 96, 0.25)])
+    need = lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(ok))
+    f = lib.trevs_pre_llm_varlen_timed
+    assert f(ctypes.byref(ok), None, FAKE, need, None, None, FAKE) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert f(ctypes.byref(ok), None, FAKE, need, None, FAKE, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert f(ctypes.byref(_pre_batch([(576, 32, 577, 0.5)])), None, FAKE, 1 << 30, None, FAKE,
+             FAKE) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert f(ctypes.byref(t.PreBatchC()), None, None, 0, None, FAKE, FAKE) == t.TREVS_ERR_INVALID_ARGUMENT
+    big = _pre_batch([(8, 1, 1, 0.5)] * 257)     # more requests than one launch chunk
+    assert f(ctypes.byref(big), None, FAKE, 1 << 30, None, FAKE, FAKE) == t.TREVS_ERR_UNSUPPORTED
+    assert f(ctypes.byref(ok), None, FAKE, need - 256, None, FAKE, FAKE) == t.TREVS_ERR_WORKSPACE
+
+
 def _in_batch(reqs, Hq=32, Hkv=32, nk=8):
     arr = (t.InRequest * len(reqs))(*[t.InRequest(*r) for r in reqs])
     b = t.InBatchC()

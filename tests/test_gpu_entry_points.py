@@ -168,3 +168,28 @@ def test_workspace_status_ok_after_calls():
     g, ws = H.run_gpu(w)
     T.workspace_status(ws)
     assert T.last_launch_count() == 0 or True
+
+
+def test_timed_stage1_matches_untimed():
+    """The measurement hook brackets the scoring grid with two events and changes nothing."""
+    from workloads.device import build_batches
+    w = synth.small_case()
+    pre, _ = build_batches(w, T.SELECT_RATIO)
+    outs = []
+    for timed in (False, True):
+        q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v,
+                       kept_idx=torch.full_like(pre.kept_idx, -1), Z_out=torch.zeros_like(pre.Z_out),
+                       s_t=torch.zeros_like(pre.s_t))
+        ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
+        if timed:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(); e1.record()                 # create both handles
+            T.trevs_pre_llm_varlen_timed(q, ws, e0, e1, T.default_params())
+            torch.cuda.synchronize()
+            assert e0.elapsed_time(e1) > 0.0
+        else:
+            T.trevs_pre_llm_varlen(q, ws, T.default_params())
+            torch.cuda.synchronize()
+        outs.append((q.s_t.cpu().numpy(), q.kept_idx.cpu().numpy(), H.host_u16(q.Z_out)))
+    for a, b in zip(*outs):
+        np.testing.assert_array_equal(a, b)
