@@ -319,9 +319,12 @@ __global__ void __launch_bounds__(128) in_token_score_kernel(const __grid_consta
 // the softmax max and sum and the two-pass Eq. 8 row variance need only quad shuffles. The
 // block writes the attention probabilities A_h[q][i] and u_h.
 //
-// in_select_small_kernel: one block per request. H* from u; Eq. 9 p_i = max_q of the mean
-// over H* (heads summed in ascending order) with thread (key i, row group) and every load of
-// a batch in flight; then TopK(p, K2) in shared memory.
+// in_select_small_kernel: one block per (request, 16 keys). Each block forms H* from u and
+// Eq. 9 p_i = max_q of the mean over H* (heads summed in ascending order) for its keys, with
+// thread (key, row group) and all of a thread's loads in flight: a request's 4 L K1 |H*|
+// bytes of probabilities are spread over several SMs. The last block of a request to
+// finish (a ticket per request, reset by that block) ranks the K1 scores, TopK(p, K2) with
+// ties to the lower index, and writes the ordered kept list.
 template <int NCH>   // 64-key chunks: K1 <= 64 * NCH
 __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constant__ InMeta meta, const InArgs a) {
   constexpr int QR = 64;              // text rows (four m16 tiles, one per warp)
@@ -432,90 +435,120 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
   if (tid == 0) a.u[(long long)b * a.u_ld + h] = (((s_upart[0] + s_upart[1]) + s_upart[2]) + s_upart[3]) / (float)L;
 }
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 128;
+constexpr int kSelKeys = 16;                       // keys per block
+constexpr int kSelGroups = kSelThreads / kSelKeys; // row groups per block
 __global__ void __launch_bounds__(kSelThreads) in_select_small_kernel(const __grid_constant__ InMeta meta,
                                                                        const InArgs a) {
   __shared__ float s_u[kMaxHeads];
-  __shared__ int s_sel[kMaxHeads];
   __shared__ int s_heads[kMaxHeads];
-  __shared__ int s_nh;
+  __shared__ int s_wc[kSelThreads / 32];
   __shared__ float s_red[kSelThreads];
   __shared__ uint32_t s_keys[128];
-  __shared__ uint8_t s_flags[128];
-  __shared__ SelShared ss;
+  __shared__ int s_last;
   pdl_wait();                         // u and the attention probabilities come from the preceding grid
   pdl_launch_dependents();
-  const int tid = threadIdx.x;
-  const int b = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int kblocks = (int)gridDim.y;
+  const int b = blockIdx.x, kb = blockIdx.y;
   const InReq r = meta.r[b];
   const int L = r.l, K1 = r.k1, Hq = a.Hq;
-  const float* u = a.u + (long long)b * a.u_ld;
-  for (int hh = tid; hh < Hq; hh += kSelThreads) s_u[hh] = __ldcg(u + hh);
-  __syncthreads();
-  for (int hh = tid; hh < Hq; hh += kSelThreads) {   // H*: the n_keep largest u, ties to the lower head
-    const float uh = s_u[hh];
-    int rank = 0;
-    for (int x = 0; x < Hq; ++x) rank += (s_u[x] > uh) || (s_u[x] == uh && x < hh);
-    s_sel[hh] = rank < a.n_keep;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    int cnt = 0;
-    for (int hh = 0; hh < Hq && cnt < a.n_keep; ++hh)
-      if (s_sel[hh]) s_heads[cnt++] = hh;
-    s_nh = cnt;
-  }
-  __syncthreads();
-  const int nh = s_nh;
-  // thread (key i, row group rg): rows rg, rg + NG, ...; heads four at a time, all loads in flight
-  const int kp = K1 <= 64 ? 64 : 128;
-  const int NG = kSelThreads / kp;
-  const int i = tid % kp, rg = tid / kp;
-  const float* A = a.attn + r.attn_off + i;
-  const long long hstride = (long long)L * K1;
-  float m = 0.f;                      // probabilities are positive: 0 never wins the max
-  if (i < K1) {
-    constexpr int RPT = 16;           // rows per thread at most (L <= 64, NG >= 4)
-    float psum[RPT];
+  if (kb * kSelKeys < K1) {
+    const float* u = a.u + (long long)b * a.u_ld;
+    for (int hh = tid; hh < Hq; hh += kSelThreads) s_u[hh] = __ldcg(u + hh);
+    __syncthreads();
+    // H*: the n_keep largest u, ties to the lower head, listed in ascending head order
+    int nh = 0;
+    for (int h0 = 0; h0 < Hq; h0 += kSelThreads) {
+      const int hh = h0 + tid;
+      bool sel = false;
+      if (hh < Hq) {
+        const float uh = s_u[hh];
+        int rank = 0;
+        for (int x = 0; x < Hq; ++x) rank += (s_u[x] > uh) || (s_u[x] == uh && x < hh);
+        sel = rank < a.n_keep;
+      }
+      const uint32_t bal = __ballot_sync(0xffffffffu, sel);
+      if (lane == 0) s_wc[warp] = __popc(bal);
+      __syncthreads();
+      int before = nh;
+      for (int w = 0; w < warp; ++w) before += s_wc[w];
+      for (int w = 0; w < kSelThreads / 32; ++w) nh += s_wc[w];
+      if (sel) s_heads[before + __popc(bal & lanemask_lt())] = hh;
+      __syncthreads();
+    }
+    // Eq. 9 for key i: rows rg, rg + 8, ... (L <= 64: eight rows), every head's loads in flight
+    const int i = kb * kSelKeys + (tid % kSelKeys), rg = tid / kSelKeys;
+    const float* A = a.attn + r.attn_off + i;
+    const long long hstride = (long long)L * K1;
+    float m = 0.f;                    // probabilities are positive: 0 never wins the max
+    if (i < K1) {
+      constexpr int RPT = 64 / kSelGroups;
+      float psum[RPT];
 #pragma unroll
-    for (int j = 0; j < RPT; ++j) psum[j] = 0.f;
-    for (int h0 = 0; h0 < nh; h0 += 4) {
-      float v[4][RPT];
+      for (int j = 0; j < RPT; ++j) psum[j] = 0.f;
+      for (int h0 = 0; h0 < nh; h0 += 8) {
+        float v[8][RPT];
 #pragma unroll
-      for (int x = 0; x < 4; ++x) {
-        const float* Ah = A + (long long)s_heads[min(h0 + x, nh - 1)] * hstride;
+        for (int x = 0; x < 8; ++x) {
+          const float* Ah = A + (long long)s_heads[min(h0 + x, nh - 1)] * hstride;
 #pragma unroll
-        for (int j = 0; j < RPT; ++j) {
-          const int q = rg + NG * j;
-          v[x][j] = (h0 + x < nh && q < L) ? __ldcg(Ah + (long long)q * K1) : 0.f;
+          for (int j = 0; j < RPT; ++j) {
+            const int q = rg + kSelGroups * j;
+            v[x][j] = (h0 + x < nh && q < L) ? __ldcg(Ah + (long long)q * K1) : 0.f;
+          }
         }
+#pragma unroll
+        for (int x = 0; x < 8; ++x)
+#pragma unroll
+          for (int j = 0; j < RPT; ++j) psum[j] += v[x][j];
       }
 #pragma unroll
-      for (int x = 0; x < 4; ++x)
-#pragma unroll
-        for (int j = 0; j < RPT; ++j) psum[j] += v[x][j];
+      for (int j = 0; j < RPT; ++j) m = fmaxf(m, psum[j]);
     }
-#pragma unroll
-    for (int j = 0; j < RPT; ++j) m = fmaxf(m, psum[j]);
+    s_red[tid] = m;
+    __syncthreads();
+    if (tid < kSelKeys && i < K1) {
+      float mx = 0.f;
+      for (int x = 0; x < kSelGroups; ++x) mx = fmaxf(mx, s_red[x * kSelKeys + tid]);
+      a.p_bits[r.k1_off + i] = __float_as_uint(mx * (nh > 0 ? 1.0f / (float)nh : 0.f));
+    }
+    if (kb == 0 && a.heads_out)
+      for (int x = tid; x < nh; x += kSelThreads) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
   }
-  s_red[tid] = m;
+  // the last block of the request ranks all K1 scores
+  __threadfence();
   __syncthreads();
-  const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
+  if (tid == 0) {
+    const uint32_t done = atomicAdd(a.cnt_ts + b, 1u) + 1u;
+    s_last = done == (uint32_t)kblocks;
+    if (s_last) a.cnt_ts[b] = 0u;     // ready for the next launch
+  }
+  __syncthreads();
+  if (!s_last || r.k2 <= 0) return;
+  __threadfence();
+  uint32_t key = 0u;
   if (tid < K1) {
-    float mx = 0.f;
-    for (int x = 0; x < NG; ++x) mx = fmaxf(mx, s_red[x * kp + tid]);
-    const float p = mx * inv_nh;
-    a.p_bits[r.k1_off + tid] = __float_as_uint(p);
-    s_keys[tid] = score_key(p);
-    s_flags[tid] = 0;
+    key = score_key(__uint_as_float(__ldcg(a.p_bits + r.k1_off + tid)));
+    s_keys[tid] = key;
   }
-  if (a.heads_out)
-    for (int x = tid; x < nh; x += kSelThreads) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
   __syncthreads();
-  if (r.k2 > 0) {
-    block_mark_topk_small(s_keys, K1, r.k2, s_flags);
-    block_compact_flags(s_flags, K1, a.kept_local + r.k2_off, ss);
+  bool keep = false;
+  if (tid < K1) {
+    int rank = 0;
+#pragma unroll 4
+    for (int j = 0; j < K1; ++j) {
+      const uint32_t o = s_keys[j];
+      rank += (o > key) || (o == key && j < tid);
+    }
+    keep = rank < r.k2;
   }
+  const uint32_t kbal = __ballot_sync(0xffffffffu, keep);
+  if (lane == 0) s_wc[warp] = __popc(kbal);
+  __syncthreads();
+  int pos = 0;
+  for (int w = 0; w < warp; ++w) pos += s_wc[w];
+  if (keep) a.kept_local[r.k2_off + pos + __popc(kbal & lanemask_lt())] = tid;
 }
 
 // ------------------------------------------------------------------ host-side launchers
@@ -556,7 +589,8 @@ cudaError_t launch_in_small(const InMeta& meta, const InArgs& a, int max_k1, cud
   cudaError_t e = nch == 1 ? launch_kernel(in_attn_small_kernel<1>, grid, dim3(128), smem, st, true, meta, a)
                            : launch_kernel(in_attn_small_kernel<2>, grid, dim3(128), smem, st, true, meta, a);
   if (e != cudaSuccess) return e;
-  return launch_kernel(in_select_small_kernel, dim3(meta.B), dim3(kSelThreads), 0, st, true, meta, a);
+  const dim3 sgrid((unsigned)meta.B, (unsigned)((max_k1 + kSelKeys - 1) / kSelKeys));
+  return launch_kernel(in_select_small_kernel, sgrid, dim3(kSelThreads), 0, st, true, meta, a);
 }
 
 cudaError_t launch_in_token_score(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
