@@ -394,6 +394,11 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
   }
   const float ia = 1.0f / sa, ib = 1.0f / sb;
   float* A = a.attn + r.attn_off + (long long)h * L * K1;
+  float* Aa = A + (long long)ra * K1;
+  float* Ab = A + (long long)rb * K1;
+  // (key, key + 1) pairs go out as one 8-byte store when every row start is 8-byte aligned
+  const bool pairs = (K1 & 1) == 0 && ((reinterpret_cast<uintptr_t>(A) & 7) == 0);
+  const bool wa = ra < L, wb = rb < L;
   float va = 0.f, vb = 0.f;
 #pragma unroll
   for (int ch = 0; ch < NCH; ++ch)
@@ -410,14 +415,19 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
         va = fmaf(pa1 - mean, pa1 - mean, va);
         vb = fmaf(pb1 - mean, pb1 - mean, vb);
       }
-      if (key < K1) {
-        if (ra < L) {
-          A[(long long)ra * K1 + key] = pa0;
-          if (key + 1 < K1) A[(long long)ra * K1 + key + 1] = pa1;
+      if (pairs) {
+        if (key < K1) {
+          if (wa) *reinterpret_cast<float2*>(Aa + key) = make_float2(pa0, pa1);
+          if (wb) *reinterpret_cast<float2*>(Ab + key) = make_float2(pb0, pb1);
         }
-        if (rb < L) {
-          A[(long long)rb * K1 + key] = pb0;
-          if (key + 1 < K1) A[(long long)rb * K1 + key + 1] = pb1;
+      } else if (key < K1) {
+        if (wa) {
+          Aa[key] = pa0;
+          if (key + 1 < K1) Aa[key + 1] = pa1;
+        }
+        if (wb) {
+          Ab[key] = pb0;
+          if (key + 1 < K1) Ab[key + 1] = pb1;
         }
       }
     }
