@@ -257,7 +257,7 @@ trevs_status validate_params(const trevs_pre_params* p) {
 trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
                            long long n_base, long long m_base, long long k1_base, uint8_t* ws,
                            const PreWs& L, cudaStream_t st, GatherMeta* gm_out, cudaEvent_t after_score = nullptr,
-                           cudaEvent_t before_score = nullptr) {
+                           cudaEvent_t before_score = nullptr, cudaStream_t tail = nullptr, int reserve = 0) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
   meta.B = b1 - b0;
@@ -298,11 +298,15 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.mode = prm.select_mode == TREVS_SELECT_FUSED ? kModeFused : kModeRatio;
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
+  a.score_reserve = reserve;
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
   if (before_score) TREVS_TRY_CUDA(cudaEventRecord(before_score, st), "event before scoring");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
   if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "event after scoring");
-  TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, st, true)), "finishing launch");
+  // the rest of stage 1 goes on `tail` (after the scoring grid completes) when given
+  if (tail) TREVS_TRY_CUDA(cudaStreamWaitEvent(tail, after_score, 0), "tail after scoring");
+  const cudaStream_t ts = tail ? tail : st;
+  TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, ts, !tail)), "finishing launch");
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
   if (bt->Z_out && ko > 0) {
@@ -321,7 +325,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     j.src_tok = bt->z_row_stride * 2; j.dst_tok = bt->z_out_row_stride * 2;
     j.src_head = 0; j.dst_head = 0; j.heads = 1; j.row_bytes = bt->d * 2;
     j.idx = a.kept; j.rows = (int)ko; j.tab = 0;
-    if (!gm_out) TREVS_TRY_CUDA(counted(launch_gather(g, st, true)), "gather launch");
+    if (!gm_out) TREVS_TRY_CUDA(counted(launch_gather(g, ts, true)), "gather launch");
   }
   return TREVS_OK;
 }
@@ -442,7 +446,7 @@ void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden,
 // `merged`: gather jobs of stage 1 to launch together with the compaction.
 trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
                           long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st, bool overlap,
-                          GatherMeta* merged, bool launch_gather_here = true) {
+                          GatherMeta* merged, bool launch_gather_here = true, bool independent = false) {
   static thread_local InMeta meta;
   static thread_local GatherMeta gm_own;
   GatherMeta& gm = merged ? *merged : gm_own;
@@ -495,6 +499,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.hs_finalize = 1;
   a.zero_p = 1;
   a.overlap = overlap ? 1 : 0;
+  a.independent = independent ? 1 : 0;
   if (in_small_fits(bt->Hq, max_l, max_k1)) {
     TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
     ++g_launches;   // two grids
@@ -515,6 +520,23 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   }
   if (launch_gather_here && gm.njobs > 0) TREVS_TRY_CUDA(counted(launch_gather(gm, st, true)), "compaction launch");
   return TREVS_OK;
+}
+
+// SMs the scoring grid leaves to stage 2's attention and selection grids when both stages
+// run in one call: in proportion to the two stages' estimated time on the whole GPU. The
+// scoring grid streams about 37 GB/s per SM; the attention share is weighted at 5 us per
+// 1024 (request, head) blocks, which puts the LLaVA-1.5 batch of 32 at the best of a sweep
+// on GB300 (24 SMs: 84.3 us per call against 88.2 without the overlap).
+int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const PreTotals& tp) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 16)
+    return 0;
+  const double score_us = (double)tp.n * pre->d * 2.0 / (37e3 * sms);
+  const double attn_us = 5.0 * (double)in->B * in->Hq / 1024.0;
+  int r = (int)((double)sms * attn_us / (score_us + attn_us) + 0.5);
+  const int lo = 8, hi = sms / 2;
+  return r < lo ? lo : (r > hi ? hi : r);
 }
 
 trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st) {
@@ -911,12 +933,32 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
   const cudaStream_t st = (cudaStream_t)stream;
   if (pre->B > 0 && in->B > 0 && pre->B <= kMaxChunk && in->B <= kMaxChunk) {
-    // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
-    // 2 (with its own compaction) forks once that grid is enqueued, so it waits for it to
-    // finish and then runs beside the fixup, selection and gather of stage 1, which occupy
-    // few SMs.
     AuxStream* aux = nullptr;
     TREVS_TRY_CUDA(aux_stream(aux), "auxiliary stream");
+    int max_l = 0, max_k1 = 0;
+    for (int b = 0; b < in->B; ++b) {
+      max_l = in->reqs[b].l > max_l ? in->reqs[b].l : max_l;
+      max_k1 = in->reqs[b].k1 > max_k1 ? in->reqs[b].k1 : max_k1;
+    }
+    const int reserve = overlap_reserve(pre, in, tp);
+    if (reserve > 0 && in_small_fits(in->Hq, max_l, max_k1)) {
+      // One chunk each, and the stages are independent. The scoring grid leaves `reserve`
+      // SMs free; stage 2 launches right behind it on the same stream (programmatic launch,
+      // its attention grid never waits for the scoring grid), so its blocks take the free SMs
+      // while the grid streams Z. The finishing grid and gather of stage 1 follow the scoring
+      // grid's completion on the auxiliary stream, which joins back at the end.
+      s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork, nullptr, aux->stream,
+                        reserve);
+      if (s != TREVS_OK) return s;
+      s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true);
+      if (s != TREVS_OK) return s;
+      TREVS_TRY_CUDA(cudaEventRecord(aux->join, aux->stream), "join");
+      TREVS_TRY_CUDA(cudaStreamWaitEvent(st, aux->join, 0), "join");
+      return TREVS_OK;
+    }
+    // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
+    // 2 (with its own compaction) forks once that grid is enqueued, so it waits for it to
+    // finish and then runs beside the finishing grid and gather of stage 1.
     s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork);
     if (s != TREVS_OK) return s;
     TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");

@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
   constexpr int NT = 8;               // n-tiles of a 64-key chunk
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ float s_upart[4];
-  pdl_wait();                         // Q, K may come from the preceding grid
+  if (!a.independent) pdl_wait();     // Q, K may come from the preceding grid
   pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = blockIdx.x / a.Hq, h = blockIdx.x - b * a.Hq;

@@ -643,11 +643,12 @@ static int sm_count() {
   return cached[dev];
 }
 
-// Persistent scoring grid: one CTA per SM, but at least four stage units per CTA.
-static int score_grid(const PreMeta& meta, int d) {
+// Persistent scoring grid: one CTA per SM (less `reserve` SMs left to concurrent work), but
+// at least four stage units per CTA.
+static int score_grid(const PreMeta& meta, int d, int reserve) {
   const long long nzs = ((d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
   const long long W = (long long)meta.total_tiles * nzs;
-  long long P = sm_count();
+  long long P = sm_count() - (reserve > 0 ? reserve : 0);
   if (P > kMaxScoreCtas) P = kMaxScoreCtas;
   if (P > W / 4) P = W / 4;
   return P < 1 ? 1 : (int)P;
@@ -677,7 +678,7 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   if (e != cudaSuccess) return e;
   e = ensure_dynamic_smem(pre_score_kernel, smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(pre_score_kernel, dim3(score_grid(meta, a.d)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
+  return launch_kernel(pre_score_kernel, dim3(score_grid(meta, a.d, a.score_reserve)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
                        tmZ2, meta, a, L);
 }
 
@@ -693,7 +694,7 @@ cudaError_t launch_pre_finish(const PreMeta& meta, const PreArgs& a, int max_m, 
   for (int b = 0; b < meta.B; ++b) jobs_of[b] = 0;
   if (scored && meta.total_tiles > 0) {
     const int nzs = ((a.d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
-    const int P = score_grid(meta, a.d);
+    const int P = score_grid(meta, a.d, a.score_reserve);
     const int W = meta.total_tiles * nzs;
     int b = 0;
     for (int c = 1; c < P; ++c) {

@@ -29,6 +29,7 @@ struct PreArgs {
   uint32_t* counters;  // [B] tiles finished per request (self-resetting)
   int4* sal;           // [B] saliency side of the selection (see saliency_prepare)
   int sal_ready;       // 1: sal was filled by the saliency kernel earlier in the stream
+  int score_reserve;   // SMs the scoring grid leaves to work that runs beside it
   uint32_t* err;       // device status word: bit 0 = a bounded wait gave up
   int d;
   int mode;
