@@ -522,18 +522,24 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   return TREVS_OK;
 }
 
-// SMs the scoring grid leaves to stage 2's attention and selection grids when both stages
-// run in one call: in proportion to the two stages' estimated time on the whole GPU. The
-// scoring grid streams about 37 GB/s per SM; the attention share is weighted at 5 us per
-// 1024 (request, head) blocks, which puts the LLaVA-1.5 batch of 32 at the best of a sweep
-// on GB300 (24 SMs: 84.3 us per call against 88.2 without the overlap).
-int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const PreTotals& tp) {
+// SMs the scoring grid leaves to stage 2's first grids when both stages run in one call:
+// in proportion to the two stages' estimated time on the whole GPU. The scoring grid streams
+// about 37 GB/s per SM. Stage 2 is weighted at 5 us per 1024 (request, head) blocks on the
+// small path and at 2.5 us per million text-to-vision logits on the larger one. Sweeps on
+// GB300 put these at or next to the best reserve: 24 SMs for the LLaVA-1.5 batch of 32
+// (84.3 us per call against 88.2 without the overlap), 48 for LLaVA-NeXT 8 x 2,880 (112.6
+// against 122.8) and for 2 x 16,384 video tokens (158.1 against 172.0).
+constexpr double LARGE_US_PER_MLOGIT = 2.5;
+
+int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const PreTotals& tp, bool small) {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 16)
     return 0;
   const double score_us = (double)tp.n * pre->d * 2.0 / (37e3 * sms);
-  const double attn_us = 5.0 * (double)in->B * in->Hq / 1024.0;
+  double logits = 0.0;
+  for (int b = 0; b < in->B; ++b) logits += (double)in->Hq * in->reqs[b].l * in->reqs[b].k1;
+  const double attn_us = small ? 5.0 * (double)in->B * in->Hq / 1024.0 : LARGE_US_PER_MLOGIT * logits * 1e-6;
   int r = (int)((double)sms * attn_us / (score_us + attn_us) + 0.5);
   const int lo = 8, hi = sms / 2;
   return r < lo ? lo : (r > hi ? hi : r);
@@ -940,8 +946,8 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
       max_l = in->reqs[b].l > max_l ? in->reqs[b].l : max_l;
       max_k1 = in->reqs[b].k1 > max_k1 ? in->reqs[b].k1 : max_k1;
     }
-    const int reserve = overlap_reserve(pre, in, tp);
-    if (reserve > 0 && in_small_fits(in->Hq, max_l, max_k1)) {
+    const int reserve = overlap_reserve(pre, in, tp, in_small_fits(in->Hq, max_l, max_k1));
+    if (reserve > 0) {
       // One chunk each, and the stages are independent. The scoring grid leaves `reserve`
       // SMs free; stage 2 launches right behind it on the same stream (programmatic launch,
       // its attention grid never waits for the scoring grid), so its blocks take the free SMs

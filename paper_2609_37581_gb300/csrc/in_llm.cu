@@ -69,7 +69,7 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
   constexpr int NT = KW / 8;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_last;
-  if (!a.overlap) pdl_wait();   // Q, K may come from the preceding grid
+  if (!a.overlap && !a.independent) pdl_wait();   // Q, K may come from the preceding grid
   pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
   }
 
   // completion of this grid implies completion of the preceding one
-  if (a.overlap) pdl_wait();
+  if (a.overlap && !a.independent) pdl_wait();
   if (!a.hs_finalize) return;
   __threadfence();
   __syncthreads();

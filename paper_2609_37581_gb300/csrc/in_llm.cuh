@@ -34,8 +34,8 @@ struct InArgs {
   int hs_finalize;          // head-statistics blocks reduce u (ticket)
   int zero_p;               // ... and clear p for the token-score pass
   int overlap;              // head statistics need not wait for the preceding grid at start
-  int independent;          // Q and K do not come from the preceding grid: the small-path
-                            // attention grid never waits for it (it may run beside it)
+  int independent;          // Q and K do not come from the preceding grid: the first
+                            // stage-2 grid never waits for it (it may run beside it)
 };
 
 }  // namespace trevs
