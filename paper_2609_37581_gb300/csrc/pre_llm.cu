@@ -386,9 +386,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 
 // Finishing grid of stage 1, one CTA per job. A job with tile >= 0 is a tile split between
 // scoring CTAs: s^t of its rows from the partial sums its contributors left, added in stage
-// order. Thread (row, q) adds column groups q, q + 4, ... of one row with all of a pass's
-// loads in flight (the data sit in L2; dependent round trips would dominate), and the four
-// partial row sums meet in shared memory. The host lists the jobs (tile, request, first
+// order, with whole rows per load instruction (an SM takes in only about 45 GB/s from L2,
+// so half-used sectors would double the time). The host lists the jobs (tile, request, first
 // contributor, contributor count, slot of the first contributor, jobs of the request);
 // requests without a split tile get one job with tile = -1. The last job of a request to
 // finish (a ticket per request, reset by that job) goes on with the request's selection
@@ -402,85 +401,89 @@ struct FinMeta {
   FinJob job[kMaxScoreCtas + kMaxChunk];
 };
 
-__device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, const PreArgs& a,
-                                  float (*red)[kTileRows], float* rt) {
+__device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, const PreArgs& a) {
+  // Warp w owns rows 8w .. 8w + 7 of the tile. A row's partial sums are mld contiguous floats:
+  // P lanes (a power of two, 4..32) read it as consecutive 16-byte groups, so each load
+  // instruction covers whole rows; lane gl of a segment owns groups gl, gl + P.
   const int row0 = (jb.tile - r.tile_off) * kTileRows;
   const int h = min(kTileRows, r.n - row0);
   const int m = r.m;
-  const int row = threadIdx.x & (kTileRows - 1), q = threadIdx.x >> 7;
   const long long sf = score_slot_floats(mld);
+  const int gpr = mld >> 2;
+  int P = 4;
+  while (P < gpr && P < 32) P <<= 1;
+  const int RPW = 32 / P;                             // rows per warp pass (<= 8)
+  const int ng = (gpr + P - 1) / P;                   // groups per lane (<= 2 for M <= 256)
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int sub = lane / P, gl = lane % P;
   const float* p0 = a.part + (2 * (long long)jb.c0 + jb.slot0) * sf;
-  for (int j = threadIdx.x; j < m; j += kFinishThreads) rt[j] = __ldcg(a.t_rinv + r.m_off + j);
-  __syncthreads();
-  const int ng = (m + 3) >> 2;
-  float sum = 0.f;
-  for (int g0 = q; g0 < ng; g0 += 16) {            // up to four groups of this thread per pass
-    float4 acc[4];
+  float rt[2][4];
+#pragma unroll
+  for (int k = 0; k < 2; ++k)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int col = 4 * (gl + P * k) + e;
+      rt[k][e] = (k < ng && col < m) ? __ldcg(a.t_rinv + r.m_off + col) : 0.f;
+    }
+  for (int pr = 0; pr < 8; pr += RPW) {
+    const int row = 8 * warp + pr + sub;
+    float4 acc[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
     float zsq = 0.f;
+    for (int x0 = 0; x0 < jb.nc; x0 += 4) {           // four contributors' loads in flight
+      float4 v[4][2];
+      float zv[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k0 = 0; k0 < jb.nc; k0 += 2) {         // two contributors' loads in flight at a time
-      float4 v[2][4];
-      float zv[2];
+      for (int x = 0; x < 4; ++x) {
+        const bool live = x0 + x < jb.nc;
+        const float* base = x0 + x == 0 ? p0 : a.part + 2 * (long long)(jb.c0 + x0 + x) * sf;
+        zv[x] = (live && gl == 0) ? __ldcg(base + (long long)kTileRows * mld + row) : 0.f;
 #pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int x = k0 + k;
-        const float* base = x == 0 ? p0 : a.part + 2 * (long long)(jb.c0 + x) * sf;
-        const bool live = x < jb.nc;
-        zv[k] = live ? __ldcg(base + (long long)kTileRows * mld + row) : 0.f;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int g = g0 + 4 * i;
-          v[k][i] = (live && g < ng) ? __ldcg(reinterpret_cast<const float4*>(base + (long long)row * mld + 4 * g))
-                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int k = 0; k < 2; ++k) {
+          const int g = gl + P * k;
+          v[x][k] = (live && k < ng && g < gpr)
+                        ? __ldcg(reinterpret_cast<const float4*>(base + (long long)row * mld + 4 * g))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
         }
       }
 #pragma unroll
-      for (int k = 0; k < 2; ++k) {                 // stage order: contributor c0 first
-        zsq += zv[k];
+      for (int x = 0; x < 4; ++x) {                   // stage order: contributor c0 first
+        zsq += zv[x];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          acc[i].x += v[k][i].x; acc[i].y += v[k][i].y; acc[i].z += v[k][i].z; acc[i].w += v[k][i].w;
+        for (int k = 0; k < 2; ++k) {
+          acc[k].x += v[x][k].x; acc[k].y += v[x][k].y; acc[k].z += v[x][k].z; acc[k].w += v[x][k].w;
         }
       }
     }
-    const float rz = zsq > 0.f ? 1.0f / sqrtf(zsq) : 0.f;
+    const float zrow = __shfl_sync(0xffffffffu, zsq, lane - gl);
+    const float rz = zrow > 0.f ? 1.0f / sqrtf(zrow) : 0.f;
+    float sum = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int g = g0 + 4 * i;
-      const float gv[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
+    for (int k = 0; k < 2; ++k) {
+      const float gv[4] = {acc[k].x, acc[k].y, acc[k].z, acc[k].w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        if (4 * g + e < m) {
-          const float xx = fmaxf(gv[e] * rt[4 * g + e] * rz, 0.f);
+        if (k < ng && 4 * (gl + P * k) + e < m) {
+          const float xx = fmaxf(gv[e] * rt[k][e] * rz, 0.f);
           sum = fmaf(xx, xx, sum);
         }
       }
     }
+    for (int o = P >> 1; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = sqrtf(sum / (float)m);
   }
-  red[q][row] = sum;
-  __syncthreads();
-  if (q == 0 && row < h)
-    a.s_t[r.n_off + row0 + row] = sqrtf(((red[0][row] + red[1][row]) + (red[2][row] + red[3][row])) / (float)m);
 }
 
 __global__ void __launch_bounds__(kFinishThreads, 1) pre_finish_kernel(const __grid_constant__ PreMeta meta,
                                                                        const __grid_constant__ FinMeta fm,
                                                                        const PreArgs a, int smem_bytes) {
   extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ union {
-    struct {
-      float red[4][kTileRows];
-      float rt[256];
-    } fx;
-    SelScratch sel;
-  } sh;
+  __shared__ SelScratch sh;
   __shared__ int s_last;
   pdl_launch_dependents();   // the next grid (the gather) waits for this one to complete
   const FinJob& jb = fm.job[blockIdx.x];
   const PreReq& r = meta.r[jb.b];
   pdl_wait();   // partial sums and s^t come from the scoring grid (1 / ||t|| and rules from before it)
-  if (jb.tile >= 0) fixup_tile(jb, r, fm.mld, a, sh.fx.red, sh.fx.rt);
+  if (jb.tile >= 0) fixup_tile(jb, r, fm.mld, a);
   if (jb.count > 1) {
     __threadfence();   // this job's s^t rows before its ticket
     __syncthreads();
@@ -495,7 +498,7 @@ __global__ void __launch_bounds__(kFinishThreads, 1) pre_finish_kernel(const __g
   } else {
     __syncthreads();
   }
-  select_request_512(a, r, jb.b, smem, smem_bytes, sh.sel);
+  select_request_512(a, r, jb.b, smem, smem_bytes, sh);
 }
 
 // Pre-pass, run ahead of the scoring grid. Blocks [0, n_sal): the saliency side of the
