@@ -529,17 +529,19 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
 // GB300 put these at or next to the best reserve: 24 SMs for the LLaVA-1.5 batch of 32
 // (84.3 us per call against 88.2 without the overlap), 48 for LLaVA-NeXT 8 x 2,880 (112.6
 // against 122.8) and for 2 x 16,384 video tokens (158.1 against 172.0).
-constexpr double LARGE_US_PER_MLOGIT = 2.5;
+constexpr double kScoreBytesPerUsPerSm = 37e3;    // 37 GB/s
+constexpr double kSmallUsPer1024Heads = 5.0;
+constexpr double kLargeUsPerMLogits = 2.5;
 
 int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const PreTotals& tp, bool small) {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 16)
     return 0;
-  const double score_us = (double)tp.n * pre->d * 2.0 / (37e3 * sms);
+  const double score_us = (double)tp.n * pre->d * 2.0 / (kScoreBytesPerUsPerSm * sms);
   double logits = 0.0;
   for (int b = 0; b < in->B; ++b) logits += (double)in->Hq * in->reqs[b].l * in->reqs[b].k1;
-  const double attn_us = small ? 5.0 * (double)in->B * in->Hq / 1024.0 : LARGE_US_PER_MLOGIT * logits * 1e-6;
+  const double attn_us = small ? kSmallUsPer1024Heads * in->B * in->Hq / 1024.0 : kLargeUsPerMLogits * logits * 1e-6;
   int r = (int)((double)sms * attn_us / (score_us + attn_us) + 0.5);
   const int lo = 8, hi = sms / 2;
   return r < lo ? lo : (r > hi ? hi : r);
