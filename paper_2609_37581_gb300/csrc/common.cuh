@@ -775,18 +775,6 @@ __device__ inline void block_fill_keys2(uint32_t* keys, const float* a, const fl
   block_key_range(l, h, s, lo, hi);
 }
 
-__device__ __forceinline__ float bf16_sq_sum8(uint4 v) {
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-  float s = 0.f;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    float2 f = __bfloat1622float2(h[j]);
-    s = fmaf(f.x, f.x, s);
-    s = fmaf(f.y, f.y, s);
-  }
-  return s;
-}
-
 // Physical 16-byte chunk of logical chunk c in a 128-byte row r (XOR swizzle, conflict-free
 // for ldmatrix and for row-wise reads).
 __device__ __forceinline__ int swz(int r, int c) { return c ^ (r & 7); }
