@@ -298,10 +298,13 @@ TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,
                                  void* workspace, size_t workspace_bytes, void* stream);
 
 /* Both stages on independent inputs (in a model the two stages are separated by the first l*
- * LLM layers). Stage 2 runs as a parallel branch on an internal stream forked from and
- * joined back into `stream` with two events; the stream and events are created on the
- * first call of each host thread on each device and kept for the thread's life. The
- * call stays asynchronous and can be captured into a CUDA graph. */
+ * LLM layers). When each stage fits one launch chunk (B <= 256), the stage-1 scoring grid
+ * leaves a few SMs free and stage 2 starts beside it on `stream` (Q and K must not be
+ * written by work still running on `stream` when the call is made); the rest of stage 1
+ * runs on an internal stream forked from and joined back into `stream` with two events.
+ * Larger batches run the stages one after the other. The internal stream and events are
+ * created on the first call of each host thread on each device and kept for the thread's
+ * life. The call stays asynchronous and can be captured into a CUDA graph. */
 TREVS_API trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_params* p,
                                 const trevs_in_batch* in,
                                 void* workspace, size_t workspace_bytes, void* stream);
