@@ -299,8 +299,7 @@ TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,
 
 /* Both stages on independent inputs (in a model the two stages are separated by the first l*
  * LLM layers). When each stage fits one launch chunk (B <= 256), the stage-1 scoring grid
- * leaves a few SMs free and stage 2 starts beside it on `stream` (Q and K must not be
- * written by work still running on `stream` when the call is made); the rest of stage 1
+ * leaves a few SMs free and stage 2 starts beside it on `stream`; the rest of stage 1
  * runs on an internal stream forked from and joined back into `stream` with two events.
  * Larger batches run the stages one after the other. The internal stream and events are
  * created on the first call of each host thread on each device and kept for the thread's
