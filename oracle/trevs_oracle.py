@@ -24,6 +24,14 @@ Readings where the paper is silent or leaves a choice open:
     text); scale 1/sqrt(d_h); query head h reads key head floor(h*Hkv/Hq).
   * Var_i in Eq. 8 is the population variance (divide by K1), two-pass.
   * H* holds n_keep_heads heads (the paper's default is half of the heads).
+  * Context preservation (Sec. 3.1): the K_d diversity tokens are drawn by farthest
+    point sampling over C = [N] minus the pivots S_r. The distance of a candidate to
+    the selected set is its smallest cosine distance 1 - cos(z_i, z_s) to any token
+    selected so far, the pivots included; each step takes the candidate of largest
+    distance (ties to the lower index). With no pivots every candidate starts at
+    distance +inf, so the first pick is the lowest index of C.
+  * K_d = floor(rho*K1 + 0.5) for a diversity share rho (the paper's K_r:K_d = 3:1 is
+    rho = 0.25); the pivots are the top K_r = K1 - K_d of the stage-1 rule.
 
 Parity pins: every function here is pinned by tests/test_oracle_pins.py against
 closed forms, hand-derived worked examples (tests/golden/), brute force on tiny
@@ -135,6 +143,47 @@ def select_fused(s_v, s_t, k1, tau_v=1.4, tau_t=1.0, lam=1.0, eps=1e-6):
     return top_k(s, k1), s
 
 
+def cosine_distance_to(Z: np.ndarray, j: int) -> np.ndarray:
+    """1 - cos(z_i, z_j) for every row i of Z (Sec. 3.1); a zero-norm row has cosine 0."""
+    Z = np.asarray(Z, dtype=np.float64)
+    nz = np.sqrt(np.sum(Z * Z, axis=1))
+    zbar = np.divide(Z, nz[:, None], out=np.zeros_like(Z), where=nz[:, None] > 0)
+    return 1.0 - zbar @ zbar[j]
+
+
+def farthest_point_sampling(Z: np.ndarray, pivots, k_d: int):
+    """Sec. 3.1 context preservation: S_d = FPS({z_i | i in C}, K_d), C = [N] minus S_r.
+
+    Z is [N, d'] (float64 values); `pivots` is S_r. Each of the K_d steps takes the
+    candidate farthest from everything selected so far: its distance is the minimum of
+    1 - cos over the selected tokens (pivots and earlier picks); ties go to the lower
+    index. Returns (picks in the order they are taken, the distance of each when taken).
+    """
+    Z = np.asarray(Z, dtype=np.float64)
+    N = len(Z)
+    cand = np.ones(N, dtype=bool)
+    dist = np.full(N, np.inf)
+    for s in np.asarray(pivots, dtype=np.int64):
+        cand[s] = False
+        dist = np.minimum(dist, cosine_distance_to(Z, int(s)))
+    if k_d < 0 or k_d > int(cand.sum()):
+        raise ValueError(f"farthest_point_sampling: K_d={k_d} outside [0, {int(cand.sum())}]")
+    picks, taken_at = [], []
+    for _ in range(k_d):
+        idx = np.flatnonzero(cand)
+        j = int(idx[np.argmax(dist[idx])])     # first maximum = lowest index among ties
+        picks.append(j)
+        taken_at.append(dist[j])
+        cand[j] = False
+        dist = np.minimum(dist, cosine_distance_to(Z, j))
+    return np.array(picks, dtype=np.int64), np.array(taken_at, dtype=np.float64)
+
+
+def diversity_count(k1: int, rho: float) -> int:
+    """K_d = floor(rho * K1 + 0.5): the diversity share of the stage-1 budget (Sec. 3.1)."""
+    return int(math.floor(float(np.float32(rho)) * k1 + 0.5))
+
+
 def gather_rows(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
     """Sec. 4.1: the kept rows, in ascending index order, are passed to the LLM."""
     return np.asarray(X)[np.asarray(idx, dtype=np.int64)]
@@ -190,8 +239,13 @@ def token_scores(A: np.ndarray, heads: np.ndarray) -> np.ndarray:
 
 
 def pre_llm_request(Z_bits, T_bits, s_v, k1, ratio, mode="ratio", tau_v=1.4, tau_t=1.0,
-                    lam=1.0, eps=1e-6):
-    """Stage 1 for one request: s^t (Eq. 4-5), selection, gather of the kept rows."""
+                    lam=1.0, eps=1e-6, diversity=0.0):
+    """Stage 1 for one request: s^t (Eq. 4-5), selection, gather of the kept rows.
+
+    With a diversity share rho > 0 the rule picks the K_r = K1 - K_d pivots S_r and
+    farthest point sampling adds K_d = floor(rho*K1 + 0.5) tokens (Sec. 3.1); the kept
+    set is S_r and S_d together, in ascending order.
+    """
     Z = bf16_bits_to_f64(Z_bits)
     T = bf16_bits_to_f64(T_bits)
     s_v = np.asarray(s_v, dtype=np.float64)
@@ -201,13 +255,19 @@ def pre_llm_request(Z_bits, T_bits, s_v, k1, ratio, mode="ratio", tau_v=1.4, tau
                 "Z_out": np.asarray(Z_bits)[:0]}
     s_t = textual_relevance(Z, T)
     out = {"s_t": s_t}
+    k_d = diversity_count(k1, diversity)
+    k_r = k1 - k_d
     if mode == "ratio":
-        kept = select_ratio(s_v, s_t, k1, ratio)
+        kept = select_ratio(s_v, s_t, k_r, ratio)
     elif mode == "fused":
-        kept, s = select_fused(s_v, s_t, k1, tau_v, tau_t, lam, eps)
+        kept, s = select_fused(s_v, s_t, k_r, tau_v, tau_t, lam, eps)
         out["s_fused"] = s
     else:
         raise ValueError(mode)
+    if k_d > 0:
+        picks, taken_at = farthest_point_sampling(Z, kept, k_d)
+        out["pivots"], out["fps"], out["fps_dist"] = kept, picks, taken_at
+        kept = np.sort(np.concatenate([kept, picks]))
     out["kept"] = kept
     out["Z_out"] = gather_rows(np.asarray(Z_bits), kept)
     return out

@@ -304,4 +304,127 @@ def pin_bf16_decode():
     assert list(got) == want
 
 
+
+# ------------------------------------------------------------- Sec. 3.1, context preservation
+
+
+def _hypercube16():
+    return np.array([[1 - 2 * ((k >> c) & 1) for c in range(4)] for k in range(16)], dtype=np.float64)
+
+
+def pin_fps_worked_example():
+    g = _golden("fps_hypercube_16.json")
+    Z = _hypercube16()
+    picks, dist = O.farthest_point_sampling(Z, g["pivots"], len(g["order"]))
+    assert list(picks) == g["order"]
+    assert list(dist) == g["dist"]
+    assert list(O.farthest_point_sampling(Z, [], 16)[0]) == g["order_no_pivots"]
+    Z0 = np.vstack([Z, np.zeros((1, 4))])
+    assert list(O.farthest_point_sampling(Z0, g["pivots"], 16)[0]) == g["order_zero_row"]
+    # positive row scales by powers of two change no bit of a cosine
+    scale = 2.0 ** np.arange(-3, 13)[:, None]
+    assert list(O.farthest_point_sampling(Z * scale, g["pivots"], 15)[0]) == g["order"]
+    # fewer picks are a prefix of the sequence
+    assert list(O.farthest_point_sampling(Z, g["pivots"], 4)[0]) == g["order"][:4]
+
+
+def _euclid_fps(Z, pivots, k):
+    """FPS by squared Euclidean distance between the unit rows, from scipy's cdist: on the
+    unit sphere |a - b|^2 = 2 (1 - cos(a, b)), so the picks are the same."""
+    from scipy.spatial.distance import cdist
+    U = Z / np.linalg.norm(Z, axis=1, keepdims=True)
+    D = cdist(U, U, "sqeuclidean")
+    sel = list(pivots)
+    picks, dists = [], []
+    for _ in range(k):
+        best, best_d = None, -1.0
+        for i in range(len(Z)):
+            if i in sel:
+                continue
+            di = min((D[i, s] for s in sel), default=np.inf)
+            if di > best_d:
+                best, best_d = i, di
+        sel.append(best)
+        picks.append(best)
+        dists.append(best_d / 2.0)
+    return picks, dists
+
+
+def pin_fps_euclidean_equivalence():
+    rng = np.random.default_rng(21)
+    for n in range(2, 13):
+        for _ in range(4):
+            Z = rng.standard_normal((n, 5))
+            kr = int(rng.integers(0, n))
+            piv = sorted(rng.choice(n, size=kr, replace=False).tolist())
+            k = n - kr
+            picks, dist = O.farthest_point_sampling(Z, piv, k)
+            want, want_d = _euclid_fps(Z, piv, k)
+            assert list(picks) == want
+            fin = np.isfinite(want_d)
+            assert list(np.isfinite(dist)) == list(fin)
+            _close(np.asarray(dist)[fin], np.asarray(want_d)[fin], 1e-9)
+
+
+def pin_fps_two_approximation():
+    """Greedy farthest-point selection covers within twice the best possible radius
+    (Gonzalez), for the Euclidean metric on the unit rows; brute force over all subsets."""
+    rng = np.random.default_rng(23)
+    for n in range(3, 10):
+        for _ in range(3):
+            Z = rng.standard_normal((n, 3))
+            U = Z / np.linalg.norm(Z, axis=1, keepdims=True)
+            E = np.sqrt(np.maximum(((U[:, None, :] - U[None, :, :]) ** 2).sum(-1), 0.0))
+            piv = [int(rng.integers(0, n))]
+            cand = [i for i in range(n) if i not in piv]
+            for k in range(1, len(cand)):
+                picks, _ = O.farthest_point_sampling(Z, piv, k)
+                S = piv + list(picks)
+                radius = max(min(E[i, s] for s in S) for i in range(n))
+                best = min(max(min(E[i, s] for s in piv + list(c)) for i in range(n))
+                           for c in itertools.combinations(cand, k))
+                assert radius <= 2.0 * best + 1e-12
+
+
+def pin_fps_invariants():
+    rng = np.random.default_rng(29)
+    Z = rng.standard_normal((40, 16))
+    piv = [3, 17, 22, 39]
+    picks, dist = O.farthest_point_sampling(Z, piv, 36)
+    assert sorted(picks) == [i for i in range(40) if i not in piv]   # K_d = |C|: all of C
+    assert np.all(np.diff(dist) <= 0)                                # distances never grow
+    p2, d2 = O.farthest_point_sampling(Z * rng.uniform(0.1, 10.0, size=(40, 1)), piv, 36)
+    assert list(p2) == list(picks)                                   # positive row scales
+    _close(d2, dist, 1e-12)
+    # an orthonormal basis: every distance is 1, so picks go in index order
+    p3, d3 = O.farthest_point_sampling(np.eye(9), [4], 8)
+    assert list(p3) == [0, 1, 2, 3, 5, 6, 7, 8] and list(d3) == [1.0] * 8
+    # a duplicate of a pivot is at distance 0 and comes last
+    Zd = np.vstack([Z[:6], Z[2:3]])
+    p4, d4 = O.farthest_point_sampling(Zd, [2], 6)
+    assert p4[-1] == 6 and abs(d4[-1]) < 1e-12
+
+
+def pin_diversity_share():
+    assert O.diversity_count(64, 0.25) == 16
+    assert O.diversity_count(192, 0.25) == 48
+    assert O.diversity_count(10, 0.25) == 3     # 2.5 rounds half up
+    assert O.diversity_count(6, 0.25) == 2      # 1.5 + 0.5
+    assert O.diversity_count(7, 0.0) == 0
+    # a request with rho > 0: the pivots are the rule's top K1 - K_d, FPS adds K_d more
+    rng = np.random.default_rng(31)
+    N, d, M, K1 = 48, 64, 5, 12
+    f32 = lambda x: (np.asarray(x, np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    Zb, Tb = f32(rng.standard_normal((N, d))), f32(rng.standard_normal((M, d)))
+    sv = rng.random(N)
+    for mode in ("fused", "ratio"):
+        r = O.pre_llm_request(Zb, Tb, sv, K1, 0.5, mode, diversity=0.25)
+        base = O.pre_llm_request(Zb, Tb, sv, K1 - 3, 0.5, mode)
+        assert list(r["pivots"]) == list(base["kept"])
+        assert len(r["fps"]) == 3 and not set(r["fps"]) & set(base["kept"])
+        assert list(r["kept"]) == sorted(list(base["kept"]) + list(r["fps"]))
+        assert list(O.pre_llm_request(Zb, Tb, sv, K1, 0.5, mode, diversity=0.0)["kept"]) == \
+            list(O.pre_llm_request(Zb, Tb, sv, K1, 0.5, mode)["kept"])
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

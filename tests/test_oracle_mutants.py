@@ -180,6 +180,60 @@ def _decode_truncating(bits):
     return (np.asarray(bits, np.uint16).astype(np.int64) / 16384.0)
 
 
+
+def _fps_generic(Z, pivots, k_d, *, use_pivots=True, setdist=np.minimum, pick="far_low", normalise=True):
+    Z = np.asarray(Z, dtype=np.float64)
+    N = len(Z)
+    nz = np.sqrt((Z * Z).sum(1))
+    U = np.divide(Z, nz[:, None], out=np.zeros_like(Z), where=nz[:, None] > 0) if normalise else Z
+    cand = np.ones(N, dtype=bool)
+    first = setdist is np.minimum
+    dist = np.full(N, np.inf if first else -np.inf)
+    for s in pivots:
+        cand[s] = False
+        if use_pivots:
+            dist = setdist(dist, 1.0 - U @ U[s])
+    picks, at = [], []
+    for _ in range(k_d):
+        idx = np.flatnonzero(cand)
+        v = dist[idx]
+        if pick == "far_low":
+            j = idx[np.argmax(v)]
+        elif pick == "far_high":
+            j = idx[len(v) - 1 - np.argmax(v[::-1])]
+        else:
+            j = idx[np.argmin(v)]
+        picks.append(int(j))
+        at.append(dist[j])
+        cand[j] = False
+        dist = setdist(dist, 1.0 - U @ U[j])
+    return np.array(picks, dtype=np.int64), np.array(at)
+
+
+def _fps_ignores_pivots(Z, pivots, k_d):
+    return _fps_generic(Z, pivots, k_d, use_pivots=False)
+
+
+def _fps_max_not_min(Z, pivots, k_d):
+    return _fps_generic(Z, pivots, k_d, setdist=np.maximum)
+
+
+def _fps_tie_high(Z, pivots, k_d):
+    return _fps_generic(Z, pivots, k_d, pick="far_high")
+
+
+def _fps_nearest(Z, pivots, k_d):
+    return _fps_generic(Z, pivots, k_d, pick="near")
+
+
+def _fps_unnormalised(Z, pivots, k_d):
+    return _fps_generic(Z, pivots, k_d, normalise=False)
+
+
+def _diversity_floor(k1, rho):
+    return int(np.floor(np.float32(rho) * k1))
+
+
 MUTANTS = {
     "cos_no_relu": ("rectified_cosine", _no_relu),
     "cos_wrong_norm": ("rectified_cosine", _wrong_norm),
@@ -211,6 +265,12 @@ MUTANTS = {
     "p_all_heads": ("token_scores", _all_heads),
     "gather_reversed": ("gather_rows", _gather_reversed),
     "bf16_decode_wrong": ("bf16_bits_to_f64", _decode_truncating),
+    "fps_ignores_pivots": ("farthest_point_sampling", _fps_ignores_pivots),
+    "fps_max_not_min": ("farthest_point_sampling", _fps_max_not_min),
+    "fps_tie_high_index": ("farthest_point_sampling", _fps_tie_high),
+    "fps_nearest": ("farthest_point_sampling", _fps_nearest),
+    "fps_unnormalised": ("farthest_point_sampling", _fps_unnormalised),
+    "diversity_floor": ("diversity_count", _diversity_floor),
 }
 
 
