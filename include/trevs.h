@@ -99,7 +99,8 @@ TREVS_API int32_t trevs_last_launch_count(void);
 /* Reads the device status word at the start of a workspace and waits for `stream` to get
  * there (the one call of this library that synchronises). TREVS_OK, or TREVS_ERR_TIMEOUT
  * if a bounded device-side wait of a call that used this workspace gave up since the
- * workspace was last zero-filled. */
+ * workspace was last zero-filled, or TREVS_ERR_INVALID_ARGUMENT if farthest point sampling
+ * found fewer candidates than draws (inputs that break its documented preconditions). */
 TREVS_API trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* stream);
 
 /* Zero-fills `bytes` of workspace on `stream` (cudaMemsetAsync). */
@@ -139,6 +140,26 @@ TREVS_API trevs_status trevs_pre_llm_select(const float* s_v, const float* s_t, 
 TREVS_API trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
                                   const int32_t* kept_idx, int32_t K1,
                                   uint16_t* Z_out, int64_t z_out_row_stride, void* stream);
+
+/* Workspace bytes for trevs_pre_llm_fps on one request of N tokens with K_r pivots. */
+TREVS_API size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r);
+
+/* Sec. 3.1 context preservation: S_d = FPS({z_i | i in C}, K_d), the K_d diversity tokens
+ * drawn by farthest point sampling in cosine distance from the candidates C = [N] minus the
+ * pivots S_r = pivots[0..K_r) (request-local rows of Z, any order; device memory).
+ * Each draw takes the candidate whose smallest distance 1 - cos(z_i, z_s) to the tokens
+ * selected so far (the pivots and the earlier draws) is largest, ties to the lower index;
+ * a zero row has cosine 0 with everything. With K_r = 0 the first draw is row 0.
+ * picks[0..K_d) receives the draws in the order they are made (the one index output of this
+ * library that is not ascending) and pick_dist[0..K_d), if non-NULL, the distance of each
+ * draw when made (+inf for the first draw without pivots). `pool` is the number of
+ * candidates whose pairwise cosines are kept on chip (0: automatic; at most 128); the draws
+ * do not depend on it beyond rounding. A pivot outside [0, N) reads as a zero row and
+ * excludes nothing. Limits: K_r <= TREVS_MAX_TEXT_TOKENS, K_r + K_d <= N, d % 8 == 0. */
+TREVS_API trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                               const int32_t* pivots, int32_t K_r, int32_t K_d, int32_t pool,
+                               int32_t* picks, float* pick_dist,
+                               void* workspace, size_t workspace_bytes, void* stream);
 
 /* ===================================================================== stage 2, one request
  *

@@ -7,6 +7,7 @@
 #include <mutex>
 #include <vector>
 
+#include "fps.cuh"
 #include "in_llm.cuh"
 #include "pre_llm.cuh"
 #include "trevs.h"
@@ -18,6 +19,7 @@ cudaError_t launch_pre_finish(const PreMeta&, const PreArgs&, int max_m, int max
                               bool pdl);
 cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
+cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 bool in_small_fits(int Hq, int max_l, int max_k1);
@@ -177,6 +179,33 @@ InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, i
   const size_t padded = (size_t)total_k1 + 4 * (size_t)kMaxChunk + 4;   // per-request 16-byte alignment
   w.keys = o;      o = al256(o + 4 * padded);
   w.flags = o;     o = al256(o + padded);
+  w.end = o;
+  return w;
+}
+
+// Farthest point sampling (Sec. 3.1), from byte offset `o` on: 1 / ||z_s|| of the pivots
+// (piv_space entries, indexed like the pivots), the partial sums of the pivot contraction
+// (up to max_kr pivots), the largest cosine of every row to its pivots, the bounds and
+// stamps of the draw, and flag / key scratch for the rows.
+// `zero` is 256 bytes that nothing writes: the row-0 pivot of a draw without pivots.
+struct FpsWs {
+  size_t zero, t_rinv, part, maxcos, ub, stamp, flags, keys, end;
+};
+
+FpsWs fps_ws(size_t o, long long total_n, long long piv_space, int max_kr) {
+  FpsWs w;
+  const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
+  if (piv_space < 1) piv_space = 1;
+  if (max_kr < 1) max_kr = 1;
+  o = al256(o);
+  w.zero = o;    o = al256(o + 256);
+  w.t_rinv = o;  o = al256(o + 4 * (size_t)(piv_space > 0 ? piv_space : 0));
+  w.part = o;    o = al256(o + (total_n > 0 && max_kr > 0 ? pre_score_part_bytes(max_kr) : 0));
+  w.maxcos = o;  o = al256(o + 4 * (size_t)total_n);
+  w.ub = o;      o = al256(o + 4 * (size_t)total_n);
+  w.stamp = o;   o = al256(o + 4 * (size_t)total_n);
+  w.flags = o;   o = al256(o + padded);
+  w.keys = o;    o = al256(o + 4 * padded);
   w.end = o;
   return w;
 }
@@ -601,6 +630,8 @@ trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* s
                  "status read");
   TREVS_TRY_CUDA(cudaStreamSynchronize((cudaStream_t)stream), "status read");
   if (word & 1u) return fail(TREVS_ERR_TIMEOUT, "a bounded device-side wait gave up (status word 0x%x)", word);
+  if (word & 2u)
+    return fail(TREVS_ERR_INVALID_ARGUMENT, "farthest point sampling found no candidate left (status word 0x%x)", word);
   return TREVS_OK;
 }
 
@@ -663,6 +694,70 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, (cudaStream_t)stream)), "pre-pass launch");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream, true)), "pre_score launch");
   TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, M, N, true, (cudaStream_t)stream, true)), "finishing launch");
+  return TREVS_OK;
+}
+
+size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r) {
+  if (N < 0 || K_r < 0) return 0;
+  return fps_ws(kStatusBytes, N, K_r, K_r).end;
+}
+
+trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
+                               const int32_t* pivots, int32_t K_r, int32_t K_d, int32_t pool, int32_t* picks,
+                               float* pick_dist, void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  TREVS_CHECK(N >= 0 && K_r >= 0 && K_d >= 0, "N = %d, K_r = %d, K_d = %d: none may be negative", N, K_r, K_d);
+  TREVS_CHECK((long long)K_r + K_d <= N, "K_r + K_d = %lld exceeds N = %d", (long long)K_r + K_d, N);
+  TREVS_CHECK(pool >= 0, "pool = %d < 0", pool);
+  if (K_r > TREVS_MAX_TEXT_TOKENS)
+    return fail(TREVS_ERR_UNSUPPORTED, "K_r = %d > %d pivots", K_r, TREVS_MAX_TEXT_TOKENS);
+  if (K_d == 0) return TREVS_OK;
+  TREVS_CHECK(d >= 8 && d % 8 == 0, "d = %d must be a positive multiple of 8", d);
+  TREVS_CHECK(Z != nullptr && aligned16(Z), "Z must be non-NULL and 16-byte aligned");
+  TREVS_CHECK(z_row_stride >= d && z_row_stride % 8 == 0, "z_row_stride must be >= d and a multiple of 8");
+  TREVS_CHECK(K_r == 0 || pivots != nullptr, "pivots is NULL");
+  TREVS_CHECK(picks != nullptr, "picks is NULL");
+  const FpsWs L = fps_ws(kStatusBytes, N, K_r, K_r);
+  trevs_status s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  const cudaStream_t st = (cudaStream_t)stream;
+  float* maxcos = reinterpret_cast<float*>(ws + L.maxcos);
+  // without pivots row 0 is the first draw and the one pivot of the contraction
+  const int lead = K_r == 0 ? 1 : 0;
+  const int kr = K_r + lead;
+  const int32_t* piv = lead ? reinterpret_cast<const int32_t*>(ws + L.zero) : pivots;
+  {   // the largest cosine of every row to the pivots: the scoring contraction
+    static thread_local PreMeta meta;
+    meta.B = 1;
+    meta.r[0] = PreReq{0, N, 0, kr, 0, 0, 0, 0};
+    meta.total_tiles = (N + kScoreTileRows - 1) / kScoreTileRows;
+    PreArgs a;
+    memset(&a, 0, sizeof(a));
+    a.Z = reinterpret_cast<const __nv_bfloat16*>(Z); a.z_stride = z_row_stride;
+    a.t_idx = piv;
+    a.s_t = maxcos;
+    a.t_rinv = reinterpret_cast<float*>(ws + L.t_rinv);
+    a.total_m = kr;
+    a.part = reinterpret_cast<float*>(ws + L.part);
+    a.err = reinterpret_cast<uint32_t*>(ws);
+    a.d = d; a.mode = kModeRatio; a.action = kActFpsSeed;
+    TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, st)), "pivot norms launch");
+    TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, kr, N, st, true)), "pivot contraction launch");
+    TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, kr, N, true, st, true)), "pivot fixup launch");
+  }
+  static thread_local FpsMeta fm;
+  fm.B = 1;
+  fm.r[0] = FpsReq{0, N, 0, kr, K_d, lead, 0, 0};
+  FpsArgs f;
+  memset(&f, 0, sizeof(f));
+  f.Z = reinterpret_cast<const __nv_bfloat16*>(Z); f.z_stride = z_row_stride; f.d = d;
+  f.piv = piv; f.maxcos = maxcos;
+  f.ub = reinterpret_cast<float*>(ws + L.ub); f.stamp = reinterpret_cast<int*>(ws + L.stamp);
+  f.flags = ws + L.flags; f.keys = reinterpret_cast<uint32_t*>(ws + L.keys);
+  f.picks = picks; f.pick_dist = pick_dist; f.kept = nullptr; f.pool = pool;
+  f.err = reinterpret_cast<uint32_t*>(ws);
+  TREVS_TRY_CUDA(counted(launch_fps(fm, f, st, true)), "farthest point sampling launch");
   return TREVS_OK;
 }
 

@@ -89,6 +89,9 @@ __device__ __forceinline__ void for_each_subtile(const PreMeta& meta, int nzs, l
   }
 }
 
+// kSeed: the pivot rows of Z stand in for the text rows (t_idx) and each row's output is the
+// largest cosine to them, unrectified (the distances of farthest point sampling, Sec. 3.1).
+template <bool kSeed>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     pre_score_kernel(const __grid_constant__ CUtensorMap tmZ3, const __grid_constant__ CUtensorMap tmZ2,
                      const __grid_constant__ PreMeta meta, const PreArgs a, const ScoreLaunch L) {
@@ -235,7 +238,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
       const PreReq& r = meta.r[st.b];
       const int pieces = r.m * 8;
-      const uint8_t* tsrc = reinterpret_cast<const uint8_t*>(a.T + (long long)r.m_off * a.t_stride);
+      const uint8_t* tsrc = kSeed ? nullptr : reinterpret_cast<const uint8_t*>(a.T + (long long)r.m_off * a.t_stride);
       for (int zs = st.zs0; zs < st.zs1; ++zs) {
         const int ns = min(kZSlices, nk - zs * kZSlices);
         for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
@@ -252,8 +255,15 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             for (int p = ct; p < pieces; p += kTCopyThreads) {
               const int row = p >> 3, q = p & 7;
               const int col = kc * kChunk + q * 8;
-              const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
-              cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, col < d ? 16 : 0);   // zero past d'
+              if constexpr (kSeed) {
+                const int zi = __ldg(a.t_idx + r.m_off + row);
+                const bool ok = col < d && zi >= 0 && zi < r.n;
+                const __nv_bfloat16* src = ok ? a.Z + ((long long)r.n_off + zi) * a.z_stride + col : a.Z;
+                cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, ok ? 16 : 0);
+              } else {
+                const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
+                cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, col < d ? 16 : 0);   // zero past d'
+              }
             }
           }
           cp_async_arrive_noinc(smem_u32(&tfull[ts]));
@@ -327,7 +337,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       const uint32_t lane_base = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * L.acc_cols);
       const float zsq = zsq_s[buf][0][row] + zsq_s[buf][1][row];
       const float rz = zsq > 0.f ? 1.0f / sqrtf(zsq) : 0.f;
-      float sum = 0.f;
+      float sum = 0.f, mx = -INFINITY;
       if (st.slot < 0) {
         for (int c0 = 0; c0 < m; c0 += 32) {
           float v[32];
@@ -335,8 +345,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 #pragma unroll
           for (int jj = 0; jj < 32; ++jj) {
             if (c0 + jj < m) {
-              const float x = fmaxf(v[jj] * rt[c0 + jj] * rz, 0.f);
-              sum = fmaf(x, x, sum);
+              if constexpr (kSeed) {
+                mx = fmaxf(mx, v[jj] * rt[c0 + jj] * rz);
+              } else {
+                const float x = fmaxf(v[jj] * rt[c0 + jj] * rz, 0.f);
+                sum = fmaf(x, x, sum);
+              }
             }
           }
         }
@@ -361,7 +375,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         mbar_arrive(smem_u32(&acc_empty[buf]));
         mbar_arrive(smem_u32(&norm_empty[buf]));
       }
-      if (st.slot < 0 && row < st.h) a.s_t[r.n_off + st.row0 + row] = sqrtf(sum / (float)m);
+      if (st.slot < 0 && row < st.h) a.s_t[r.n_off + st.row0 + row] = kSeed ? mx : sqrtf(sum / (float)m);
       ++j;
       return true;
     });
@@ -401,6 +415,7 @@ struct FinMeta {
   FinJob job[kMaxScoreCtas + kMaxChunk];
 };
 
+template <bool kSeed>
 __device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, const PreArgs& a) {
   // Warp w owns rows 8w .. 8w + 7 of the tile. A row's partial sums are mld contiguous floats:
   // P lanes (a power of two, 4..32) read it as consecutive 16-byte groups, so each load
@@ -456,20 +471,29 @@ __device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, co
     }
     const float zrow = __shfl_sync(0xffffffffu, zsq, lane - gl);
     const float rz = zrow > 0.f ? 1.0f / sqrtf(zrow) : 0.f;
-    float sum = 0.f;
+    float sum = 0.f, mx = -INFINITY;
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
       const float gv[4] = {acc[k].x, acc[k].y, acc[k].z, acc[k].w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         if (k < ng && 4 * (gl + P * k) + e < m) {
-          const float xx = fmaxf(gv[e] * rt[k][e] * rz, 0.f);
-          sum = fmaf(xx, xx, sum);
+          if constexpr (kSeed) {
+            mx = fmaxf(mx, gv[e] * rt[k][e] * rz);
+          } else {
+            const float xx = fmaxf(gv[e] * rt[k][e] * rz, 0.f);
+            sum = fmaf(xx, xx, sum);
+          }
         }
       }
     }
-    for (int o = P >> 1; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = sqrtf(sum / (float)m);
+    if constexpr (kSeed) {
+      for (int o = P >> 1; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = mx;
+    } else {
+      for (int o = P >> 1; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = sqrtf(sum / (float)m);
+    }
   }
 }
 
@@ -483,7 +507,11 @@ __global__ void __launch_bounds__(kFinishThreads, 1) pre_finish_kernel(const __g
   const FinJob& jb = fm.job[blockIdx.x];
   const PreReq& r = meta.r[jb.b];
   pdl_wait();   // partial sums and s^t come from the scoring grid (1 / ||t|| and rules from before it)
-  if (jb.tile >= 0) fixup_tile(jb, r, fm.mld, a);
+  if (a.action == kActFpsSeed) {   // pivot cosines: the split tiles only
+    if (jb.tile >= 0) fixup_tile<true>(jb, r, fm.mld, a);
+    return;
+  }
+  if (jb.tile >= 0) fixup_tile<false>(jb, r, fm.mld, a);
   if (jb.count > 1) {
     __threadfence();   // this job's s^t rows before its ticket
     __syncthreads();
@@ -514,7 +542,20 @@ __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant
     const long long row = (long long)(blockIdx.x - n_sal) * 16 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= a.total_m) return;
-    const uint4* t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
+    const uint4* t;
+    if (a.t_idx) {   // the pivot rows of Z (farthest point sampling): request b owns [m_off, m_off + m)
+      const int b = find_request(meta.B, (int)row, [&](int i) { return meta.r[i].m_off; });
+      const PreReq& r = meta.r[b];
+      if ((int)row - r.m_off >= r.m) return;
+      const int zi = __ldg(a.t_idx + row);
+      if (zi < 0 || zi >= r.n) {
+        if (lane == 0) a.t_rinv[row] = 0.f;
+        return;
+      }
+      t = reinterpret_cast<const uint4*>(a.Z + ((long long)r.n_off + zi) * a.z_stride);
+    } else {
+      t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
+    }
     const int nv = a.d / 8;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int p0 = 0; p0 < nv; p0 += 16 * 32) {
@@ -679,9 +720,10 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   if (e != cudaSuccess) return e;
   e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, kZBoxRows);
   if (e != cudaSuccess) return e;
-  e = ensure_dynamic_smem(pre_score_kernel, smem);
+  auto kernel = a.t_idx ? pre_score_kernel<true> : pre_score_kernel<false>;
+  e = ensure_dynamic_smem(kernel, smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(pre_score_kernel, dim3(score_grid(meta, a.d, a.score_reserve)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
+  return launch_kernel(kernel, dim3(score_grid(meta, a.d, a.score_reserve)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
                        tmZ2, meta, a, L);
 }
 
@@ -716,7 +758,7 @@ cudaError_t launch_pre_finish(const PreMeta& meta, const PreArgs& a, int max_m, 
       ++jobs_of[b];
     }
   }
-  const bool per_request = a.action != kActScores;
+  const bool per_request = a.action != kActScores && a.action != kActFpsSeed;
   if (per_request)
     for (int b = 0; b < meta.B; ++b)
       if (jobs_of[b] == 0 && meta.r[b].n > 0) {

@@ -80,6 +80,9 @@ _SIGS = {
     "trevs_pre_llm_select": (_c_i32, [_vp, _vp, _vp, _c_i32, _c_i32, _c_f32, ctypes.POINTER(PreParams),
                                       _vp, _vp, _c_sz, _vp]),
     "trevs_pre_llm_gather": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _vp, _c_i64, _vp]),
+    "trevs_pre_llm_fps_workspace_size": (_c_sz, [_c_i32, _c_i32]),
+    "trevs_pre_llm_fps": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _c_i32, _c_i32, _vp, _vp,
+                                   _vp, _c_sz, _vp]),
     "trevs_in_llm_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
     "trevs_in_llm_head_scores": (_c_i32, [_vp, _c_i64, _c_i64, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
                                           _c_i32, _c_i32, _c_i32, _c_f32, _vp, _vp, _vp, _c_sz, _vp]),
@@ -201,6 +204,20 @@ def trevs_pre_llm_gather(Z, kept_idx, Z_out, stream=None):
     N, d = Z.shape
     check(load().trevs_pre_llm_gather(_ptr(Z), Z.stride(0), N, d, _ptr(kept_idx), kept_idx.numel(),
                                       _ptr(Z_out), Z_out.stride(0), _stream(stream)))
+
+
+def trevs_pre_llm_fps_workspace_size(N, K_r):
+    return int(load().trevs_pre_llm_fps_workspace_size(N, K_r))
+
+
+def trevs_pre_llm_fps(Z, pivots, K_d, picks, pick_dist=None, pool=0, ws=None, stream=None):
+    """Sec. 3.1 context preservation: K_d draws of farthest point sampling over the rows of Z
+    that are not in `pivots` (int32, may be None for none), in draw order into `picks`."""
+    N, d = Z.shape
+    K_r = 0 if pivots is None else pivots.numel()
+    w, nb = _ws_args(ws)
+    check(load().trevs_pre_llm_fps(_ptr(Z), Z.stride(0), N, d, _ptr(pivots), K_r, K_d, pool, _ptr(picks),
+                                   _ptr(pick_dist), w, nb, _stream(stream)))
 
 
 def trevs_in_llm_head_scores(Q, K, Hq, Hkv, L, K1, u_out, attn_out, q_strides, k_strides,

@@ -85,6 +85,32 @@ def test_scores_validation(lib):
     assert lib.trevs_pre_llm_scores(None, 0, 0, 4096, None, 0, 0, None, None, None, None, None, 0, None) == 0
 
 
+def test_fps_validation(lib):
+    need = lib.trevs_pre_llm_fps_workspace_size(576, 48)
+    assert need > 0 and need % 256 == 0
+    assert lib.trevs_pre_llm_fps_workspace_size(576, 48) > lib.trevs_pre_llm_fps_workspace_size(100, 48)
+    assert lib.trevs_pre_llm_fps_workspace_size(-1, 0) == 0
+
+    def fps(N=576, d=4096, K_r=48, K_d=16, pool=0, zs=4096, Z=FAKE, piv=FAKE, picks=FAKE, ws=FAKE, nb=need):
+        return lib.trevs_pre_llm_fps(Z, zs, N, d, piv, K_r, K_d, pool, picks, None, ws, nb, None)
+    assert fps(K_r=500, K_d=100) == t.TREVS_ERR_INVALID_ARGUMENT          # K_r + K_d > N
+    assert "exceeds" in _err(lib)
+    assert fps(K_d=-1) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(pool=-2) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(K_r=257, N=1000) == t.TREVS_ERR_UNSUPPORTED               # pivots play the text rows
+    assert fps(d=4100, zs=4100) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(zs=4000) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(Z=ctypes.c_void_p(0x10002)) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(piv=None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(picks=None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert fps(nb=need - 1) == t.TREVS_ERR_WORKSPACE
+    assert fps(ws=ctypes.c_void_p(0x10010)) == t.TREVS_ERR_WORKSPACE
+    # K_d = 0 is a valid no-op, and so is an empty request
+    assert fps(K_d=0, Z=None, piv=None, picks=None, ws=None, nb=0) == 0
+    assert fps(N=0, K_r=0, K_d=0, Z=None, piv=None, picks=None, ws=None, nb=0) == 0
+    assert t.last_launch_count() == 0
+
+
 def test_stage2_validation(lib):
     def hs(Hq, Hkv, L, K1, dh):
         return lib.trevs_in_llm_head_scores(FAKE, 4096, 128, FAKE, 8192, 128, Hq, Hkv, L, K1, dh, 0.0,
