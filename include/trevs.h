@@ -76,6 +76,10 @@ typedef struct trevs_pre_params {
   float lambda;        /* consistency-reward weight, default 1.0 */
   float eps;           /* MAD stabiliser, default 1e-6 (the paper leaves it unstated) */
   int32_t select_mode; /* TREVS_SELECT_RATIO (default) or TREVS_SELECT_FUSED */
+  float diversity;     /* share rho of K1 drawn by farthest point sampling (Sec. 3.1 context
+                          preservation): K_d = floor(rho*K1 + 1/2) tokens join the K1 - K_d
+                          pivots of the rule above; the paper's K_r:K_d = 3:1 is 0.25.
+                          Default 0 (no draws). Batched calls only. */
 } trevs_pre_params;
 
 /* Limits of this build (TREVS_ERR_UNSUPPORTED beyond them). */
@@ -296,7 +300,11 @@ TREVS_API size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch)
 TREVS_API size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in);
 
 /* Stage 1 for a batch: Eq. 4-5 scores, selection (ratio or fused, *p; NULL = defaults)
- * and gather of the kept rows. */
+ * and gather of the kept rows. With p->diversity = rho > 0 (Sec. 3.1 context preservation)
+ * the rule keeps K_r = K1 - K_d pivots (the ratio split applies to K_r), farthest point
+ * sampling (as trevs_pre_llm_fps) adds K_d = floor(rho*K1 + 1/2) tokens, and kept_idx holds
+ * both sets together in ascending order. TREVS_ERR_UNSUPPORTED if some request would have
+ * more than TREVS_MAX_TEXT_TOKENS pivots. */
 TREVS_API trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_params* p,
                                   void* workspace, size_t workspace_bytes, void* stream);
 

@@ -140,24 +140,38 @@ inline size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 constexpr size_t kStatusBytes = 256;
 
 struct PreWs {
-  size_t counters, sal, t_rinv, part, s_t, s_fused, keys, flags, end;
+  size_t counters, sal, t_rinv, part, s_t, s_fused, keys, flags;
+  size_t fps_zero, fps_rinv, fps_maxcos, fps_ub, fps_stamp, fps_picks, end;
 };
 
 // Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request;
 // t_rinv holds 1 / ||t_j|| of the text rows; part the partial sums of the scoring tiles
-// that two or more scoring CTAs share (up to max_m text rows).
-PreWs pre_ws(long long total_n, long long total_m, int max_m) {
+// that two or more scoring CTAs share (up to max_m text rows, or up to the pivots of the
+// farthest-point contraction, min(max_k1, TREVS_MAX_TEXT_TOKENS), which reuses it). The
+// fps_* regions serve farthest point sampling (Sec. 3.1) when the call asks for it: a
+// 256-byte zero block, 1 / ||z|| of the pivots and the draws (indexed like kept_idx), and
+// the largest pivot cosine, bound and stamp of every row.
+PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1 = 0, int max_k1 = 0) {
   PreWs w;
   const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
+  const int max_kr = max_k1 < TREVS_MAX_TEXT_TOKENS ? max_k1 : TREVS_MAX_TEXT_TOKENS;
+  const int part_rows = max_m > max_kr ? max_m : max_kr;
+  const size_t k1 = (size_t)(total_k1 > 0 ? total_k1 : 0), fn = total_k1 > 0 ? (size_t)total_n : 0;
   size_t o = kStatusBytes;
   w.counters = o; o = al256(o + 4 * (size_t)kMaxChunk);
   w.sal = o;      o = al256(o + 16 * (size_t)kMaxChunk);
   w.t_rinv = o;   o = al256(o + 4 * (size_t)(total_m > 0 ? total_m : 0));
-  w.part = o;     o = al256(o + (total_n > 0 ? pre_score_part_bytes(max_m > 0 ? max_m : 1) : 0));
+  w.part = o;     o = al256(o + (total_n > 0 ? pre_score_part_bytes(part_rows > 0 ? part_rows : 1) : 0));
   w.s_t = o;      o = al256(o + 4 * (size_t)total_n);
   w.s_fused = o;  o = al256(o + 4 * (size_t)total_n);
   w.keys = o;     o = al256(o + 4 * padded);
   w.flags = o;    o = al256(o + padded);
+  w.fps_zero = o;   o = al256(o + (k1 > 0 ? 256 : 0));
+  w.fps_rinv = o;   o = al256(o + 4 * k1);
+  w.fps_picks = o;  o = al256(o + 4 * k1);
+  w.fps_maxcos = o; o = al256(o + 4 * fn);
+  w.fps_ub = o;     o = al256(o + 4 * fn);
+  w.fps_stamp = o;  o = al256(o + 4 * fn);
   w.end = o;
   return w;
 }
@@ -227,7 +241,7 @@ int textual_count(int k1, float ratio) {
 
 struct PreTotals {
   long long n = 0, m = 0, k1 = 0;
-  int max_n = 0, max_m = 0;
+  int max_n = 0, max_m = 0, max_k1 = 0;
 };
 
 trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
@@ -251,6 +265,7 @@ trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
     }
     t.n += r.n; t.m += r.m; t.k1 += r.k1;
     t.max_n = r.n > t.max_n ? r.n : t.max_n;
+    t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
     if (r.n > 0) t.max_m = r.m > t.max_m ? r.m : t.max_m;   // requests without visual rows score nothing
   }
   TREVS_CHECK(t.n < (1ll << 31) && t.m < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
@@ -277,6 +292,26 @@ trevs_status validate_params(const trevs_pre_params* p) {
   TREVS_CHECK(std::isfinite(p->tau_v) && p->tau_v > 0.f && std::isfinite(p->tau_t) && p->tau_t > 0.f,
               "temperatures must be positive");
   TREVS_CHECK(std::isfinite(p->lambda) && std::isfinite(p->eps) && p->eps >= 0.f, "lambda / eps invalid");
+  TREVS_CHECK(std::isfinite(p->diversity) && p->diversity >= 0.f && p->diversity <= 1.f,
+              "diversity share %g outside [0, 1]", (double)p->diversity);
+  return TREVS_OK;
+}
+
+// K_d = floor(rho * K1 + 1/2): the tokens farthest point sampling adds to the K1 - K_d
+// pivots of the selection rule (Sec. 3.1).
+int diversity_count(int k1, float rho) {
+  int kd = (int)std::floor((double)rho * (double)k1 + 0.5);
+  return kd < 0 ? 0 : (kd > k1 ? k1 : kd);
+}
+
+// Pivots above TREVS_MAX_TEXT_TOKENS do not fit the contraction that measures distances.
+trevs_status validate_diversity(const trevs_pre_batch* bt, const trevs_pre_params& p) {
+  if (p.diversity <= 0.f) return TREVS_OK;
+  for (int b = 0; b < bt->B; ++b) {
+    const int k1 = bt->reqs[b].k1, kd = diversity_count(k1, p.diversity);
+    if (kd > 0 && k1 - kd > TREVS_MAX_TEXT_TOKENS)
+      return fail(TREVS_ERR_UNSUPPORTED, "request %d: %d pivots (K1 - K_d) > %d", b, k1 - kd, TREVS_MAX_TEXT_TOKENS);
+  }
   return TREVS_OK;
 }
 
@@ -289,14 +324,20 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
                            cudaEvent_t before_score = nullptr, cudaStream_t tail = nullptr, int reserve = 0) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
+  static thread_local int kd_of[kMaxChunk];
   meta.B = b1 - b0;
   int tiles = 0, max_n = 0, max_m = 0;
+  bool draws = false;
   long long no = 0, mo = 0, ko = 0;
   for (int b = b0; b < b1; ++b) {
     const trevs_pre_request& q = bt->reqs[b];
     PreReq& r = meta.r[b - b0];
+    // with a diversity share the rule picks the K_r = K1 - K_d pivots (Sec. 3.1)
+    const int kd = prm.diversity > 0.f ? diversity_count(q.k1, prm.diversity) : 0;
+    kd_of[b - b0] = kd;
+    draws = draws || kd > 0;
     r.n_off = (int)no; r.n = q.n; r.m_off = (int)mo; r.m = q.m;
-    r.k1_off = (int)ko; r.k1 = q.k1; r.kt = textual_count(q.k1, q.ratio);
+    r.k1_off = (int)ko; r.k1 = q.k1 - kd; r.kt = textual_count(q.k1 - kd, q.ratio);
     r.tile_off = tiles;
     tiles += (q.n + kScoreTileRows - 1) / kScoreTileRows;
     no += q.n; mo += q.m; ko += q.k1;
@@ -336,6 +377,48 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   if (tail) TREVS_TRY_CUDA(cudaStreamWaitEvent(tail, after_score, 0), "tail after scoring");
   const cudaStream_t ts = tail ? tail : st;
   TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, ts, !tail)), "finishing launch");
+  if (draws) {
+    // Farthest point sampling of the K_d diversity tokens (Sec. 3.1) behind the pivots: the
+    // scoring contraction again, over the requests that draw, with their pivots (kept_idx)
+    // as the text rows; then one block per request draws and writes S_r and S_d together.
+    static thread_local PreMeta dm;
+    static thread_local FpsMeta fm;
+    dm.B = 0;
+    fm.B = 0;
+    int dtiles = 0, max_kr = 0;
+    for (int i = 0; i < meta.B; ++i) {
+      const int kd = kd_of[i];
+      if (kd <= 0) continue;
+      const PreReq& r = meta.r[i];
+      const int lead = r.k1 == 0 ? 1 : 0;   // no pivots: row 0 is the first draw and the pivot
+      const int kr = r.k1 + lead;
+      if (lead)
+        TREVS_TRY_CUDA(counted(cudaMemsetAsync(a.kept + r.k1_off, 0, sizeof(int32_t), ts)), "row-0 pivot");
+      dm.r[dm.B++] = PreReq{r.n_off, r.n, r.k1_off, kr, 0, 0, 0, dtiles};
+      dtiles += (r.n + kScoreTileRows - 1) / kScoreTileRows;
+      max_kr = kr > max_kr ? kr : max_kr;
+      fm.r[fm.B++] = FpsReq{r.n_off, r.n, r.k1_off, kr, kd, lead, r.k1_off, r.k1_off};
+    }
+    dm.total_tiles = dtiles;
+    PreArgs da = a;
+    da.t_idx = a.kept;
+    da.s_t = reinterpret_cast<float*>(ws + L.fps_maxcos);
+    da.t_rinv = reinterpret_cast<float*>(ws + L.fps_rinv);
+    da.total_m = ko;
+    da.action = kActFpsSeed;
+    TREVS_TRY_CUDA(counted(launch_pre_saliency(dm, da, max_n, false, ts)), "pivot norms launch");
+    TREVS_TRY_CUDA(counted(launch_pre_score(dm, da, max_kr, no, ts, true)), "pivot contraction launch");
+    TREVS_TRY_CUDA(counted(launch_pre_finish(dm, da, max_kr, max_n, true, ts, true)), "pivot fixup launch");
+    FpsArgs f;
+    memset(&f, 0, sizeof(f));
+    f.Z = a.Z; f.z_stride = a.z_stride; f.d = a.d;
+    f.piv = a.kept; f.maxcos = da.s_t;
+    f.ub = reinterpret_cast<float*>(ws + L.fps_ub); f.stamp = reinterpret_cast<int*>(ws + L.fps_stamp);
+    f.flags = a.flags; f.keys = a.keys;
+    f.picks = reinterpret_cast<int*>(ws + L.fps_picks); f.pick_dist = nullptr;
+    f.kept = a.kept; f.pool = 0; f.err = a.err;
+    TREVS_TRY_CUDA(counted(launch_fps(fm, f, ts, true)), "farthest point sampling launch");
+  }
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
   if (bt->Z_out && ko > 0) {
@@ -598,7 +681,7 @@ trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, 
   return TREVS_OK;
 }
 
-const trevs_pre_params kDefaults = {1.4f, 1.0f, 1.0f, 1e-6f, TREVS_SELECT_RATIO};
+const trevs_pre_params kDefaults = {1.4f, 1.0f, 1.0f, 1e-6f, TREVS_SELECT_RATIO, 0.0f};
 
 }  // namespace
 
@@ -951,15 +1034,17 @@ trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_str
 
 size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
-  long long n = 0, m = 0;
-  int max_m = 0;
+  long long n = 0, m = 0, k1 = 0;
+  int max_m = 0, max_k1 = 0;
   for (int b = 0; b < batch->B; ++b) {
     const trevs_pre_request& r = batch->reqs[b];
     n += r.n > 0 ? r.n : 0;
     m += r.m > 0 ? r.m : 0;
+    k1 += r.k1 > 0 ? r.k1 : 0;
     if (r.n > 0 && r.m > max_m) max_m = r.m;
+    if (r.k1 > max_k1) max_k1 = r.k1;
   }
-  return pre_ws(n, m, max_m).end;
+  return pre_ws(n, m, max_m, k1, max_k1).end;
 }
 
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
@@ -986,7 +1071,9 @@ trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_
   PreTotals t;
   s = validate_pre_batch(batch, t);
   if (s != TREVS_OK || batch->B == 0) return s;
-  const PreWs L = pre_ws(t.n, t.m, t.max_m);
+  s = validate_diversity(batch, prm);
+  if (s != TREVS_OK) return s;
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -1005,7 +1092,9 @@ trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, const trev
   if (s != TREVS_OK) return s;
   TREVS_CHECK(batch->B >= 1, "B = 0: nothing to time");
   if (batch->B > kMaxChunk) return fail(TREVS_ERR_UNSUPPORTED, "B = %d > %d requests", batch->B, kMaxChunk);
-  const PreWs L = pre_ws(t.n, t.m, t.max_m);
+  s = validate_diversity(batch, prm);
+  if (s != TREVS_OK) return s;
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_chunk(batch, prm, 0, batch->B, 0, 0, 0, reinterpret_cast<uint8_t*>(workspace), L,
@@ -1036,7 +1125,9 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   s = validate_in_batch(in, ti);
   if (s != TREVS_OK) return s;
-  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m);
+  s = validate_diversity(pre, prm);
+  if (s != TREVS_OK) return s;
+  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
   const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);

@@ -38,7 +38,7 @@ class TrevsError(RuntimeError):
 
 class PreParams(ctypes.Structure):
     _fields_ = [("tau_v", _c_f32), ("tau_t", _c_f32), ("lambda_", _c_f32), ("eps", _c_f32),
-                ("select_mode", _c_i32)]
+                ("select_mode", _c_i32), ("diversity", _c_f32)]
 
 
 class PreRequest(ctypes.Structure):

@@ -44,6 +44,7 @@ def test_version_and_defaults(lib):
     assert t.version().count(".") == 2
     p = t.default_params()
     assert (round(p.tau_v, 6), p.tau_t, p.lambda_, p.select_mode) == (1.4, 1.0, 1.0, t.SELECT_RATIO)
+    assert p.diversity == 0.0
     assert abs(p.eps - 1e-6) < 1e-12
 
 
@@ -164,6 +165,25 @@ def test_varlen_validation(lib):
     assert lib.trevs_pre_llm_varlen(ctypes.byref(ok), None, FAKE, need - 256, None) == t.TREVS_ERR_WORKSPACE
     empty = t.PreBatchC()
     assert lib.trevs_pre_llm_varlen(ctypes.byref(empty), None, None, 0, None) == 0
+
+
+def test_varlen_diversity_validation(lib):
+    ok = _pre_batch([(576, 32, 64, 0.5), (2880, 64, 320, 0.5)])
+    need = lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(ok))
+    for rho in (-0.1, 1.5, float("nan")):
+        p = t.default_params(t.SELECT_FUSED, diversity=rho)
+        assert lib.trevs_pre_llm_varlen(ctypes.byref(ok), ctypes.byref(p), FAKE, need, None) == \
+            t.TREVS_ERR_INVALID_ARGUMENT
+        assert "diversity" in _err(lib)
+    # K1 = 1024 at rho = 0.25 leaves 768 pivots: more than the contraction takes
+    big = _pre_batch([(16384, 128, 1024, 0.5)], d=3584)
+    nb = lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(big))
+    p = t.default_params(t.SELECT_FUSED, diversity=0.25)
+    assert lib.trevs_pre_llm_varlen(ctypes.byref(big), ctypes.byref(p), FAKE, nb, None) == t.TREVS_ERR_UNSUPPORTED
+    assert "pivots" in _err(lib)
+    # at rho = 0.75 the same request has 256 pivots, which fit: validation passes up to the workspace
+    p = t.default_params(t.SELECT_FUSED, diversity=0.75)
+    assert lib.trevs_pre_llm_varlen(ctypes.byref(big), ctypes.byref(p), FAKE, nb - 256, None) == t.TREVS_ERR_WORKSPACE
 
 
 def test_varlen_timed_validation(lib):
