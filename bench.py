@@ -45,6 +45,7 @@ UNIT = "visual tokens/s"
 WORKLOAD = dict(k1=64, ratio=0.5, k2=32)
 ROTATING_SETS = 4
 DOMINANT = "pre_score_kernel"
+METHOD_RHO = 0.25   # K_r:K_d = 3:1, the paper's setting for the diversity draws (Sec. 3.1)
 
 
 def workload():
@@ -72,7 +73,12 @@ def algorithmic_bytes(w):
     stage1 = score + sk1 * w.d * 2
     stage2 = (sl * w.hq * w.dh * 2 + sk1 * w.hkv * w.dh * 2
               + 2 * sk2 * (w.d + 2 * w.hkv * w.dh) * 2 + sk2 * 4)
-    return {"score_kernel": score, "stage1": stage1, "stage2": stage2, "step": stage1 + stage2}
+    # the diversity draws need the distances of every row to the pivots, which exist only once
+    # all of Z is scored: a second read of Z (and of the K_r pivot rows), the largest cosine per row
+    skr = sum(r.k1 - int(np.floor(np.float32(METHOD_RHO) * r.k1 + 0.5)) for r in w.reqs)
+    pivot_pass = sn * w.d * 2 + skr * w.d * 2 + sn * 4
+    return {"score_kernel": score, "stage1": stage1, "stage2": stage2, "step": stage1 + stage2,
+            "pivot_pass": pivot_pass, "method_step": stage1 + stage2 + pivot_pass}
 
 
 def peaks():
@@ -248,6 +254,19 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
             with torch.cuda.graph(g, stream=stream):
                 c(stream)
             graphs.append(g)
+        # the paper's Method settings on the same batch: Eq. 6-7 fused score for the K_r pivots
+        # and K_d = K1 / 4 diversity draws by farthest point sampling (Sec. 3.1)
+        mparams = T.default_params(T.SELECT_FUSED, diversity=METHOD_RHO)
+        mcalls = [T.PreparedCall(p, i, ws, mparams) for p, i in batches]
+        for c in mcalls:
+            c(stream)
+        method_launches = T.last_launch_count()
+        mgraphs = []
+        for c in mcalls:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                c(stream)
+            mgraphs.append(g)
     torch.cuda.synchronize()
 
     import torch.distributed as dist
@@ -288,6 +307,18 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
             T.trevs_pre_llm_varlen_timed(q, wsq, evs[i][0], evs[i][1], params, stream)
         torch.cuda.synchronize()
         kernel_ms = statistics.median(a.elapsed_time(b) for a, b in evs[8:])
+        # the Method settings, same protocol (graph replay over the rotating input sets)
+        msteps = max(10, min(args.steps, 4000))
+        for i in range(max(3, args.warmup // 10)):
+            mgraphs[i % ROTATING_SETS].replay()
+        torch.cuda.synchronize()
+        m0, m1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        m0.record(stream)
+        for i in range(msteps):
+            mgraphs[i % ROTATING_SETS].replay()
+        m1.record(stream)
+        torch.cuda.synchronize()
+        method_ms = m0.elapsed_time(m1) / msteps
 
     if distributed:
         elapsed_ms = max_over_ranks(elapsed_ms, dev)
@@ -351,6 +382,7 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
     if rank != 0:
         return None
     ms, value = replica_throughput(elapsed_ms, args.steps, w.visual_tokens(), world)
+    method_kd = int(np.floor(np.float32(METHOD_RHO) * WORKLOAD["k1"] + 0.5))
     nbytes = algorithmic_bytes(w)
     peak, src = peaks()
     achieved = nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9
@@ -375,6 +407,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         "gpu_launches": launches_per_step * args.steps,
         "launches_per_step": launches_per_step,
         "clocks": clk,
+        "method_path": {
+            "select": "fused (Eq. 6-7)", "diversity": METHOD_RHO, "K_r": WORKLOAD["k1"] - method_kd,
+            "K_d": method_kd, "us_per_prune": round(method_ms * 1e3, 2),
+            "value": w.visual_tokens() / (method_ms * 1e-3), "unit": UNIT, "steps": msteps,
+            "launches_per_step": method_launches, "algorithmic_bytes": nbytes["method_step"],
+            "frac": round(nbytes["method_step"] / (method_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
+            "timed": "CUDA events around graph replays of trevs_prune_varlen, 4 rotating input sets"},
     }
 
 
@@ -418,16 +457,18 @@ def reference_arm(args, w):
 
 
 def profile_run(w, stage="stage1", launches=5):
-    """Stage 1 (scoring + selection) or stage 2 of the bench batch, launched eagerly."""
+    """Stage 1 (scoring + selection; "method": with the fused score and the diversity draws)
+    or stage 2 of the bench batch, launched eagerly."""
     import torch
     from paper_2609_37581_gb300 import trevs as T
     from workloads.device import build_batches
     T.load()
     pre, inb = build_batches(w, T.SELECT_RATIO)
-    if stage == "stage1":
+    if stage in ("stage1", "method"):
         q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v, kept_idx=pre.kept_idx, s_t=pre.s_t)
         ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
-        params = T.default_params(T.SELECT_RATIO)
+        params = (T.default_params(T.SELECT_RATIO) if stage == "stage1"
+                  else T.default_params(T.SELECT_FUSED, diversity=METHOD_RHO))
         for _ in range(launches):
             T.trevs_pre_llm_varlen(q, ws, params)
     else:
@@ -445,8 +486,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--profile", nargs="?", const="stage1", choices=["stage1", "stage2"],
-                    help="only run stage 1 (or stage 2) of the bench batch a few times, for an ncu capture")
+    ap.add_argument("--profile", nargs="?", const="stage1", choices=["stage1", "stage2", "method"],
+                    help="only run stage 1 (stage 2, or stage 1 with the Method's diversity draws) of the "
+                         "bench batch a few times, for an ncu capture")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

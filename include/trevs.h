@@ -145,8 +145,8 @@ TREVS_API trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_str
                                   const int32_t* kept_idx, int32_t K1,
                                   uint16_t* Z_out, int64_t z_out_row_stride, void* stream);
 
-/* Workspace bytes for trevs_pre_llm_fps on one request of N tokens with K_r pivots. */
-TREVS_API size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r);
+/* Workspace bytes for trevs_pre_llm_fps on one request of N tokens of width d with K_r pivots. */
+TREVS_API size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r, int32_t d);
 
 /* Sec. 3.1 context preservation: S_d = FPS({z_i | i in C}, K_d), the K_d diversity tokens
  * drawn by farthest point sampling in cosine distance from the candidates C = [N] minus the

@@ -141,7 +141,7 @@ constexpr size_t kStatusBytes = 256;
 
 struct PreWs {
   size_t counters, sal, t_rinv, part, s_t, s_fused, keys, flags;
-  size_t fps_zero, fps_rinv, fps_maxcos, fps_ub, fps_stamp, fps_picks, end;
+  size_t fps_zero, fps_prow, fps_rinv, fps_maxcos, fps_ub, fps_stamp, fps_picks, end;
 };
 
 // Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request;
@@ -149,9 +149,10 @@ struct PreWs {
 // that two or more scoring CTAs share (up to max_m text rows, or up to the pivots of the
 // farthest-point contraction, min(max_k1, TREVS_MAX_TEXT_TOKENS), which reuses it). The
 // fps_* regions serve farthest point sampling (Sec. 3.1) when the call asks for it: a
-// 256-byte zero block, 1 / ||z|| of the pivots and the draws (indexed like kept_idx), and
-// the largest pivot cosine, bound and stamp of every row.
-PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1 = 0, int max_k1 = 0) {
+// 256-byte zero block, copies of the pivot rows (d columns), 1 / ||z|| of the pivots and the
+// draws (all indexed like kept_idx), and the largest pivot cosine, bound and stamp of every row.
+PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1 = 0, int max_k1 = 0,
+             int d = 0) {
   PreWs w;
   const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
   const int max_kr = max_k1 < TREVS_MAX_TEXT_TOKENS ? max_k1 : TREVS_MAX_TEXT_TOKENS;
@@ -167,6 +168,7 @@ PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1
   w.keys = o;     o = al256(o + 4 * padded);
   w.flags = o;    o = al256(o + padded);
   w.fps_zero = o;   o = al256(o + (k1 > 0 ? 256 : 0));
+  w.fps_prow = o;   o = al256(o + 2 * k1 * (size_t)(d > 0 ? d : 0));
   w.fps_rinv = o;   o = al256(o + 4 * k1);
   w.fps_picks = o;  o = al256(o + 4 * k1);
   w.fps_maxcos = o; o = al256(o + 4 * fn);
@@ -201,18 +203,20 @@ InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, i
 // (piv_space entries, indexed like the pivots), the partial sums of the pivot contraction
 // (up to max_kr pivots), the largest cosine of every row to its pivots, the bounds and
 // stamps of the draw, and flag / key scratch for the rows.
-// `zero` is 256 bytes that nothing writes: the row-0 pivot of a draw without pivots.
+// `zero` is 256 bytes that nothing writes: the row-0 pivot of a draw without pivots; `prow`
+// holds copies of the pivot rows (d columns each), which the contraction reads as text rows.
 struct FpsWs {
-  size_t zero, t_rinv, part, maxcos, ub, stamp, flags, keys, end;
+  size_t zero, prow, t_rinv, part, maxcos, ub, stamp, flags, keys, end;
 };
 
-FpsWs fps_ws(size_t o, long long total_n, long long piv_space, int max_kr) {
+FpsWs fps_ws(size_t o, long long total_n, long long piv_space, int max_kr, int d) {
   FpsWs w;
   const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
   if (piv_space < 1) piv_space = 1;
   if (max_kr < 1) max_kr = 1;
   o = al256(o);
   w.zero = o;    o = al256(o + 256);
+  w.prow = o;    o = al256(o + 2 * (size_t)piv_space * (size_t)(d > 0 ? d : 0));
   w.t_rinv = o;  o = al256(o + 4 * (size_t)(piv_space > 0 ? piv_space : 0));
   w.part = o;    o = al256(o + (total_n > 0 && max_kr > 0 ? pre_score_part_bytes(max_kr) : 0));
   w.maxcos = o;  o = al256(o + 4 * (size_t)total_n);
@@ -400,8 +404,24 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
       fm.r[fm.B++] = FpsReq{r.n_off, r.n, r.k1_off, kr, kd, lead, r.k1_off, r.k1_off};
     }
     dm.total_tiles = dtiles;
+    // copies of every request's kept slots (the pivots lead each request's K1 slots)
+    static thread_local GatherMeta pg;
+    uint16_t* prow = reinterpret_cast<uint16_t*>(ws + L.fps_prow);
+    pg.njobs = 1;
+    GatherTable& pt = pg.t[0];
+    pt.B = meta.B;
+    for (int i = 0; i < meta.B; ++i) {
+      pt.dst_off[i] = meta.r[i].k1_off; pt.src_off[i] = meta.r[i].n_off; pt.src_rows[i] = meta.r[i].n;
+    }
+    pt.dst_off[meta.B] = (int)ko;
+    GatherJob& pj = pg.job[0];
+    pj.src = reinterpret_cast<const uint8_t*>(a.Z); pj.dst = reinterpret_cast<uint8_t*>(prow);
+    pj.src_tok = a.z_stride * 2; pj.dst_tok = (long long)a.d * 2; pj.src_head = 0; pj.dst_head = 0;
+    pj.heads = 1; pj.row_bytes = a.d * 2; pj.idx = a.kept; pj.rows = (int)ko; pj.tab = 0;
+    TREVS_TRY_CUDA(counted(launch_gather(pg, ts, true)), "pivot rows launch");
     PreArgs da = a;
-    da.t_idx = a.kept;
+    da.T = reinterpret_cast<const __nv_bfloat16*>(prow);
+    da.t_stride = a.d;
     da.s_t = reinterpret_cast<float*>(ws + L.fps_maxcos);
     da.t_rinv = reinterpret_cast<float*>(ws + L.fps_rinv);
     da.total_m = ko;
@@ -780,9 +800,9 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   return TREVS_OK;
 }
 
-size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r) {
-  if (N < 0 || K_r < 0) return 0;
-  return fps_ws(kStatusBytes, N, K_r, K_r).end;
+size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r, int32_t d) {
+  if (N < 0 || K_r < 0 || d < 0) return 0;
+  return fps_ws(kStatusBytes, N, K_r, K_r, d).end;
 }
 
 trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
@@ -800,7 +820,7 @@ trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t 
   TREVS_CHECK(z_row_stride >= d && z_row_stride % 8 == 0, "z_row_stride must be >= d and a multiple of 8");
   TREVS_CHECK(K_r == 0 || pivots != nullptr, "pivots is NULL");
   TREVS_CHECK(picks != nullptr, "picks is NULL");
-  const FpsWs L = fps_ws(kStatusBytes, N, K_r, K_r);
+  const FpsWs L = fps_ws(kStatusBytes, N, K_r, K_r, d);
   trevs_status s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
@@ -810,7 +830,19 @@ trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t 
   const int lead = K_r == 0 ? 1 : 0;
   const int kr = K_r + lead;
   const int32_t* piv = lead ? reinterpret_cast<const int32_t*>(ws + L.zero) : pivots;
-  {   // the largest cosine of every row to the pivots: the scoring contraction
+  {   // the largest cosine of every row to the pivots: the scoring contraction over copies of
+      // the pivot rows (an index outside [0, N) leaves its zero-filled row in place)
+    uint16_t* prow = reinterpret_cast<uint16_t*>(ws + L.prow);
+    TREVS_TRY_CUDA(counted(cudaMemsetAsync(prow, 0, 2 * (size_t)kr * d, st)), "pivot rows clear");
+    static thread_local GatherMeta pg;
+    pg.njobs = 1;
+    pg.t[0].B = 1;
+    pg.t[0].dst_off[0] = 0; pg.t[0].dst_off[1] = kr; pg.t[0].src_off[0] = 0; pg.t[0].src_rows[0] = N;
+    GatherJob& j = pg.job[0];
+    j.src = reinterpret_cast<const uint8_t*>(Z); j.dst = reinterpret_cast<uint8_t*>(prow);
+    j.src_tok = z_row_stride * 2; j.dst_tok = (long long)d * 2; j.src_head = 0; j.dst_head = 0;
+    j.heads = 1; j.row_bytes = d * 2; j.idx = piv; j.rows = kr; j.tab = 0;
+    TREVS_TRY_CUDA(counted(launch_gather(pg, st, false)), "pivot rows launch");
     static thread_local PreMeta meta;
     meta.B = 1;
     meta.r[0] = PreReq{0, N, 0, kr, 0, 0, 0, 0};
@@ -818,7 +850,7 @@ trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t 
     PreArgs a;
     memset(&a, 0, sizeof(a));
     a.Z = reinterpret_cast<const __nv_bfloat16*>(Z); a.z_stride = z_row_stride;
-    a.t_idx = piv;
+    a.T = reinterpret_cast<const __nv_bfloat16*>(prow); a.t_stride = d;
     a.s_t = maxcos;
     a.t_rinv = reinterpret_cast<float*>(ws + L.t_rinv);
     a.total_m = kr;
@@ -1044,7 +1076,7 @@ size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
     if (r.n > 0 && r.m > max_m) max_m = r.m;
     if (r.k1 > max_k1) max_k1 = r.k1;
   }
-  return pre_ws(n, m, max_m, k1, max_k1).end;
+  return pre_ws(n, m, max_m, k1, max_k1, batch->d).end;
 }
 
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
@@ -1073,7 +1105,7 @@ trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_
   if (s != TREVS_OK || batch->B == 0) return s;
   s = validate_diversity(batch, prm);
   if (s != TREVS_OK) return s;
-  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -1094,7 +1126,7 @@ trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, const trev
   if (batch->B > kMaxChunk) return fail(TREVS_ERR_UNSUPPORTED, "B = %d > %d requests", batch->B, kMaxChunk);
   s = validate_diversity(batch, prm);
   if (s != TREVS_OK) return s;
-  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_chunk(batch, prm, 0, batch->B, 0, 0, 0, reinterpret_cast<uint8_t*>(workspace), L,
@@ -1127,7 +1159,7 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   s = validate_diversity(pre, prm);
   if (s != TREVS_OK) return s;
-  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1);
+  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1, pre->d);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
   const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);

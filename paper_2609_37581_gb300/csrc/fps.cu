@@ -7,9 +7,9 @@
 // block of 512 threads per request then draws the K_d tokens:
 //
 //   * The pool: the W candidates farthest from the pivots (W <= 128, about 2 K_d). Their
-//     pairwise cosines are one small contraction (mma.sync over 64-column chunks of the
-//     gathered rows, double-buffered with cp.async) kept in shared memory, so a step inside
-//     the pool costs an argmax over W and one row of the Gram matrix.
+//     pairwise cosines are one small contraction (mma.sync over 256-column chunks of the
+//     gathered rows, streamed through a ring of up to four chunks with cp.async) kept in
+//     shared memory, so a step inside the pool costs an argmax over W and one row of it.
 //   * Every candidate outside the pool keeps an upper bound of its distance (the distance to
 //     the pivots, lowered when refreshed) and the number of picks the bound accounts for.
 //     A distance only falls as picks are added, so the best pool candidate is the exact
@@ -26,10 +26,10 @@
 
 namespace trevs {
 
-constexpr int kFpsStageRow = 128;                            // bytes of a staged row: 64 bf16
-constexpr int kFpsStageBytes = kFpsMaxPool * kFpsStageRow;   // one buffer of staged rows
-constexpr int kFpsGramLd = kFpsMaxPool + 4;                  // fp32 row stride of the pool cosines
-constexpr int kFpsSmem = 2 * kFpsStageBytes + kFpsMaxPool * kFpsGramLd * 4 + 4 * kFpsMaxPool * 4;
+constexpr int kFpsSlices = 4;                 // 64-column slices per staged chunk (256 columns)
+constexpr int kFpsRingBytes = 128 * 1024;     // ring of staged chunks of the pool rows
+constexpr int kFpsGramLd = kFpsMaxPool + 4;   // fp32 row stride of the pool cosines
+constexpr int kFpsSmem = kFpsRingBytes + kFpsMaxPool * kFpsGramLd * 4 + 4 * kFpsMaxPool * 4;
 
 // (d_a, i_a) comes before (d_b, i_b): farther, or as far and a lower index.
 __device__ __forceinline__ bool fps_before(float da, int ia, float db, int ib) {
@@ -119,7 +119,7 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
   const int n = r.n, kd = r.kd, d = a.d;
   uint8_t* stage = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(fps_smem_raw) + 127) & ~uintptr_t(127));
-  float* gram = reinterpret_cast<float*>(stage + 2 * kFpsStageBytes);
+  float* gram = reinterpret_cast<float*>(stage + kFpsRingBytes);
   int* pool = reinterpret_cast<int*>(gram + kFpsMaxPool * kFpsGramLd);
   float* pdist = reinterpret_cast<float*>(pool + kFpsMaxPool);
   float* prinv = pdist + kFpsMaxPool;
@@ -194,17 +194,22 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
     ppick[p] = 0;
   }
 
-  // ---- cosines within the pool: G = Z_pool Z_pool^T (bf16 mma.sync, fp32), then normalised
-  {
+  // ---- cosines within the pool: G = Z_pool Z_pool^T (bf16 mma.sync, fp32), then normalised.
+  // The pool rows stream through a ring of S chunks of 256 columns (S = 2..4 as W allows),
+  // so that 64-96 KB are in flight while the block computes.
+  if (W > 0) {
     const int W16 = (W + 15) & ~15, nmt = W16 >> 4, nblk = nmt * nmt;
-    const int nch = (d + 63) >> 6;
+    const int slice_bytes = W16 * 128, chunk_bytes = kFpsSlices * slice_bytes;
+    const int S = min(4, kFpsRingBytes / chunk_bytes);
+    const int nch = (d + 64 * kFpsSlices - 1) / (64 * kFpsSlices);
     const uint32_t sbase = smem_u32(stage);
-    auto load_chunk = [&](int ch, int buf) {
-      for (int idx = tid; idx < W16 * 8; idx += nthr) {
-        const int row = idx >> 3, c = idx & 7, col = ch * 64 + c * 8;
+    auto load_chunk = [&](int ch, int slot) {
+      for (int idx = tid; idx < W16 * 8 * kFpsSlices; idx += nthr) {
+        const int row = idx >> 5, q = idx & 31, sl = q >> 3, c = q & 7;
+        const int col = ch * 64 * kFpsSlices + q * 8;
         const bool ok = row < W && col < d;
         const void* src = ok ? (const void*)(Zb + (long long)pool[row] * a.z_stride + col) : (const void*)a.Z;
-        cp_async16(sbase + buf * kFpsStageBytes + row * kFpsStageRow + (swz(row, c) << 4), src, ok ? 16 : 0);
+        cp_async16(sbase + slot * chunk_bytes + sl * slice_bytes + row * 128 + (swz(row, c) << 4), src, ok ? 16 : 0);
       }
     };
     float acc[4][2][4];
@@ -215,34 +220,42 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
 #pragma unroll
         for (int y = 0; y < 4; ++y) acc[j][x][y] = 0.f;
     __syncthreads();   // pool[] is read by every thread's copies
-    load_chunk(0, 0);
-    cp_async_commit();
-    for (int ch = 0; ch < nch; ++ch) {
-      if (ch + 1 < nch) load_chunk(ch + 1, (ch + 1) & 1);
+    for (int c = 0; c < S - 1; ++c) {
+      if (c < nch) load_chunk(c, c);
       cp_async_commit();
-      cp_async_wait<1>();
-      __syncthreads();
-      const uint32_t B0 = sbase + (ch & 1) * kFpsStageBytes;
+    }
+    for (int ch = 0; ch < nch; ++ch) {
+      // chunk ch is the oldest of the S - 1 groups in flight
+      if (S == 4) cp_async_wait<2>();
+      else if (S == 3) cp_async_wait<1>();
+      else cp_async_wait<0>();
+      __syncthreads();   // chunk ch is visible to all; slot (ch - 1) % S is free again
+      if (ch + S - 1 < nch) load_chunk(ch + S - 1, (ch + S - 1) % S);
+      cp_async_commit();
+      const uint32_t B0 = sbase + (ch % S) * chunk_bytes;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int bi = warp + 16 * j;   // 16 x 16 output block (mt, pr)
         if (bi < nblk) {
           const int mt = bi / nmt, pr = bi - mt * nmt;
 #pragma unroll
-          for (int ks = 0; ks < 4; ++ks) {
-            uint32_t af[4];
-            const int ar = mt * 16 + (lane & 15), ac = 2 * ks + (lane >> 4);
-            ldmatrix_x4(B0 + ar * kFpsStageRow + (swz(ar, ac) << 4), af[0], af[1], af[2], af[3]);
-            const int mi = lane >> 3;
-            const int br = pr * 16 + 8 * (mi >> 1) + (lane & 7), bc = 2 * ks + (mi & 1);
-            uint32_t b0, b1, b2, b3;
-            ldmatrix_x4(B0 + br * kFpsStageRow + (swz(br, bc) << 4), b0, b1, b2, b3);
-            mma_bf16_16816(acc[j][0], af, b0, b1);
-            mma_bf16_16816(acc[j][1], af, b2, b3);
+          for (int sl = 0; sl < kFpsSlices; ++sl) {
+            const uint32_t Bs = B0 + sl * slice_bytes;
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+              uint32_t af[4];
+              const int ar = mt * 16 + (lane & 15), ac = 2 * ks + (lane >> 4);
+              ldmatrix_x4(Bs + ar * 128 + (swz(ar, ac) << 4), af[0], af[1], af[2], af[3]);
+              const int mi = lane >> 3;
+              const int br = pr * 16 + 8 * (mi >> 1) + (lane & 7), bc = 2 * ks + (mi & 1);
+              uint32_t b0, b1, b2, b3;
+              ldmatrix_x4(Bs + br * 128 + (swz(br, bc) << 4), b0, b1, b2, b3);
+              mma_bf16_16816(acc[j][0], af, b0, b1);
+              mma_bf16_16816(acc[j][1], af, b2, b3);
+            }
           }
         }
       }
-      __syncthreads();   // the buffer is refilled two chunks later
     }
     cp_async_wait<0>();
     const int g = lane >> 2, t4 = lane & 3;
@@ -271,8 +284,8 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
       const int p = x / W, q = x - p * W;
       gram[p * kFpsGramLd + q] = gram[p * kFpsGramLd + q] * prinv[p] * prinv[q];
     }
-    __syncthreads();
   }
+  __syncthreads();
 
   fps_outside_best(ub, stamp, n, s_wi, s_wd, &s_o, &s_od);
 

@@ -89,8 +89,8 @@ __device__ __forceinline__ void for_each_subtile(const PreMeta& meta, int nzs, l
   }
 }
 
-// kSeed: the pivot rows of Z stand in for the text rows (t_idx) and each row's output is the
-// largest cosine to them, unrectified (the distances of farthest point sampling, Sec. 3.1).
+// kSeed: the "text" rows are the pivot rows of Z (gathered beforehand) and each row's output
+// is the largest cosine to them, unrectified (the distances of farthest point sampling, Sec. 3.1).
 template <bool kSeed>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     pre_score_kernel(const __grid_constant__ CUtensorMap tmZ3, const __grid_constant__ CUtensorMap tmZ2,
@@ -238,7 +238,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
       const PreReq& r = meta.r[st.b];
       const int pieces = r.m * 8;
-      const uint8_t* tsrc = kSeed ? nullptr : reinterpret_cast<const uint8_t*>(a.T + (long long)r.m_off * a.t_stride);
+      const uint8_t* tsrc = reinterpret_cast<const uint8_t*>(a.T + (long long)r.m_off * a.t_stride);
       for (int zs = st.zs0; zs < st.zs1; ++zs) {
         const int ns = min(kZSlices, nk - zs * kZSlices);
         for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
@@ -255,15 +255,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             for (int p = ct; p < pieces; p += kTCopyThreads) {
               const int row = p >> 3, q = p & 7;
               const int col = kc * kChunk + q * 8;
-              if constexpr (kSeed) {
-                const int zi = __ldg(a.t_idx + r.m_off + row);
-                const bool ok = col < d && zi >= 0 && zi < r.n;
-                const __nv_bfloat16* src = ok ? a.Z + ((long long)r.n_off + zi) * a.z_stride + col : a.Z;
-                cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, ok ? 16 : 0);
-              } else {
-                const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
-                cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, col < d ? 16 : 0);   // zero past d'
-              }
+              const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
+              cp_async16(Bc + row * 128 + (swz(row, q) << 4), src, col < d ? 16 : 0);   // zero past d'
             }
           }
           cp_async_arrive_noinc(smem_u32(&tfull[ts]));
@@ -542,20 +535,7 @@ __global__ void __launch_bounds__(512) pre_saliency_kernel(const __grid_constant
     const long long row = (long long)(blockIdx.x - n_sal) * 16 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (row >= a.total_m) return;
-    const uint4* t;
-    if (a.t_idx) {   // the pivot rows of Z (farthest point sampling): request b owns [m_off, m_off + m)
-      const int b = find_request(meta.B, (int)row, [&](int i) { return meta.r[i].m_off; });
-      const PreReq& r = meta.r[b];
-      if ((int)row - r.m_off >= r.m) return;
-      const int zi = __ldg(a.t_idx + row);
-      if (zi < 0 || zi >= r.n) {
-        if (lane == 0) a.t_rinv[row] = 0.f;
-        return;
-      }
-      t = reinterpret_cast<const uint4*>(a.Z + ((long long)r.n_off + zi) * a.z_stride);
-    } else {
-      t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
-    }
+    const uint4* t = reinterpret_cast<const uint4*>(a.T + row * a.t_stride);
     const int nv = a.d / 8;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int p0 = 0; p0 < nv; p0 += 16 * 32) {
@@ -720,7 +700,7 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   if (e != cudaSuccess) return e;
   e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, kZBoxRows);
   if (e != cudaSuccess) return e;
-  auto kernel = a.t_idx ? pre_score_kernel<true> : pre_score_kernel<false>;
+  auto kernel = a.action == kActFpsSeed ? pre_score_kernel<true> : pre_score_kernel<false>;
   e = ensure_dynamic_smem(kernel, smem);
   if (e != cudaSuccess) return e;
   return launch_kernel(kernel, dim3(score_grid(meta, a.d, a.score_reserve)), dim3(kScoreThreads), smem, st, pdl, tmZ3,

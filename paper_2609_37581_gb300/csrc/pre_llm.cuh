@@ -12,15 +12,13 @@ constexpr int kScoreTileRows = 128;   // visual rows per scoring tile (UMMA M)
 constexpr int kMaxScoreCtas = 256;    // CTAs of the persistent scoring grid, at most
 enum { kActScores = 0, kActScoresFused = 1, kActSelect = 2, kActFpsSeed = 3 };
 // kActFpsSeed: the scoring contraction for farthest point sampling (Sec. 3.1). The "text"
-// rows are the pivot rows of Z (t_idx), and s_t receives max_j cos(z_i, z_pivot_j).
+// rows are copies of the pivot rows of Z, and s_t receives max_j cos(z_i, z_pivot_j).
 
 struct PreArgs {
   const __nv_bfloat16* Z;
   long long z_stride;
   const __nv_bfloat16* T;
   long long t_stride;
-  const int* t_idx;    // kActFpsSeed: text row j of request b is Z row t_idx[m_off + j] of b
-                       // (request-local; outside [0, n) reads as a zero row)
   const float* s_v;
   float* s_t;          // [sum n]
   float* s_fused;      // [sum n] (fused mode)

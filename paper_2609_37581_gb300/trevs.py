@@ -80,7 +80,7 @@ _SIGS = {
     "trevs_pre_llm_select": (_c_i32, [_vp, _vp, _vp, _c_i32, _c_i32, _c_f32, ctypes.POINTER(PreParams),
                                       _vp, _vp, _c_sz, _vp]),
     "trevs_pre_llm_gather": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _vp, _c_i64, _vp]),
-    "trevs_pre_llm_fps_workspace_size": (_c_sz, [_c_i32, _c_i32]),
+    "trevs_pre_llm_fps_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
     "trevs_pre_llm_fps": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _c_i32, _c_i32, _vp, _vp,
                                    _vp, _c_sz, _vp]),
     "trevs_in_llm_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
@@ -206,8 +206,8 @@ def trevs_pre_llm_gather(Z, kept_idx, Z_out, stream=None):
                                       _ptr(Z_out), Z_out.stride(0), _stream(stream)))
 
 
-def trevs_pre_llm_fps_workspace_size(N, K_r):
-    return int(load().trevs_pre_llm_fps_workspace_size(N, K_r))
+def trevs_pre_llm_fps_workspace_size(N, K_r, d):
+    return int(load().trevs_pre_llm_fps_workspace_size(N, K_r, d))
 
 
 def trevs_pre_llm_fps(Z, pivots, K_d, picks, pick_dist=None, pool=0, ws=None, stream=None):

@@ -87,10 +87,10 @@ def test_scores_validation(lib):
 
 
 def test_fps_validation(lib):
-    need = lib.trevs_pre_llm_fps_workspace_size(576, 48)
+    need = lib.trevs_pre_llm_fps_workspace_size(576, 48, 4096)
     assert need > 0 and need % 256 == 0
-    assert lib.trevs_pre_llm_fps_workspace_size(576, 48) > lib.trevs_pre_llm_fps_workspace_size(100, 48)
-    assert lib.trevs_pre_llm_fps_workspace_size(-1, 0) == 0
+    assert lib.trevs_pre_llm_fps_workspace_size(576, 48, 4096) > lib.trevs_pre_llm_fps_workspace_size(100, 48, 4096)
+    assert lib.trevs_pre_llm_fps_workspace_size(-1, 0, 4096) == 0
 
     def fps(N=576, d=4096, K_r=48, K_d=16, pool=0, zs=4096, Z=FAKE, piv=FAKE, picks=FAKE, ws=FAKE, nb=need):
         return lib.trevs_pre_llm_fps(Z, zs, N, d, piv, K_r, K_d, pool, picks, None, ws, nb, None)

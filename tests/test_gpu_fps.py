@@ -68,7 +68,7 @@ def run_fps(Z_bits, pivots, k_d, pool=0):
     piv = torch.tensor(np.asarray(pivots, np.int32), device="cuda") if len(pivots) else None
     picks = torch.full((max(k_d, 1),), -7, dtype=torch.int32, device="cuda")
     dist = torch.full((max(k_d, 1),), -7.0, dtype=torch.float32, device="cuda")
-    ws = T.workspace(T.trevs_pre_llm_fps_workspace_size(N, len(pivots)))
+    ws = T.workspace(T.trevs_pre_llm_fps_workspace_size(N, len(pivots), d))
     T.trevs_pre_llm_fps(Z, piv, k_d, picks, dist, pool=pool, ws=ws)
     T.workspace_status(ws)
     return picks.cpu().numpy()[:k_d], dist.cpu().numpy()[:k_d]
