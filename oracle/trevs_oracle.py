@@ -32,6 +32,9 @@ Readings where the paper is silent or leaves a choice open:
     distance +inf, so the first pick is the lowest index of C.
   * K_d = floor(rho*K1 + 0.5) for a diversity share rho (the paper's K_r:K_d = 3:1 is
     rho = 0.25); the pivots are the top K_r = K1 - K_d of the stage-1 rule.
+  * [CLS] saliency (Eq. 2-3): the softmax of each head runs over the N patch keys, as Eq. 2
+    writes it (K_v holds the patch keys only), with scale 1/sqrt(d_h); s^v is the plain mean
+    of the H heads' distributions.
 
 Parity pins: every function here is pinned by tests/test_oracle_pins.py against
 closed forms, hand-derived worked examples (tests/golden/), brute force on tiny
@@ -53,6 +56,25 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
 
 
 # ---------------------------------------------------------------- stage 1 (Sec. 4.1)
+
+
+def cls_saliency(q_cls: np.ndarray, K_v: np.ndarray, scale: float | None = None) -> np.ndarray:
+    """Eq. 2-3: s^v_i = (1/H) sum_h Softmax_i( q^h_[CLS] . k^h_i / sqrt(d_h) ).
+
+    q_cls is [H, d_h] (the [CLS] query of every head), K_v is [N, H, d_h] (the patch keys of
+    the penultimate ViT layer). Returns s^v, [N], a distribution over the patches.
+    """
+    q = np.asarray(q_cls, dtype=np.float64)
+    K = np.asarray(K_v, dtype=np.float64)
+    N, H, dh = K.shape
+    if scale is None:
+        scale = 1.0 / math.sqrt(dh)
+    A = np.empty((H, N), dtype=np.float64)
+    for h in range(H):
+        logits = (K[:, h, :] @ q[h]) * scale                  # Eq. 2, before the softmax
+        e = np.exp(logits - logits.max())
+        A[h] = e / e.sum()
+    return A.sum(axis=0) / H                                  # Eq. 3
 
 
 def rectified_cosine(Z: np.ndarray, T: np.ndarray) -> np.ndarray:

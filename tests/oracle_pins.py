@@ -18,7 +18,7 @@ import numpy as np
 import oracle.trevs_oracle as O
 
 GOLDEN = pathlib.Path(__file__).parent / "golden"
-_ENV = {"__builtins__": {}, "sqrt": math.sqrt, "ln2": math.log(2.0)}
+_ENV = {"__builtins__": {}, "sqrt": math.sqrt, "ln2": math.log(2.0), "ln3": math.log(3.0)}
 
 
 def _val(expr) -> float:
@@ -425,6 +425,52 @@ def pin_diversity_share():
         assert list(r["kept"]) == sorted(list(base["kept"]) + list(r["fps"]))
         assert list(O.pre_llm_request(Zb, Tb, sv, K1, 0.5, mode, diversity=0.0)["kept"]) == \
             list(O.pre_llm_request(Zb, Tb, sv, K1, 0.5, mode)["kept"])
+
+
+
+# ------------------------------------------------------------- Eq. 2-3, [CLS] saliency
+
+
+def pin_cls_saliency_worked_example():
+    g = _golden("cls_saliency_3x2.json")
+    q = _vals(g["q_cls"])
+    K = _vals(g["K_v"])
+    _close(O.cls_saliency(q, K), _vals(g["s_v"]), 1e-12)
+
+
+def pin_cls_saliency_single_head_is_softmax():
+    from scipy.special import softmax
+    rng = np.random.default_rng(37)
+    for N, dh in ((1, 8), (5, 64), (300, 128)):
+        q = rng.standard_normal((1, dh))
+        K = 3.0 * rng.standard_normal((N, 1, dh))
+        _close(O.cls_saliency(q, K), softmax(K[:, 0, :] @ q[0] / math.sqrt(dh)), 1e-12)
+
+
+def pin_cls_saliency_closed_forms():
+    rng = np.random.default_rng(41)
+    N, H, dh = 9, 4, 16
+    K = rng.standard_normal((N, H, dh))
+    _close(O.cls_saliency(np.zeros((H, dh)), K), np.full(N, 1.0 / N))            # q = 0: uniform
+    _close(O.cls_saliency(rng.standard_normal((H, dh)), np.repeat(K[:1], N, 0)), np.full(N, 1.0 / N))
+    # one key along q: logit x, the others 0 -> e^x / (e^x + N - 1)
+    q = np.zeros((1, 4)); q[0, 0] = 2.0
+    Kx = np.zeros((N, 1, 4)); Kx[5, 0, 0] = 1.5              # logit 2 * 1.5 / sqrt(4) = 1.5
+    want = np.full(N, 1.0 / (math.exp(1.5) + N - 1)); want[5] = math.exp(1.5) / (math.exp(1.5) + N - 1)
+    _close(O.cls_saliency(q, Kx), want)
+
+
+def pin_cls_saliency_invariants():
+    rng = np.random.default_rng(43)
+    N, H, dh = 50, 6, 32
+    q = rng.standard_normal((H, dh))
+    K = 2.0 * rng.standard_normal((N, H, dh))
+    s = O.cls_saliency(q, K)
+    assert abs(s.sum() - 1.0) < 1e-12 and np.all(s > 0)
+    perm = rng.permutation(H)
+    _close(O.cls_saliency(q[perm], K[:, perm]), s)                           # head order
+    _close(O.cls_saliency(q * 4.0, K / 4.0), s)                              # q.k unchanged
+    _close(O.cls_saliency(q, K + rng.standard_normal((1, H, dh))), s, 1e-10)  # one shift per head
 
 
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

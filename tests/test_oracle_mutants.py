@@ -234,6 +234,37 @@ def _diversity_floor(k1, rho):
     return int(np.floor(np.float32(rho) * k1))
 
 
+
+def _cls_generic(q_cls, K_v, scale=None, *, scaled=True, reduce="mean", axis="tokens"):
+    q = np.asarray(q_cls, dtype=np.float64)
+    K = np.asarray(K_v, dtype=np.float64)
+    N, H, dh = K.shape
+    L = np.einsum("nhd,hd->hn", K, q) * (1.0 / np.sqrt(dh) if scaled else 1.0)
+    if axis == "tokens":
+        e = np.exp(L - L.max(axis=1, keepdims=True))
+        A = e / e.sum(axis=1, keepdims=True)
+    else:
+        e = np.exp(L - L.max(axis=0, keepdims=True))
+        A = e / e.sum(axis=0, keepdims=True)
+    return A.sum(0) / H if reduce == "mean" else (A.sum(0) if reduce == "sum" else A.max(0))
+
+
+def _cls_no_scale(q, K, scale=None):
+    return _cls_generic(q, K, scaled=False)
+
+
+def _cls_sum_heads(q, K, scale=None):
+    return _cls_generic(q, K, reduce="sum")
+
+
+def _cls_max_heads(q, K, scale=None):
+    return _cls_generic(q, K, reduce="max")
+
+
+def _cls_softmax_over_heads(q, K, scale=None):
+    return _cls_generic(q, K, axis="heads")
+
+
 MUTANTS = {
     "cos_no_relu": ("rectified_cosine", _no_relu),
     "cos_wrong_norm": ("rectified_cosine", _wrong_norm),
@@ -271,6 +302,10 @@ MUTANTS = {
     "fps_nearest": ("farthest_point_sampling", _fps_nearest),
     "fps_unnormalised": ("farthest_point_sampling", _fps_unnormalised),
     "diversity_floor": ("diversity_count", _diversity_floor),
+    "cls_no_scale": ("cls_saliency", _cls_no_scale),
+    "cls_sum_heads": ("cls_saliency", _cls_sum_heads),
+    "cls_max_heads": ("cls_saliency", _cls_max_heads),
+    "cls_softmax_over_heads": ("cls_saliency", _cls_softmax_over_heads),
 }
 
 
