@@ -46,6 +46,7 @@ WORKLOAD = dict(k1=64, ratio=0.5, k2=32)
 ROTATING_SETS = 4
 DOMINANT = "pre_score_kernel"
 METHOD_RHO = 0.25   # K_r:K_d = 3:1, the paper's setting for the diversity draws (Sec. 3.1)
+CLS_HEADS, CLS_DH = 16, 64   # the [CLS] attention of CLIP ViT-L/14 (Eq. 2-3)
 
 
 def workload():
@@ -319,6 +320,29 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         m1.record(stream)
         torch.cuda.synchronize()
         method_ms = m0.elapsed_time(m1) / msteps
+        # [CLS] saliency (Eq. 2-3) for the same requests: CLIP ViT-L/14 keys, 16 heads of 64,
+        # 4 rotating input sets (151 MB > L2); the calls are queued behind a spin kernel so
+        # that none waits on the host
+        cn = [r.n for r in w.reqs]
+        csets = []
+        for k in range(ROTATING_SETS):
+            qb, kb = synth.cls_inputs(cn, CLS_HEADS, CLS_DH, seed=500 + k)
+            csets.append((dev_bf16(qb), dev_bf16(kb)))
+        cs_v = torch.zeros(sum(cn), dtype=torch.float32, device=dev)
+        cws = T.workspace(T.trevs_cls_saliency_workspace_size(cn, CLS_HEADS))
+        for k in range(8):
+            T.trevs_cls_saliency_varlen(*csets[k % ROTATING_SETS], cn, cs_v, ws=cws, stream=stream)
+        torch.cuda.synchronize()
+        csteps = 200
+        torch.cuda._sleep(int(2e9 * 3e-5 * csteps))   # about 30 us of host time per queued call
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record(stream)
+        for k in range(csteps):
+            T.trevs_cls_saliency_varlen(*csets[k % ROTATING_SETS], cn, cs_v, ws=cws, stream=stream)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        cls_ms = c0.elapsed_time(c1) / csteps
+        cls_bytes = sum(x.numel() * x.element_size() for x in csets[0]) + cs_v.numel() * 4
 
     if distributed:
         elapsed_ms = max_over_ranks(elapsed_ms, dev)
@@ -414,6 +438,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
             "launches_per_step": method_launches, "algorithmic_bytes": nbytes["method_step"],
             "frac": round(nbytes["method_step"] / (method_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
             "timed": "CUDA events around graph replays of trevs_prune_varlen, 4 rotating input sets"},
+        "cls_saliency": {
+            "config": f"{w.B} x 576 patches, {CLS_HEADS} heads x {CLS_DH} (CLIP ViT-L/14 penultimate layer)",
+            "us_per_call": round(cls_ms * 1e3, 2), "algorithmic_bytes": cls_bytes,
+            "achieved_gbs": round(cls_bytes / (cls_ms * 1e-3) / 1e9, 1),
+            "frac": round(cls_bytes / (cls_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
+            "timed": "CUDA events around 200 trevs_cls_saliency_varlen calls queued behind a spin kernel, "
+                     "4 rotating input sets"},
     }
 
 

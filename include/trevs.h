@@ -117,6 +117,21 @@ TREVS_API trevs_status trevs_workspace_init(void* workspace, size_t bytes, void*
  * s_v [N] float32                                [CLS] saliency s^v_i          (Eq. 3)
  */
 
+/* Eq. 2-3, the vision encoder's [CLS] saliency for a batch of B requests:
+ *   s_v[i] = (1/H) sum_h Softmax_i(q_h . k_{i,h} * scale) over the n[b] patch keys of request b,
+ * scale = `scale` if > 0, else 1/sqrt(d_h). q_cls holds the [CLS] query of every head, element
+ * (b, h, c) at q_cls + b*q_req_stride + h*q_head_stride + c; K_v the patch keys of the
+ * penultimate ViT layer, packed over the requests, element (i, h, c) at
+ * K_v + i*k_tok_stride + h*k_head_stride + c; s_v [sum n] float32 receives the saliency,
+ * ready for the stage-1 calls. n is a host array [B]. Limits: d_h in {32, 64, 128},
+ * H <= TREVS_MAX_HEADS, n[b] <= 16384. The softmax spans the patch keys only, as Eq. 2
+ * writes it. */
+TREVS_API size_t trevs_cls_saliency_workspace_size(int32_t B, const int32_t* n, int32_t H);
+TREVS_API trevs_status trevs_cls_saliency_varlen(const uint16_t* q_cls, int64_t q_req_stride, int64_t q_head_stride,
+                                       const uint16_t* K_v, int64_t k_tok_stride, int64_t k_head_stride,
+                                       int32_t B, const int32_t* n, int32_t H, int32_t d_h, float scale,
+                                       float* s_v, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Workspace bytes for trevs_pre_llm_scores / trevs_pre_llm_select on one request of N tokens. */
 TREVS_API size_t trevs_pre_llm_workspace_size(int32_t N);
 

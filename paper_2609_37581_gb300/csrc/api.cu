@@ -7,6 +7,7 @@
 #include <mutex>
 #include <vector>
 
+#include "cls.cuh"
 #include "fps.cuh"
 #include "in_llm.cuh"
 #include "pre_llm.cuh"
@@ -20,6 +21,7 @@ cudaError_t launch_pre_finish(const PreMeta&, const PreArgs&, int max_m, int max
 cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
+cudaError_t launch_cls_saliency(const ClsMeta&, const ClsArgs&, int dh, int max_n, cudaStream_t);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 bool in_small_fits(int Hq, int max_l, int max_k1);
@@ -224,6 +226,20 @@ FpsWs fps_ws(size_t o, long long total_n, long long piv_space, int max_kr, int d
   w.stamp = o;   o = al256(o + 4 * (size_t)total_n);
   w.flags = o;   o = al256(o + padded);
   w.keys = o;    o = al256(o + 4 * padded);
+  w.end = o;
+  return w;
+}
+
+// [CLS] saliency (Eq. 2-3): per-request tickets, then the H softmax rows of every patch.
+struct ClsWs {
+  size_t cnt, attn, end;
+};
+
+ClsWs cls_ws(long long total_n, int H) {
+  ClsWs w;
+  size_t o = kStatusBytes;
+  w.cnt = o;  o = al256(o + 4 * (size_t)kMaxChunk);
+  w.attn = o; o = al256(o + 4 * (size_t)(H > 0 ? H : 0) * (size_t)(total_n > 0 ? total_n : 0));
   w.end = o;
   return w;
 }
@@ -797,6 +813,74 @@ trevs_status trevs_pre_llm_scores(const uint16_t* Z, int64_t z_row_stride, int32
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, (cudaStream_t)stream)), "pre-pass launch");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, M, N, (cudaStream_t)stream, true)), "pre_score launch");
   TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, M, N, true, (cudaStream_t)stream, true)), "finishing launch");
+  return TREVS_OK;
+}
+
+size_t trevs_cls_saliency_workspace_size(int32_t B, const int32_t* n, int32_t H) {
+  if (B <= 0 || !n || H <= 0) return 0;
+  long long total = 0;
+  for (int b = 0; b < B; ++b) total += n[b] > 0 ? n[b] : 0;
+  return cls_ws(total, H).end;
+}
+
+trevs_status trevs_cls_saliency_varlen(const uint16_t* q_cls, int64_t q_req_stride, int64_t q_head_stride,
+                                       const uint16_t* K_v, int64_t k_tok_stride, int64_t k_head_stride,
+                                       int32_t B, const int32_t* n, int32_t H, int32_t d_h, float scale,
+                                       float* s_v, void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  TREVS_CHECK(B >= 0, "B = %d < 0", B);
+  if (B == 0) return TREVS_OK;
+  TREVS_CHECK(n != nullptr, "n is NULL");
+  TREVS_CHECK(H >= 1, "H = %d < 1", H);
+  if (H > TREVS_MAX_HEADS) return fail(TREVS_ERR_UNSUPPORTED, "H = %d > %d", H, TREVS_MAX_HEADS);
+  if (!cls_head_dim_supported(d_h)) return fail(TREVS_ERR_UNSUPPORTED, "d_h = %d: 32, 64 or 128 supported", d_h);
+  long long total = 0;
+  int max_n = 0;
+  for (int b = 0; b < B; ++b) {
+    TREVS_CHECK(n[b] >= 0, "request %d: n = %d < 0", b, n[b]);
+    if (n[b] > kClsMaxN) return fail(TREVS_ERR_UNSUPPORTED, "request %d: n = %d > %d patches", b, n[b], kClsMaxN);
+    total += n[b];
+    max_n = n[b] > max_n ? n[b] : max_n;
+  }
+  TREVS_CHECK(total < (1ll << 31), "batch too large for int32 offsets");
+  if (total == 0) return TREVS_OK;
+  TREVS_CHECK(q_cls && K_v && s_v, "q_cls, K_v and s_v must be non-NULL");
+  TREVS_CHECK(aligned16(q_cls) && aligned16(K_v), "q_cls and K_v must be 16-byte aligned");
+  TREVS_CHECK(q_req_stride >= 0 && q_head_stride >= 0 && k_tok_stride >= 0 && k_head_stride >= 0 &&
+                  q_req_stride % 8 == 0 && q_head_stride % 8 == 0 && k_tok_stride % 8 == 0 && k_head_stride % 8 == 0,
+              "strides must be non-negative multiples of 8");
+  TREVS_CHECK(std::isfinite(scale), "scale must be finite");
+  const ClsWs L = cls_ws(total, H);
+  trevs_status s = check_ws(workspace, workspace_bytes, L.end);
+  if (s != TREVS_OK) return s;
+  uint8_t* ws = reinterpret_cast<uint8_t*>(workspace);
+  static thread_local ClsMeta meta;
+  long long n_base = 0;
+  for (int b0 = 0; b0 < B; b0 += kMaxChunk) {
+    const int b1 = b0 + kMaxChunk < B ? b0 + kMaxChunk : B;
+    meta.B = 0;
+    meta.H = H;
+    long long no = 0;
+    int chunk_max = 0;
+    for (int b = b0; b < b1; ++b) {
+      if (n[b] > 0) meta.r[meta.B++] = ClsReq{(int)no, n[b], b - b0};
+      no += n[b];
+      chunk_max = n[b] > chunk_max ? n[b] : chunk_max;
+    }
+    ClsArgs a;
+    a.q = reinterpret_cast<const __nv_bfloat16*>(q_cls) + (long long)b0 * q_req_stride;
+    a.q_req = q_req_stride; a.q_head = q_head_stride;
+    a.K = reinterpret_cast<const __nv_bfloat16*>(K_v) + n_base * k_tok_stride;
+    a.k_tok = k_tok_stride; a.k_head = k_head_stride;
+    a.scale = scale > 0.f ? scale : 1.0f / std::sqrt((float)d_h);
+    a.attn = reinterpret_cast<float*>(ws + L.attn);
+    a.attn_ld = no;
+    a.s_v = s_v + n_base;
+    a.cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
+    TREVS_TRY_CUDA(counted(launch_cls_saliency(meta, a, d_h, chunk_max, (cudaStream_t)stream)), "saliency launch");
+    n_base += no;
+  }
+  (void)max_n;
   return TREVS_OK;
 }
 

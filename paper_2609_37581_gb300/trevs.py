@@ -80,6 +80,9 @@ _SIGS = {
     "trevs_pre_llm_select": (_c_i32, [_vp, _vp, _vp, _c_i32, _c_i32, _c_f32, ctypes.POINTER(PreParams),
                                       _vp, _vp, _c_sz, _vp]),
     "trevs_pre_llm_gather": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _vp, _c_i64, _vp]),
+    "trevs_cls_saliency_workspace_size": (_c_sz, [_c_i32, ctypes.POINTER(_c_i32), _c_i32]),
+    "trevs_cls_saliency_varlen": (_c_i32, [_vp, _c_i64, _c_i64, _vp, _c_i64, _c_i64, _c_i32,
+                                           ctypes.POINTER(_c_i32), _c_i32, _c_i32, _c_f32, _vp, _vp, _c_sz, _vp]),
     "trevs_pre_llm_fps_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
     "trevs_pre_llm_fps": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i32, _c_i32, _c_i32, _vp, _vp,
                                    _vp, _c_sz, _vp]),
@@ -204,6 +207,27 @@ def trevs_pre_llm_gather(Z, kept_idx, Z_out, stream=None):
     N, d = Z.shape
     check(load().trevs_pre_llm_gather(_ptr(Z), Z.stride(0), N, d, _ptr(kept_idx), kept_idx.numel(),
                                       _ptr(Z_out), Z_out.stride(0), _stream(stream)))
+
+
+def _i32_array(xs):
+    xs = [int(x) for x in xs]
+    return (_c_i32 * max(len(xs), 1))(*xs)
+
+
+def trevs_cls_saliency_workspace_size(n, H):
+    arr = _i32_array(n)
+    return int(load().trevs_cls_saliency_workspace_size(len(n), arr, H))
+
+
+def trevs_cls_saliency_varlen(q_cls, K_v, n, s_v, scale=0.0, ws=None, stream=None):
+    """Eq. 2-3 for a batch: q_cls [B, H, d_h] and K_v [sum n, H, d_h] (bf16, any strides with
+    a unit innermost stride), n the patch count of each request; writes s_v [sum n]."""
+    B, H, dh = q_cls.shape
+    arr = _i32_array(n)
+    w, nb = _ws_args(ws)
+    check(load().trevs_cls_saliency_varlen(_ptr(q_cls), q_cls.stride(0), q_cls.stride(1), _ptr(K_v),
+                                           K_v.stride(0), K_v.stride(1), B, arr, H, dh, scale, _ptr(s_v),
+                                           w, nb, _stream(stream)))
 
 
 def trevs_pre_llm_fps_workspace_size(N, K_r, d):

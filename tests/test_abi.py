@@ -112,6 +112,32 @@ def test_fps_validation(lib):
     assert t.last_launch_count() == 0
 
 
+def test_cls_saliency_validation(lib):
+    arr = lambda xs: (ctypes.c_int32 * len(xs))(*xs)
+    n = arr([576, 0, 1000])
+    need = lib.trevs_cls_saliency_workspace_size(3, n, 16)
+    assert need > 4 * 16 * 1576 and need % 256 == 0
+    assert lib.trevs_cls_saliency_workspace_size(0, n, 16) == 0
+
+    def cls(B=3, nn=n, H=16, dh=64, q=FAKE, K=FAKE, s=FAKE, ws=FAKE, nb=need, strides=(1024, 64, 1024, 64),
+            scale=0.0):
+        return lib.trevs_cls_saliency_varlen(q, strides[0], strides[1], K, strides[2], strides[3], B, nn, H, dh,
+                                             scale, s, ws, nb, None)
+    assert cls(dh=72) == t.TREVS_ERR_UNSUPPORTED
+    assert cls(H=129) == t.TREVS_ERR_UNSUPPORTED
+    assert cls(nn=arr([576, 16385, 1])) == t.TREVS_ERR_UNSUPPORTED
+    assert cls(nn=arr([576, -1, 1])) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(H=0) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(K=ctypes.c_void_p(0x10008)) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(strides=(1024, 64, 1020, 64)) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(s=None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(scale=float("inf")) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert cls(nb=need - 1) == t.TREVS_ERR_WORKSPACE
+    assert cls(B=0, nn=None, q=None, K=None, s=None, ws=None, nb=0) == 0
+    assert cls(B=2, nn=arr([0, 0]), q=None, K=None, s=None, ws=None, nb=0) == 0
+    assert t.last_launch_count() == 0
+
+
 def test_stage2_validation(lib):
     def hs(Hq, Hkv, L, K1, dh):
         return lib.trevs_in_llm_head_scores(FAKE, 4096, 128, FAKE, 8192, 128, Hq, Hkv, L, K1, dh, 0.0,

@@ -200,6 +200,26 @@ def small_case(seed_cfg=90, n=(300, 77, 129), m=(5, 17, 1), d=200, hq=4, hkv=2, 
                      2.0, 0, 64)
 
 
+def cls_inputs(n, heads=16, dh=64, seed=77, spikes=8):
+    """Inputs of Eq. 2-3 for requests of n[b] patches, as bf16 bits: the [CLS] query of every
+    head, [B, heads, dh], and the patch keys of the penultimate ViT layer, [sum n, heads, dh].
+    Queries carry per-head scales U(0.5, 2); in every request `spikes` patches get keys pushed
+    along their head's query (the few patches [CLS] attends to). CLIP ViT-L/14 has 16 heads of
+    width 64."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    B = len(n)
+    q = rng.standard_normal((B, heads, dh)) * rng.uniform(0.5, 2.0, size=(B, heads, 1))
+    K = rng.standard_normal((int(sum(n)), heads, dh))
+    off = 0
+    for b, nb in enumerate(n):
+        if nb > 0 and spikes > 0:
+            idx = rng.choice(nb, size=min(spikes, nb), replace=False)
+            u = q[b] / np.linalg.norm(q[b], axis=1, keepdims=True)
+            K[off + idx] += 4.0 * u[None, :, :]
+        off += nb
+    return f32_to_bf16_bits(q.astype(np.float32)), f32_to_bf16_bits(K.astype(np.float32))
+
+
 WORKLOADS = {
     "llava15_576_single": llava15_single,
     "llava15_576_b32": llava15_batch32,
