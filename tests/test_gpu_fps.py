@@ -22,13 +22,9 @@ if not torch.cuda.is_available():   # pragma: no cover - CPU container
 from paper_2609_37581_gb300 import trevs as T  # noqa: E402
 from tests import gpu_harness as H  # noqa: E402
 
-TOL = 5e-5
-
-
-def _unit_rows(Z_bits):
-    Z = O.bf16_bits_to_f64(Z_bits)
-    nz = np.sqrt((Z * Z).sum(1))
-    return np.divide(Z, nz[:, None], out=np.zeros_like(Z), where=nz[:, None] > 0)
+TOL = H.FPS_TOL
+_unit_rows = H.unit_rows
+check_method_stage1 = H.check_method_stage1
 
 
 def check_draws(Z_bits, pivots, picks, dist, k_d):
@@ -176,64 +172,6 @@ def test_fps_pivot_outside_range_is_a_zero_row():
 
 
 # ------------------------------------------------------------------ the batched Method path
-
-
-def _check_draw_set(Z_bits, pivots, draws):
-    """`draws` (a set) is what K_d farthest-point steps from `pivots` can yield: replayed
-    greedily, every step's farthest member of the set is within TOL of the farthest row."""
-    U = _unit_rows(Z_bits)
-    cand = np.ones(len(U), dtype=bool)
-    cur = np.full(len(U), np.inf)
-    for s in pivots:
-        cand[s] = False
-        cur = np.minimum(cur, 1.0 - U @ U[s])
-    left = set(int(x) for x in draws)
-    while left:
-        g = max(left, key=lambda i: (cur[i], -i))
-        assert cur[g] >= cur[cand].max() - TOL, f"draw {g} at {cur[g]!r}, the farthest is at {cur[cand].max()!r}"
-        left.remove(g)
-        cand[g] = False
-        cur = np.minimum(cur, 1.0 - U @ U[g])
-
-
-def check_method_stage1(w, g, mode, rho):
-    """Stage 1 with diversity draws against the oracle, request by request. Returns
-    (exact, near): near counts requests that left the oracle's set at a near tie, either of
-    the rule at K_r (then the set only has to be well formed) or of the draws (then the
-    pivots must match and the draws form a valid farthest-point set)."""
-    n_off, m_off, k1_off = w.offsets("n"), w.offsets("m"), w.offsets("k1")
-    exact = near = 0
-    for b, r in enumerate(w.reqs):
-        Zb = w.Z[n_off[b]:n_off[b + 1]]
-        ref = O.pre_llm_request(Zb, w.T[m_off[b]:m_off[b + 1]], w.s_v[n_off[b]:n_off[b + 1]], r.k1, r.ratio,
-                                mode, diversity=rho)
-        kept = g.kept1[k1_off[b]:k1_off[b + 1]]
-        assert len(kept) == r.k1
-        if r.k1 == 0:
-            continue
-        assert np.all(np.diff(kept) > 0) and kept[0] >= 0 and kept[-1] < r.n, f"req {b}: bad kept set"
-        np.testing.assert_array_equal(g.Z_out[k1_off[b]:k1_off[b + 1]], Zb[kept])
-        if list(kept) == list(ref["kept"]):
-            exact += 1
-            continue
-        kd = O.diversity_count(r.k1, rho)
-        kr = r.k1 - kd
-        piv = list(ref.get("pivots", ref["kept"]))
-        if not set(piv) <= set(kept.tolist()):
-            sv = w.s_v[n_off[b]:n_off[b + 1]].astype(np.float64)
-            if mode == "fused":
-                gap = H.boundary_gap(ref["s_fused"], kr)
-            else:
-                kt = O.textual_count(kr, r.ratio)
-                Sv = O.top_k(sv, kr - kt)
-                rest = np.ones(r.n, bool)
-                rest[Sv] = False
-                gap = min(H.boundary_gap(sv, kr - kt), H.boundary_gap(ref["s_t"], kt, rest))
-            assert gap < H.NEAR_TIE, f"req {b}: pivots differ without a near tie (gap {gap})"
-        else:
-            _check_draw_set(Zb, piv, sorted(set(kept.tolist()) - set(piv)))
-        near += 1
-    return exact, near
 
 
 @pytest.mark.parametrize("mode", ["fused", "ratio"])
