@@ -835,12 +835,10 @@ trevs_status trevs_cls_saliency_varlen(const uint16_t* q_cls, int64_t q_req_stri
   if (H > TREVS_MAX_HEADS) return fail(TREVS_ERR_UNSUPPORTED, "H = %d > %d", H, TREVS_MAX_HEADS);
   if (!cls_head_dim_supported(d_h)) return fail(TREVS_ERR_UNSUPPORTED, "d_h = %d: 32, 64 or 128 supported", d_h);
   long long total = 0;
-  int max_n = 0;
   for (int b = 0; b < B; ++b) {
     TREVS_CHECK(n[b] >= 0, "request %d: n = %d < 0", b, n[b]);
     if (n[b] > kClsMaxN) return fail(TREVS_ERR_UNSUPPORTED, "request %d: n = %d > %d patches", b, n[b], kClsMaxN);
     total += n[b];
-    max_n = n[b] > max_n ? n[b] : max_n;
   }
   TREVS_CHECK(total < (1ll << 31), "batch too large for int32 offsets");
   if (total == 0) return TREVS_OK;
@@ -880,7 +878,6 @@ trevs_status trevs_cls_saliency_varlen(const uint16_t* q_cls, int64_t q_req_stri
     TREVS_TRY_CUDA(counted(launch_cls_saliency(meta, a, d_h, chunk_max, (cudaStream_t)stream)), "saliency launch");
     n_base += no;
   }
-  (void)max_n;
   return TREVS_OK;
 }
 
