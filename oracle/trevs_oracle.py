@@ -32,6 +32,12 @@ Readings where the paper is silent or leaves a choice open:
     distance +inf, so the first pick is the lowest index of C.
   * K_d = floor(rho*K1 + 0.5) for a diversity share rho (the paper's K_r:K_d = 3:1 is
     rho = 0.25); the pivots are the top K_r = K1 - K_d of the stage-1 rule.
+  * Full-sequence variant of the Sec. 4.2 softmax (off by default): given lse_other[h, q],
+    the log of the summed exp-logits of row q's non-visual keys (system and text tokens),
+    the denominator also counts that mass, as the LLM's own softmax over the whole sequence
+    does; rows then sum to less than 1, and Eq. 8-9 take those values as they are.
+  * Eq. 1 compares each head's visual-token attention distribution under two questions; a
+    head's distribution is its attention averaged over the text rows (a distribution again).
   * [CLS] saliency (Eq. 2-3): the softmax of each head runs over the N patch keys, as Eq. 2
     writes it (K_v holds the patch keys only), with scale 1/sqrt(d_h); s^v is the plain mean
     of the H heads' distributions.
@@ -214,11 +220,14 @@ def gather_rows(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
 # ---------------------------------------------------------------- stage 2 (Sec. 4.2)
 
 
-def text_to_vision_attention(Q: np.ndarray, K: np.ndarray, scale: float | None = None):
+def text_to_vision_attention(Q: np.ndarray, K: np.ndarray, scale: float | None = None,
+                             lse_other: np.ndarray | None = None):
     """A^h_{T->V}[q, i] = softmax_i( Q[q, h] . K[i, g(h)] * scale ), g(h) = floor(h*Hkv/Hq).
 
     Q is [L, Hq, dh] (text rows at layer l*), K is [K1, Hkv, dh] (visual keys).
-    Returns A as [Hq, L, K1]; every row is a distribution over the K1 visual keys.
+    Returns A as [Hq, L, K1]; every row is a distribution over the K1 visual keys. With
+    lse_other [Hq, L] the denominator of row (h, q) also holds exp(lse_other[h, q]), the mass
+    of the row's non-visual keys, and the row sums to less than 1.
     """
     Q = np.asarray(Q, dtype=np.float64)
     K = np.asarray(K, dtype=np.float64)
@@ -230,9 +239,35 @@ def text_to_vision_attention(Q: np.ndarray, K: np.ndarray, scale: float | None =
     for h in range(Hq):
         g = (h * Hkv) // Hq
         logits = (Q[:, h, :] @ K[:, g, :].T) * scale          # [L, K1]
-        e = np.exp(logits - logits.max(axis=1, keepdims=True))
-        A[h] = e / e.sum(axis=1, keepdims=True)
+        mx = logits.max(axis=1, keepdims=True)
+        if lse_other is not None:
+            other = np.asarray(lse_other, dtype=np.float64)[h][:, None]
+            mx = np.maximum(mx, other)
+        e = np.exp(logits - mx)
+        den = e.sum(axis=1, keepdims=True)
+        if lse_other is not None:
+            den = den + np.exp(other - mx)
+        A[h] = e / den
     return A
+
+
+def head_visual_attention(A: np.ndarray) -> np.ndarray:
+    """s_h of Eq. 1: head h's attention over the visual tokens, averaged over the text rows.
+
+    A is [Hq, L, K1] (text-to-vision attention); returns [Hq, K1].
+    """
+    A = np.asarray(A, dtype=np.float64)
+    return A.sum(axis=1) / A.shape[1]
+
+
+def textual_sensitivity(s1: np.ndarray, s2: np.ndarray) -> np.ndarray:
+    """Eq. 1: TS_h = 1 - cos(s_h^(1), s_h^(2)) for the distributions of every head under two
+    questions; s1 and s2 are [Hq, K1]. Returns [Hq]."""
+    s1 = np.asarray(s1, dtype=np.float64)
+    s2 = np.asarray(s2, dtype=np.float64)
+    num = (s1 * s2).sum(axis=1)
+    den = np.sqrt((s1 * s1).sum(axis=1)) * np.sqrt((s2 * s2).sum(axis=1))
+    return 1.0 - num / den
 
 
 def head_variance(A: np.ndarray) -> np.ndarray:

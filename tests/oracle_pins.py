@@ -473,4 +473,61 @@ def pin_cls_saliency_invariants():
     _close(O.cls_saliency(q, K + rng.standard_normal((1, H, dh))), s, 1e-10)  # one shift per head
 
 
+
+# ------------------------------------------------------------- Sec. 4.2 full-sequence variant, Eq. 1
+
+
+def pin_full_sequence_softmax_is_a_restriction():
+    """The variant with lse_other = logsumexp of some extra keys' logits equals the plain
+    softmax over the visual keys and those extra keys, restricted to the visual columns."""
+    from scipy.special import logsumexp, softmax
+    rng = np.random.default_rng(47)
+    L, Hq, Hkv, dh, K1, E = 5, 4, 2, 16, 11, 7
+    Q = rng.standard_normal((L, Hq, dh)) * 2.0
+    K = rng.standard_normal((K1, Hkv, dh))
+    Kx = rng.standard_normal((E, Hkv, dh))                 # the non-visual keys
+    lse = np.empty((Hq, L))
+    want = np.empty((Hq, L, K1))
+    for h in range(Hq):
+        g = (h * Hkv) // Hq
+        lv = Q[:, h, :] @ K[:, g, :].T / 4.0
+        lx = Q[:, h, :] @ Kx[:, g, :].T / 4.0
+        lse[h] = logsumexp(lx, axis=1)
+        want[h] = softmax(np.concatenate([lv, lx], axis=1), axis=1)[:, :K1]
+    _close(O.text_to_vision_attention(Q, K, lse_other=lse), want, 1e-12)
+
+
+def pin_full_sequence_softmax_closed_forms():
+    rng = np.random.default_rng(53)
+    L, H, dh, K1 = 3, 2, 8, 6
+    K = rng.standard_normal((K1, H, dh))
+    # Q = 0: every logit is 0, so a row is 1 / (K1 + c) with lse_other = ln c
+    A = O.text_to_vision_attention(np.zeros((L, H, dh)), K, lse_other=np.full((H, L), math.log(3.0)))
+    _close(A, np.full((H, L, K1), 1.0 / (K1 + 3.0)))
+    # lse_other = -inf is the plain softmax
+    Q = rng.standard_normal((L, H, dh))
+    _close(O.text_to_vision_attention(Q, K, lse_other=np.full((H, L), -np.inf)),
+           O.text_to_vision_attention(Q, K))
+
+
+def pin_textual_sensitivity():
+    s1 = np.array([[1.0, 0.0], [0.25, 0.75], [0.5, 0.5]])
+    s2 = np.array([[0.5, 0.5], [0.25, 0.75], [1.0, 0.0]])
+    # head 0: cos = (1/2) / (1 * sqrt(1/2)) = 1/sqrt(2); head 1: identical; head 2: cos = 1/sqrt(2)
+    _close(O.textual_sensitivity(s1, s2), [1 - 1 / math.sqrt(2), 0.0, 1 - 1 / math.sqrt(2)])
+    _close(O.textual_sensitivity(np.array([[1.0, 0.0, 0.0]]), np.array([[0.0, 0.3, 0.7]])), [1.0])   # disjoint
+    rng = np.random.default_rng(59)
+    a, b = rng.random((4, 9)), rng.random((4, 9))
+    _close(O.textual_sensitivity(a, 3.0 * b), O.textual_sensitivity(a, b))          # scale
+    _close(O.textual_sensitivity(a, b), O.textual_sensitivity(b, a))                # symmetric
+
+
+def pin_head_visual_attention():
+    A = np.array([[[1.0, 0.0], [0.0, 1.0]], [[0.25, 0.75], [0.75, 0.25]]])
+    _close(O.head_visual_attention(A), [[0.5, 0.5], [0.5, 0.5]])
+    rng = np.random.default_rng(61)
+    A = O.text_to_vision_attention(rng.standard_normal((7, 3, 8)), rng.standard_normal((13, 3, 8)))
+    _close(O.head_visual_attention(A).sum(axis=1), np.ones(3))
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

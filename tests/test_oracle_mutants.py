@@ -265,6 +265,27 @@ def _cls_softmax_over_heads(q, K, scale=None):
     return _cls_generic(q, K, axis="heads")
 
 
+
+_plain_attention = O.text_to_vision_attention
+
+
+def _lse_ignored(Q, K, scale=None, lse_other=None):
+    return _plain_attention(Q, K, scale)
+
+
+def _ts_cos(s1, s2):
+    s1, s2 = np.asarray(s1, float), np.asarray(s2, float)
+    return (s1 * s2).sum(1) / (np.linalg.norm(s1, axis=1) * np.linalg.norm(s2, axis=1))
+
+
+def _ts_unnormalised(s1, s2):
+    return 1.0 - (np.asarray(s1, float) * np.asarray(s2, float)).sum(1)
+
+
+def _head_attention_max(A):
+    return np.asarray(A, float).max(axis=1)
+
+
 MUTANTS = {
     "cos_no_relu": ("rectified_cosine", _no_relu),
     "cos_wrong_norm": ("rectified_cosine", _wrong_norm),
@@ -306,6 +327,10 @@ MUTANTS = {
     "cls_sum_heads": ("cls_saliency", _cls_sum_heads),
     "cls_max_heads": ("cls_saliency", _cls_max_heads),
     "cls_softmax_over_heads": ("cls_saliency", _cls_softmax_over_heads),
+    "lse_other_ignored": ("text_to_vision_attention", _lse_ignored),
+    "ts_cos_not_distance": ("textual_sensitivity", _ts_cos),
+    "ts_unnormalised": ("textual_sensitivity", _ts_unnormalised),
+    "head_attention_max": ("head_visual_attention", _head_attention_max),
 }
 
 

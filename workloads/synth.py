@@ -177,6 +177,18 @@ def long_video_batch2(batch=2):
                      3.0, 0, 16384)
 
 
+def video_llava_batch(batch=4):
+    """Video-LLaVA-shaped: 8 frames x 256 tokens = 2,048 per video, saliency per frame, 3%
+    planted in 8 clusters (one object across the frames), M ~ U{16..48}, d' = 4096 with
+    32 x 128 heads and the top half kept. K1 = 272 and K2 = 91: with the second prune after
+    layer 8 of 32, the LLM keeps (8 * 272 + 24 * 91) / 32 = 136.25 visual tokens per layer,
+    the paper's 136 of 2,048 (K1 about 3 K2)."""
+    lens = np.random.Generator(np.random.PCG64(1000 * 5 + 999)).integers(16, 49, size=batch)
+    reqs = [Request(n=2048, m=int(m), k1=272, ratio=0.5, l=int(m), k2=91) for m in lens]
+    return _assemble(f"video_llava_2048_b{batch}", 5, 4096, 32, 32, 128, 16, reqs, 0.03, 8,
+                     2.0, 0, 256)
+
+
 def ragged_serving_batch64(batch=64):
     """64 varlen requests, N in {576,1152,2880}, M log-uniform 8..256, keep 5.6% (min 32)."""
     g = np.random.Generator(np.random.PCG64(1000 * 4 + 999))
@@ -226,4 +238,5 @@ WORKLOADS = {
     "llava_next_2880_b8": llava_next_batch8,
     "long_16384_b2_gqa": long_video_batch2,
     "ragged_varlen_b64": ragged_serving_batch64,
+    "video_llava_2048_b4": video_llava_batch,
 }
