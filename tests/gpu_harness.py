@@ -14,7 +14,7 @@ import dataclasses
 import numpy as np
 
 import oracle.trevs_oracle as O
-from workloads.device import GpuRun, build_batches, collect, dev_bf16, dev_f32, host_u16, run_gpu  # noqa: F401
+from workloads.device import DeviceRun, build_batches, collect, dev_bf16, dev_f32, host_u16, run_gpu  # noqa: F401
 
 RTOL = 1e-3
 ATOL_ST = 1e-6     # s^t is a mean of squares of cosines: fp32 cosine error ~1e-7 absolute
@@ -61,7 +61,7 @@ class Tally:
     stage2_exact: int = 0
 
 
-def check_workload(w, g: GpuRun, ref, mode="ratio", tally: Tally | None = None, params=None):
+def check_workload(w, g: DeviceRun, ref, mode="ratio", tally: Tally | None = None, params=None):
     """Element-wise comparison of one GPU run with the oracle, request by request."""
     tally = tally or Tally()
     params = params or {}

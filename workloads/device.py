@@ -31,7 +31,7 @@ def host_u16(t):
 
 
 @dataclasses.dataclass
-class GpuRun:
+class DeviceRun:
     s_t: np.ndarray
     s_fused: np.ndarray | None
     kept1: np.ndarray
@@ -103,7 +103,7 @@ def run_gpu(w, mode=T.SELECT_RATIO, params=None, reps=1, stages="both"):
 def collect(w, pre, inb):
     sum_n, sum_k1 = w.Z.shape[0], sum(r.k1 for r in w.reqs)
     sum_k2 = sum(r.k2 for r in w.reqs)
-    return GpuRun(
+    return DeviceRun(
         s_t=pre.s_t.cpu().numpy()[:sum_n],
         s_fused=None if pre.s_fused is None else pre.s_fused.cpu().numpy()[:sum_n],
         kept1=pre.kept_idx.cpu().numpy()[:sum_k1], Z_out=host_u16(pre.Z_out)[:sum_k1],
