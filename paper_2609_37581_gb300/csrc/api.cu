@@ -875,7 +875,8 @@ trevs_status trevs_cls_saliency_varlen(const uint16_t* q_cls, int64_t q_req_stri
     a.attn_ld = no;
     a.s_v = s_v + n_base;
     a.cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
-    TREVS_TRY_CUDA(counted(launch_cls_saliency(meta, a, d_h, chunk_max, (cudaStream_t)stream)), "saliency launch");
+    if (meta.B > 0)
+      TREVS_TRY_CUDA(counted(launch_cls_saliency(meta, a, d_h, chunk_max, (cudaStream_t)stream)), "saliency launch");
     n_base += no;
   }
   return TREVS_OK;
