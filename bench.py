@@ -12,7 +12,10 @@ scores, the Sec. 3.1 split and gather, then attention statistics, Eq. 8-9 and co
              copies its inputs host->device and reads the kept indices back;
   roofline   the dominant kernel (stage-1 scoring + selection): algorithmic bytes per
              launch / its CUDA-event duration, against the measured HBM copy bandwidth;
-  cpu_baseline  the fp64 oracle on the host cores (one process per core, bounded sample).
+  cpu_baseline  the fp64 oracle on the host cores (one process per core, bounded sample);
+  configs    the other single-GPU workloads (LLaVA-NeXT 8 x 2,880, video 2 x 16,384 with
+             GQA, the ragged serving batch of 64), each timed the same way, with its own
+             algorithmic bytes, roofline fraction, scoring-grid time and clocks.
 
 --impl reference times the oracle itself as the reference arm. Under torchrun (N > 1)
 every rank prunes its own copy of the batch (replicas, weak scaling, no collective on
@@ -172,7 +175,7 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.monotonic(), line.strip()))
 
     def __exit__(self, *exc):
         if self.proc:
@@ -182,10 +185,14 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
 
-    def summary(self):
+    def summary(self, t0=None, t1=None):
+        """Median SM clock, max clock and active throttle reasons of the samples taken in
+        [t0, t1] (time.monotonic() seconds; all samples by default)."""
         sm, mx, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for ln in self.lines:
+        for ts, ln in list(self.lines):
+            if (t0 is not None and ts < t0) or (t1 is not None and ts > t1):
+                continue
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 7:
                 continue
@@ -220,6 +227,85 @@ def replica_throughput(max_elapsed_ms: float, steps: int, tokens_per_rank_step: 
     timed by the slowest rank."""
     ms = max_elapsed_ms / steps
     return ms, tokens_per_rank_step * world / (ms * 1e-3)
+
+
+OTHER_CONFIGS = {   # the north star's other single-GPU configurations, each timed like the headline one
+    "llava_next_2880_b8": synth.llava_next_batch8,
+    "long_16384_b2_gqa": synth.long_video_batch2,
+    "ragged_varlen_b64": synth.ragged_serving_batch64,
+}
+
+
+def time_workload(T, w, stream, sampler, steps, peak, src):
+    """us per trevs_prune_varlen call on workload `w`: CUDA-event timing around graph replays
+    over ROTATING_SETS input sets (each set > L2), the scoring grid timed alone with the
+    library's event hook, the clocks sampled meanwhile."""
+    import torch
+    from workloads.device import build_batches, dev_bf16, dev_f32
+    params = T.default_params(T.SELECT_RATIO)
+    with torch.cuda.stream(stream):
+        base = {"Z": dev_bf16(w.Z), "T": dev_bf16(w.T), "s_v": dev_f32(w.s_v), "Q": dev_bf16(w.Q),
+                "K": dev_bf16(w.K), "V": dev_bf16(w.V), "hidden": dev_bf16(w.hidden)}
+        sets = [base] + [{k: v.clone() for k, v in base.items()} for _ in range(ROTATING_SETS - 1)]
+        batches = [build_batches(w, T.SELECT_RATIO, dev=x) for x in sets]
+        ws = T.workspace(max(T.trevs_prune_varlen_workspace_size(p, i) for p, i in batches))
+        calls = [T.PreparedCall(p, i, ws, params) for p, i in batches]
+        for c in calls:
+            c(stream)
+        launches = T.last_launch_count()
+        graphs = []
+        for c in calls:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                c(stream)
+            graphs.append(g)
+        score_only = []
+        for p, _ in batches:
+            q = T.PreBatch(reqs=p.reqs, Z=p.Z, T=p.T, s_v=p.s_v, kept_idx=p.kept_idx, Z_out=None, s_t=p.s_t)
+            score_only.append((q, T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))))
+    torch.cuda.synchronize()
+    t0 = time.monotonic()
+    with torch.cuda.stream(stream):
+        for i in range(10):
+            graphs[i % ROTATING_SETS].replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for i in range(steps):
+            graphs[i % ROTATING_SETS].replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        nk = 64
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nk)]
+        for x, y in evs:
+            x.record(stream); y.record(stream)
+        torch.cuda.synchronize()
+        torch.cuda._sleep(int(2e9 * 3e-4 * nk))
+        for i in range(nk):
+            q, wsq = score_only[i % ROTATING_SETS]
+            T.trevs_pre_llm_varlen_timed(q, wsq, evs[i][0], evs[i][1], params, stream)
+        torch.cuda.synchronize()
+        kernel_ms = statistics.median(x.elapsed_time(y) for x, y in evs[8:])
+    t1 = time.monotonic()
+    nbytes = algorithmic_bytes(w)
+    del graphs, calls, score_only, sets, batches, ws
+    torch.cuda.empty_cache()
+    return {
+        "workload": w.name, "requests": w.B, "visual_tokens": w.visual_tokens(), "d": w.d,
+        "query_tokens": f"{min(r.m for r in w.reqs)}..{max(r.m for r in w.reqs)}",
+        "K1": sorted({r.k1 for r in w.reqs}), "K2": sorted({r.k2 for r in w.reqs}),
+        "heads": f"{w.hq}/{w.hkv}x{w.dh}, keep {w.n_keep_heads}",
+        "us_per_prune": round(ms * 1e3, 2), "value": w.visual_tokens() / (ms * 1e-3), "unit": UNIT,
+        "steps": steps, "launches_per_step": launches,
+        "algorithmic_bytes": nbytes["step"],
+        "achieved_gbs": round(nbytes["step"] / (ms * 1e-3) / 1e9, 1),
+        "frac": round(nbytes["step"] / (ms * 1e-3) / 1e9 / peak, 4), "peak": peak, "peak_source": src,
+        "score_kernel": {"kernel_us": round(kernel_ms * 1e3, 2), "algorithmic_bytes": nbytes["score_kernel"],
+                         "frac": round(nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9 / peak, 4)},
+        "clocks": sampler.summary(t0, t1),
+        "timed": f"CUDA events around {steps} graph replays of trevs_prune_varlen, {ROTATING_SETS} rotating "
+                 "input sets (> L2)"}
 
 
 def gpu_arm(args, rank, world, w, cpu_baseline):
@@ -287,11 +373,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         barrier()
         torch.cuda.synchronize()
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        tw0 = time.monotonic()
         ev0.record(stream)
         for i in range(args.steps):
             graphs[i % ROTATING_SETS].replay()
         ev1.record(stream)
         torch.cuda.synchronize()
+        timed_window = (tw0, time.monotonic())
         barrier()
         elapsed_ms = ev0.elapsed_time(ev1)
         # dominant kernel: the library records two CUDA events on the stream right around the
@@ -343,6 +431,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         torch.cuda.synchronize()
         cls_ms = c0.elapsed_time(c1) / csteps
         cls_bytes = sum(x.numel() * x.element_size() for x in csets[0]) + cs_v.numel() * 4
+        # the other configurations of the benchmark spec, one after the other
+        peak, src = peaks()
+        others = {}
+        if not args.no_configs:
+            del csets, cs_v, cws
+            for name, make in OTHER_CONFIGS.items():
+                others[name] = time_workload(T, make(), stream, sampler, max(50, min(args.steps, 2000)), peak, src)
 
     if distributed:
         elapsed_ms = max_over_ranks(elapsed_ms, dev)
@@ -408,9 +503,8 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
     ms, value = replica_throughput(elapsed_ms, args.steps, w.visual_tokens(), world)
     method_kd = int(np.floor(np.float32(METHOD_RHO) * WORKLOAD["k1"] + 0.5))
     nbytes = algorithmic_bytes(w)
-    peak, src = peaks()
     achieved = nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9
-    clk = sampler.summary()
+    clk = sampler.summary(*timed_window)
     return {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
@@ -445,6 +539,7 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
             "frac": round(cls_bytes / (cls_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
             "timed": "CUDA events around 200 trevs_cls_saliency_varlen calls queued behind a spin kernel, "
                      "4 rotating input sets"},
+        "configs": others,
     }
 
 
@@ -488,14 +583,18 @@ def reference_arm(args, w):
 
 
 def profile_run(w, stage="stage1", launches=5):
-    """Stage 1 (scoring + selection; "method": with the fused score and the diversity draws)
-    or stage 2 of the bench batch, launched eagerly."""
+    """Stage 1 (scoring + selection; "method": with the fused score and the diversity draws),
+    stage 2, or both stages ("both") of workload `w`, launched eagerly."""
     import torch
     from paper_2609_37581_gb300 import trevs as T
     from workloads.device import build_batches
     T.load()
     pre, inb = build_batches(w, T.SELECT_RATIO)
-    if stage in ("stage1", "method"):
+    if stage == "both":
+        ws = T.workspace(T.trevs_prune_varlen_workspace_size(pre, inb))
+        for _ in range(launches):
+            T.trevs_prune_varlen(pre, inb, ws, T.default_params(T.SELECT_RATIO))
+    elif stage in ("stage1", "method"):
         q = T.PreBatch(reqs=pre.reqs, Z=pre.Z, T=pre.T, s_v=pre.s_v, kept_idx=pre.kept_idx, s_t=pre.s_t)
         ws = T.workspace(T.trevs_pre_llm_varlen_workspace_size(q))
         params = (T.default_params(T.SELECT_RATIO) if stage == "stage1"
@@ -517,9 +616,14 @@ def main():
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--profile", nargs="?", const="stage1", choices=["stage1", "stage2", "method"],
-                    help="only run stage 1 (stage 2, or stage 1 with the Method's diversity draws) of the "
-                         "bench batch a few times, for an ncu capture")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the timing of the other configurations (2,880, 16,384 tokens, ragged batch)")
+    ap.add_argument("--profile", nargs="?", const="stage1", choices=["stage1", "stage2", "method", "both"],
+                    help="only run stage 1 (stage 2, stage 1 with the Method's diversity draws, or the "
+                         "two-stage call) of a workload a few times, for an ncu capture")
+    ap.add_argument("--workload", default="llava15_576_b32", choices=sorted(synth.WORKLOADS),
+                    help="workload of --profile (default: the bench batch)")
+    ap.add_argument("--launches", type=int, default=5, help="calls made by --profile")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -535,10 +639,11 @@ def main():
         print(json.dumps(reference_arm(args, w)), flush=True)
         return
 
-    w = workload()
     if args.profile:
-        profile_run(w, args.profile)
+        pw = workload() if args.workload == "llava15_576_b32" else synth.WORKLOADS[args.workload]()
+        profile_run(pw, args.profile, args.launches)
         return
+    w = workload()
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = time_oracle(w)                     # before any CUDA call: the pool forks safely

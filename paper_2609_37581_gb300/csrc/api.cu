@@ -341,7 +341,8 @@ trevs_status validate_diversity(const trevs_pre_batch* bt, const trevs_pre_param
 trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& prm, int b0, int b1,
                            long long n_base, long long m_base, long long k1_base, uint8_t* ws,
                            const PreWs& L, cudaStream_t st, GatherMeta* gm_out, cudaEvent_t after_score = nullptr,
-                           cudaEvent_t before_score = nullptr, cudaStream_t tail = nullptr, int reserve = 0) {
+                           cudaEvent_t before_score = nullptr, cudaStream_t tail = nullptr, int reserve = 0,
+                           bool* forked = nullptr) {
   static thread_local PreMeta meta;
   static thread_local GatherMeta gm;
   static thread_local int kd_of[kMaxChunk];
@@ -394,7 +395,10 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");
   if (after_score) TREVS_TRY_CUDA(cudaEventRecord(after_score, st), "event after scoring");
   // the rest of stage 1 goes on `tail` (after the scoring grid completes) when given
-  if (tail) TREVS_TRY_CUDA(cudaStreamWaitEvent(tail, after_score, 0), "tail after scoring");
+  if (tail) {
+    TREVS_TRY_CUDA(cudaStreamWaitEvent(tail, after_score, 0), "tail after scoring");
+    if (forked) *forked = true;
+  }
   const cudaStream_t ts = tail ? tail : st;
   TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, max_m, max_n, true, ts, !tail)), "finishing launch");
   if (draws) {
@@ -1258,6 +1262,17 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
       max_k1 = in->reqs[b].k1 > max_k1 ? in->reqs[b].k1 : max_k1;
     }
     const int reserve = overlap_reserve(pre, in, tp, in_small_fits(in->Hq, max_l, max_k1));
+    // Once work has forked onto the auxiliary stream it is joined back into `stream` on every
+    // return, errors included, so that a stream capture never ends with an unjoined branch
+    // and `stream` stays ordered after everything the call enqueued.
+    bool forked = false;
+    auto joined = [&](trevs_status status) -> trevs_status {
+      if (!forked) return status;
+      const cudaError_t e1 = cudaEventRecord(aux->join, aux->stream);
+      const cudaError_t e2 = e1 == cudaSuccess ? cudaStreamWaitEvent(st, aux->join, 0) : e1;
+      if (status == TREVS_OK && e2 != cudaSuccess) return cuda_fail(e2, "join");
+      return status;
+    };
     if (reserve > 0) {
       // One chunk each, and the stages are independent. The scoring grid leaves `reserve`
       // SMs free; stage 2 launches right behind it on the same stream (programmatic launch,
@@ -1265,13 +1280,10 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
       // while the grid streams Z. The finishing grid and gather of stage 1 follow the scoring
       // grid's completion on the auxiliary stream, which joins back at the end.
       s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork, nullptr, aux->stream,
-                        reserve);
-      if (s != TREVS_OK) return s;
+                        reserve, &forked);
+      if (s != TREVS_OK) return joined(s);
       s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true);
-      if (s != TREVS_OK) return s;
-      TREVS_TRY_CUDA(cudaEventRecord(aux->join, aux->stream), "join");
-      TREVS_TRY_CUDA(cudaStreamWaitEvent(st, aux->join, 0), "join");
-      return TREVS_OK;
+      return joined(s);
     }
     // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
     // 2 (with its own compaction) forks once that grid is enqueued, so it waits for it to
@@ -1279,11 +1291,9 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
     s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork);
     if (s != TREVS_OK) return s;
     TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
+    forked = true;
     s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true);
-    if (s != TREVS_OK) return s;
-    TREVS_TRY_CUDA(cudaEventRecord(aux->join, aux->stream), "join");
-    TREVS_TRY_CUDA(cudaStreamWaitEvent(st, aux->join, 0), "join");
-    return TREVS_OK;
+    return joined(s);
   }
   if (pre->B > 0) {
     s = run_pre_batch(pre, prm, ws, LP, st);

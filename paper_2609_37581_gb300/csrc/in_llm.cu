@@ -487,6 +487,9 @@ __global__ void __launch_bounds__(kSelThreads) in_select_small_kernel(const __gr
       if (sel) s_heads[before + __popc(bal & lanemask_lt())] = hh;
       __syncthreads();
     }
+    // at most n_keep heads, the lowest of those ranked first, even if u holds NaN (a NaN
+    // compares false with everything, so its head ranks 0 and joins the n_keep best)
+    nh = min(nh, a.n_keep);
     // Eq. 9 for key i: rows rg, rg + 8, ... (L <= 64: eight rows), every head's loads in flight
     const int i = kb * kSelKeys + (tid % kSelKeys), rg = tid / kSelKeys;
     const float* A = a.attn + r.attn_off + i;

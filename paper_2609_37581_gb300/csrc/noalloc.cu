@@ -21,8 +21,11 @@ void record_launches(int n);
 namespace {
 
 // Layout of the fixed scratch, in 32-bit words: the token scores p (atomicMax target, cleared
-// by every call), the per-request ticket of the selecting block, and the selection keys /
-// flags the kernel falls back to when they do not fit in shared memory.
+// by every call), the per-request ticket of the selecting block, and room for the selection
+// keys / flags. The token-score kernel keeps keys and flags in global memory only when its
+// dynamic shared memory is smaller than 5 K1 bytes; launch_in_token_score asks for
+// 5 K1 + 16 bytes, so with that sizing the keys / flags region is never touched. It stays as
+// a guard: the kernel's pointers must stay valid should the shared-memory sizing change.
 constexpr int kMaxK1 = TREVS_MAX_STAGE2_TOKENS;
 constexpr int kOffP = 0;
 constexpr int kOffTicket = kMaxK1;

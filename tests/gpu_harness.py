@@ -3,8 +3,13 @@
 Comparison rules (tolerances follow from fp32 accumulation of bf16 products):
   * float scores (s^t, fused s, u_h, p_i): |gpu - oracle| <= RTOL * |oracle| + ATOL;
   * kept index sets: identical, unless the oracle's K-th and (K+1)-th scores differ by
-    less than NEAR_TIE relative; such near-ties are counted, and the GPU set must then
-    still hold exactly K distinct valid indices;
+    less than NEAR_TIE relative. Such near-ties are counted, and the GPU set must then
+    equal the oracle's outside the tie band: every candidate whose oracle score lies above
+    the K-th score by more than NEAR_TIE relative is kept, none below it by more than
+    NEAR_TIE is, and the set holds exactly K distinct valid indices;
+  * at a near tie on the head variances the GPU's H* must pass the same band rule, and the
+    token scores and the stage-2 kept set are then checked against the oracle's Eq. 9 over
+    the GPU's own H*;
   * gathered / compacted rows: bit-exact copies of the rows the GPU kept.
 """
 from __future__ import annotations
@@ -52,6 +57,39 @@ def boundary_gap(scores, k, allowed=None):
     return 0.0 if den == 0 else abs(a - b) / den
 
 
+def _rel(a, b):
+    den = np.maximum(np.abs(a), np.abs(b))
+    return np.divide(np.abs(a - b), den, out=np.zeros_like(den, dtype=np.float64), where=den > 0)
+
+
+def check_band(kept, scores, k, allowed=None, what="", below=True):
+    """The band rule at a near tie: `kept` (indices) holds every candidate whose oracle score
+    exceeds the oracle's k-th score by more than NEAR_TIE relative and (with `below`) no
+    candidate that falls short of it by more than NEAR_TIE; only candidates inside the band
+    may differ from the oracle's set. Returns the number of candidates inside the band."""
+    s = np.asarray(scores, np.float64)
+    cand = np.ones(len(s), bool) if allowed is None else np.asarray(allowed, bool).copy()
+    kept = np.asarray(kept, np.int64)
+    mask = np.zeros(len(s), bool)
+    mask[kept] = True
+    assert not (mask & ~cand).any(), f"{what}: kept an index that is not a candidate"
+    if k <= 0:
+        assert not (mask & cand).any(), f"{what}: kept a candidate with k = 0"
+        return 0
+    tau = np.sort(s[cand])[::-1][k - 1]
+    far = _rel(s, tau) > NEAR_TIE
+    above = cand & far & (s > tau)
+    under = cand & far & (s < tau)
+    missing = np.flatnonzero(above & ~mask)
+    assert missing.size == 0, (f"{what}: {missing.size} candidates above the tie band dropped, "
+                               f"first {int(missing[0])} at {s[missing[0]]!r} (k-th {tau!r})")
+    if below:
+        extra = np.flatnonzero(under & mask)
+        assert extra.size == 0, (f"{what}: {extra.size} candidates below the tie band kept, "
+                                 f"first {int(extra[0])} at {s[extra[0]]!r} (k-th {tau!r})")
+    return int((cand & ~far).sum())
+
+
 @dataclasses.dataclass
 class Tally:
     requests: int = 0
@@ -65,7 +103,7 @@ def check_workload(w, g: DeviceRun, ref, mode="ratio", tally: Tally | None = Non
     """Element-wise comparison of one GPU run with the oracle, request by request."""
     tally = tally or Tally()
     params = params or {}
-    n_off, k1_off, k2_off = w.offsets("n"), w.offsets("k1"), w.offsets("k2")
+    n_off, k1_off, k2_off, l_off = w.offsets("n"), w.offsets("k1"), w.offsets("k2"), w.offsets("l")
     for b, r in enumerate(w.reqs):
         tally.requests += 1
         res = ref[b]
@@ -87,9 +125,17 @@ def check_workload(w, g: DeviceRun, ref, mode="ratio", tally: Tally | None = Non
                 # saliency decisions compare the same fp32 inputs on both sides: exact;
                 # only the computed textual scores carry a near-tie band
                 near = boundary_gap(pre["s_t"], kt, rest) < NEAR_TIE
+                if near:
+                    kept_set = set(kept.tolist())
+                    assert set(Sv.tolist()) <= kept_set, f"req {b}: saliency side S_v not kept"
+                    St = np.array(sorted(kept_set - set(Sv.tolist())), np.int64)
+                    assert len(St) == kt
+                    check_band(St, pre["s_t"], kt, rest, f"req {b} stage-1 textual side")
             else:
                 assert_close(g.s_fused[n_off[b]:n_off[b + 1]], pre["s_fused"], RTOL, ATOL_FUSED, f"req {b} fused")
                 near = boundary_gap(pre["s_fused"], r.k1) < NEAR_TIE
+                if near:
+                    check_band(kept, pre["s_fused"], r.k1, None, f"req {b} stage-1 fused")
             if near:
                 tally.stage1_near_ties += 1
             else:
@@ -108,16 +154,26 @@ def check_workload(w, g: DeviceRun, ref, mode="ratio", tally: Tally | None = Non
             assert len(kept2) == r.k2
             assert np.all(np.diff(kept2) > 0), f"req {b}: stage-2 indices not strictly ascending"
             assert kept2.size == 0 or (kept2[0] >= 0 and kept2[-1] < r.k1)
+            p_ref = inn["p"]
             if head_near:
-                tally.stage2_near_ties += 1
+                # H* may differ inside the band; Eq. 9 is then checked over the GPU's own H*
+                assert len(heads) == w.n_keep_heads and np.all(np.diff(heads) > 0), f"req {b}: bad H*"
+                check_band(heads, inn["u"], w.n_keep_heads, None, f"req {b} H*")
+                A = O.text_to_vision_attention(O.bf16_bits_to_f64(w.Q[l_off[b]:l_off[b + 1]]),
+                                               O.bf16_bits_to_f64(w.K[k1_off[b]:k1_off[b + 1]]))
+                p_ref = O.token_scores(A, heads)
             else:
                 np.testing.assert_array_equal(heads, inn["heads"], err_msg=f"req {b} heads")
-                assert_close(g.p[k1_off[b]:k1_off[b + 1]], inn["p"], RTOL, ATOL_P, f"req {b} p")
-                if boundary_gap(inn["p"], r.k2) < NEAR_TIE:
-                    tally.stage2_near_ties += 1
-                else:
-                    np.testing.assert_array_equal(kept2, inn["kept"], err_msg=f"req {b} stage-2 kept set")
-                    tally.stage2_exact += 1
+            assert_close(g.p[k1_off[b]:k1_off[b + 1]], p_ref, RTOL, ATOL_P, f"req {b} p")
+            p_near = boundary_gap(p_ref, r.k2) < NEAR_TIE
+            if p_near:
+                check_band(kept2, p_ref, r.k2, None, f"req {b} stage-2 kept set")
+            else:
+                np.testing.assert_array_equal(kept2, O.top_k(p_ref, r.k2), err_msg=f"req {b} stage-2 kept set")
+            if head_near or p_near:
+                tally.stage2_near_ties += 1
+            else:
+                tally.stage2_exact += 1
             Hb = w.hidden[k1_off[b]:k1_off[b + 1]]
             Kb = w.K[k1_off[b]:k1_off[b + 1]]
             Vb = w.V[k1_off[b]:k1_off[b + 1]]
@@ -158,8 +214,8 @@ def check_draw_set(Z_bits, pivots, draws):
 def check_method_stage1(w, g, mode, rho):
     """Stage 1 with diversity draws against the oracle, request by request. Returns
     (exact, near): near counts requests that left the oracle's set at a near tie, either of
-    the rule at K_r (then the set only has to be well formed) or of the draws (then the
-    pivots must match and the draws form a valid farthest-point set)."""
+    the rule at K_r (then every candidate above the rule's tie band must still be kept) or of
+    the draws (then the pivots must match and the draws form a valid farthest-point set)."""
     n_off, m_off, k1_off = w.offsets("n"), w.offsets("m"), w.offsets("k1")
     exact = near = 0
     for b, r in enumerate(w.reqs):
@@ -189,6 +245,16 @@ def check_method_stage1(w, g, mode, rho):
                 rest[Sv] = False
                 gap = min(boundary_gap(sv, kr - kt), boundary_gap(ref["s_t"], kt, rest))
             assert gap < NEAR_TIE, f"req {b}: pivots differ without a near tie (gap {gap})"
+            # the pivots are a subset of the kept set: every candidate above the tie band of
+            # the rule is kept (below the band a token may still be a draw)
+            if mode == "fused":
+                check_band(kept, ref["s_fused"], kr, None, f"req {b} pivots (fused)", below=False)
+            else:
+                Sv_set = set(Sv.tolist())
+                check_band(sorted(Sv_set & set(kept.tolist())), sv, kr - kt, None,
+                           f"req {b} pivots (saliency side)", below=False)
+                check_band(sorted(set(kept.tolist()) - Sv_set), ref["s_t"], kt, rest,
+                           f"req {b} pivots (textual side)", below=False)
         else:
             check_draw_set(Zb, piv, sorted(set(kept.tolist()) - set(piv)))
         near += 1

@@ -193,3 +193,34 @@ def test_timed_stage1_matches_untimed():
         outs.append((q.s_t.cpu().numpy(), q.kept_idx.cpu().numpy(), H.host_u16(q.Z_out)))
     for a, b in zip(*outs):
         np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("path", ["small", "large"])
+def test_stage2_nan_u_stays_in_bounds(path):
+    """Inputs must be finite, but a non-finite query must not make the library write out of
+    bounds: an Inf in one head's queries gives that head u = NaN, which ranks it among the
+    kept heads; H* still holds at most n_keep heads and nothing past the outputs changes."""
+    k1, l = (64, 16) if path == "small" else (300, 80)   # the small two-grid path, or the larger one
+    w = synth.small_case(seed_cfg=99, n=(k1 + 5, k1 + 9), m=(l, l), d=64, hq=8, hkv=4, n_keep_heads=3,
+                         k1=(k1, k1), ratio=(0.5, 0.5), k2=(16, 16))
+    Q = w.Q.copy()
+    Q[0, 5, 0] = 0x7F80                       # +Inf in request 0, text row 0, head 5
+    pre, inb = H.build_batches(w)
+    inb.Q = H.dev_bf16(Q)
+    canary = 0x5EEDF00D
+    heads_buf = torch.full((w.B * w.n_keep_heads + 64,), canary, dtype=torch.int32, device="cuda")
+    kept_buf = torch.full((sum(r.k2 for r in w.reqs) + 64,), canary, dtype=torch.int32, device="cuda")
+    inb.heads = heads_buf[:w.B * w.n_keep_heads].view(w.B, w.n_keep_heads)
+    inb.kept_local = kept_buf[:sum(r.k2 for r in w.reqs)]
+    ws = T.workspace(T.trevs_in_llm_varlen_workspace_size(inb))
+    T.trevs_in_llm_varlen(inb, ws)
+    torch.cuda.synchronize()
+    hb, kb = heads_buf.cpu().numpy(), kept_buf.cpu().numpy()
+    assert np.all(hb[w.B * w.n_keep_heads:] == canary), "write past heads_out"
+    assert np.all(kb[sum(r.k2 for r in w.reqs):] == canary), "write past kept_local"
+    heads = hb[:w.B * w.n_keep_heads].reshape(w.B, w.n_keep_heads)
+    assert np.all((heads >= 0) & (heads < w.hq))
+    assert np.isnan(inb.u.cpu().numpy()[0, 5])
+    # request 1 has finite inputs: its results are the oracle's
+    ref = O.in_llm_request(w.Q[l:], w.K[k1:], w.V[k1:], w.hidden[k1:], w.n_keep_heads, 16)
+    np.testing.assert_array_equal(heads[1], ref["heads"])

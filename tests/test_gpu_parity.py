@@ -83,7 +83,11 @@ def test_full_size_workloads(make):
     w = make()
     tally, _ = _run_and_check(w)
     print(f"\n{w.name}: {tally}")
-    assert tally.stage1_exact >= w.B - max(1, w.B // 8)
+    # near ties are checked by the band rule; their number stays small on these inputs
+    bound = max(1, w.B // 8)
+    assert tally.stage1_near_ties <= bound and tally.stage2_near_ties <= bound, (
+        f"{w.name}: {tally.stage1_near_ties} stage-1 and {tally.stage2_near_ties} stage-2 near ties "
+        f"of {w.B} requests (bound {bound})")
 
 
 @pytest.mark.parametrize("k1", [192, 128, 64])
@@ -95,7 +99,7 @@ def test_llava15_batch32_sweep(k1, k2):
         w = copy.copy(base)
         w.reqs = [synth.Request(r.n, r.m, r.k1, ratio, r.l, r.k2) for r in base.reqs]
         tally, _ = _run_and_check(w)
-        assert tally.stage1_exact >= w.B - 2
+        assert tally.stage1_near_ties <= 2 and tally.stage2_near_ties <= 2, f"ratio {ratio}: {tally}"
 
 
 def test_fused_full_size():
