@@ -188,6 +188,11 @@ TREVS_API trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride
  *    g < Hkv, i < K1. Query head h reads key head floor(h*Hkv/Hq) (grouped-query attention).
  * The attention A^h[q, i] = softmax over the K1 visual keys of (Q_h[q] . K_g[i]) * scale,
  * scale = softmax_scale if > 0 else 1/sqrt(d_h) (Sec. 4.2).
+ * Full-sequence variant (optional): lse_other[h, q] is the natural log of
+ * sum_j exp((Q_h[q] . k_j) * scale) over the keys of row q that are not visual (system and
+ * text tokens, as the LLM's own softmax spans them). When given, the denominator of row (h, q)
+ * also counts that mass, so the row sums to less than 1, and Eq. 8 takes the variance about
+ * the row's own mean (its visual mass / K1). -inf means no other mass (the plain softmax).
  * attn [Hq][L][K1] float32 (dense): A^h[q, i] at attn[(h*L + q)*K1 + i].
  */
 
@@ -195,12 +200,14 @@ TREVS_API trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride
 TREVS_API size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1);
 
 /* Eq. 8: u_out[h] = (1/L) sum_q Var_i A^h[q, i] (population variance over the K1 keys), and
- * the attention probabilities in attn_out (layout above). Limits: d_h == TREVS_HEAD_DIM,
- * 1 <= K1 <= TREVS_MAX_STAGE2_TOKENS, 1 <= Hq <= TREVS_MAX_HEADS, Hq % Hkv == 0, L >= 1. */
+ * the attention probabilities in attn_out (layout above). lse_other (NULL: plain softmax over
+ * the visual keys) is the full-sequence variant above, [Hq][L] float32, element (h, q) at
+ * lse_other[h*L + q]. Limits: d_h == TREVS_HEAD_DIM, 1 <= K1 <= TREVS_MAX_STAGE2_TOKENS,
+ * 1 <= Hq <= TREVS_MAX_HEADS, Hq % Hkv == 0, L >= 1. */
 TREVS_API trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
                                       const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
                                       int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
-                                      float softmax_scale, float* u_out, float* attn_out,
+                                      float softmax_scale, const float* lse_other, float* u_out, float* attn_out,
                                       void* workspace, size_t workspace_bytes, void* stream);
 
 /* H* = the n_keep_heads heads of largest u (ties to the lower head), written ascending to
@@ -212,6 +219,19 @@ TREVS_API trevs_status trevs_in_llm_select(const float* u, const float* attn, in
                                  int32_t n_keep_heads, int32_t K2, int32_t* heads_out,
                                  float* p_out, int32_t* kept_local,
                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* Eq. 1 (Sec. 3.2), textual sensitivity of every head, a diagnostic of how much a head's
+ * visual attention moves with the question: for two questions about the same K1 visual tokens,
+ * attn1 [Hq][L1][K1] and attn2 [Hq][L2][K1] (float32, the layout trevs_in_llm_head_scores
+ * writes), s_h^(x) = (1/L_x) sum_q A_x^h[q, :] and
+ *   ts_out[h] = 1 - cos(s_h^(1), s_h^(2))   (a zero distribution has cosine 0).
+ * s1_out / s2_out [Hq][K1] (either may be NULL) receive the head-mean distributions. Workspace:
+ * trevs_textual_sensitivity_workspace_size(Hq, K1) bytes, zero-filled before first use (its
+ * tickets reset themselves). Limits: Hq <= 65535. */
+TREVS_API size_t trevs_textual_sensitivity_workspace_size(int32_t Hq, int32_t K1);
+TREVS_API trevs_status trevs_textual_sensitivity(const float* attn1, int32_t L1, const float* attn2, int32_t L2,
+                                       int32_t Hq, int32_t K1, float* ts_out, float* s1_out, float* s2_out,
+                                       void* workspace, size_t workspace_bytes, void* stream);
 
 /* Allocation-free form of trevs_in_llm_select: the same H*, Eq. 9 scores and TopK(p, K2),
  * with the same arguments except the workspace. The paper has no counterpart; this is for
@@ -308,6 +328,10 @@ typedef struct trevs_in_batch {
   uint16_t* K_out;                 /* [.., sum k2 rows] with (out_head_stride, out_tok_stride) */
   uint16_t* V_out;
   int64_t out_head_stride, out_tok_stride;
+  const float* lse_other;          /* optional full-sequence variant (see stage 2 above): element
+                                      (h, row) at lse_other + h*lse_head_stride + row*lse_row_stride,
+                                      rows packed like Q's (NULL: plain softmax over the visual keys) */
+  int64_t lse_head_stride, lse_row_stride;
 } trevs_in_batch;
 
 TREVS_API size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch);

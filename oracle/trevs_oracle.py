@@ -11,7 +11,7 @@ building blocks and no blocking, fusion or reordering. Inputs arrive as
 bfloat16 bit patterns (uint16) or float32 and are widened exactly to float64.
 
 Readings where the paper is silent or leaves a choice open:
-  * A zero-norm vector has cosine 0 with everything (Eq. 4 divides by the norm).
+  * A zero-norm vector has cosine 0 with everything (Eq. 4 divides by the norm; Eq. 1 alike).
   * Med is the lower median: the ascending element of rank floor((N-1)/2) (Eq. 6).
   * epsilon of Eq. 6 defaults to 1e-6.
   * Textual-ratio selection (Sec. 3.1): K_t = floor(r*K1 + 0.5) textual tokens,
@@ -262,12 +262,12 @@ def head_visual_attention(A: np.ndarray) -> np.ndarray:
 
 def textual_sensitivity(s1: np.ndarray, s2: np.ndarray) -> np.ndarray:
     """Eq. 1: TS_h = 1 - cos(s_h^(1), s_h^(2)) for the distributions of every head under two
-    questions; s1 and s2 are [Hq, K1]. Returns [Hq]."""
+    questions; s1 and s2 are [Hq, K1]. Returns [Hq]. A zero vector has cosine 0 (as for Eq. 4)."""
     s1 = np.asarray(s1, dtype=np.float64)
     s2 = np.asarray(s2, dtype=np.float64)
     num = (s1 * s2).sum(axis=1)
     den = np.sqrt((s1 * s1).sum(axis=1)) * np.sqrt((s2 * s2).sum(axis=1))
-    return 1.0 - num / den
+    return 1.0 - np.divide(num, den, out=np.zeros_like(num), where=den > 0)
 
 
 def head_variance(A: np.ndarray) -> np.ndarray:
@@ -330,11 +330,12 @@ def pre_llm_request(Z_bits, T_bits, s_v, k1, ratio, mode="ratio", tau_v=1.4, tau
     return out
 
 
-def in_llm_request(Q_bits, K_bits, V_bits, hidden_bits, n_keep_heads, k2, scale=None):
-    """Stage 2 for one request: attention, Eq. 8 variance, H*, Eq. 9 scores, top-K2, compaction."""
+def in_llm_request(Q_bits, K_bits, V_bits, hidden_bits, n_keep_heads, k2, scale=None, lse_other=None):
+    """Stage 2 for one request: attention, Eq. 8 variance, H*, Eq. 9 scores, top-K2, compaction.
+    lse_other [Hq, L] selects the full-sequence softmax variant of Sec. 4.2."""
     Q = bf16_bits_to_f64(Q_bits)
     K = bf16_bits_to_f64(K_bits)
-    A = text_to_vision_attention(Q, K, scale)
+    A = text_to_vision_attention(Q, K, scale, lse_other)
     u = head_variance(A)
     heads = select_heads(u, n_keep_heads)
     p = token_scores(A, heads)
@@ -360,9 +361,10 @@ def run_workload(w, mode="ratio", stage1=True, stage2=True, requests=None, **par
                 w.Z[n_off[b]:n_off[b + 1]], w.T[m_off[b]:m_off[b + 1]],
                 w.s_v[n_off[b]:n_off[b + 1]], r.k1, r.ratio, mode, **params)
         if stage2:
+            lse = getattr(w, "lse_other", None)
             res["in"] = in_llm_request(
                 w.Q[l_off[b]:l_off[b + 1]], w.K[k1_off[b]:k1_off[b + 1]],
                 w.V[k1_off[b]:k1_off[b + 1]], w.hidden[k1_off[b]:k1_off[b + 1]],
-                w.n_keep_heads, r.k2)
+                w.n_keep_heads, r.k2, lse_other=None if lse is None else lse[:, l_off[b]:l_off[b + 1]])
         out.append(res)
     return out

@@ -551,6 +551,9 @@ trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
                     bt->hidden_out_row_stride >= bt->d_model && bt->hidden_out_row_stride % 8 == 0,
                 "hidden strides must be >= d_model and multiples of 8");
   }
+  if (bt->lse_other)
+    TREVS_CHECK(bt->lse_head_stride >= 0 && bt->lse_row_stride >= 0 && ((uintptr_t)bt->lse_other & 3u) == 0,
+                "lse_other must be 4-byte aligned with non-negative strides");
   if (bt->K_out || bt->V_out) {
     TREVS_CHECK(bt->K_out == nullptr || aligned16(bt->K_out), "K_out must be 16-byte aligned");
     TREVS_CHECK(bt->V_out == nullptr || (aligned16(bt->V) && aligned16(bt->V_out)), "V tensors must be 16-byte aligned");
@@ -650,6 +653,11 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + L.cnt_ts);
   a.hs_finalize = 1;
   a.zero_p = 1;
+  if (bt->lse_other) {
+    a.lse = bt->lse_other + l_base * bt->lse_row_stride;
+    a.lse_hs = bt->lse_head_stride;
+    a.lse_rs = bt->lse_row_stride;
+  }
   a.overlap = overlap ? 1 : 0;
   a.independent = independent ? 1 : 0;
   if (in_small_fits(bt->Hq, max_l, max_k1)) {
@@ -1033,7 +1041,7 @@ size_t trevs_in_llm_workspace_size(int32_t Hq, int32_t L, int32_t K1) {
 trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, int64_t q_tok_stride,
                                       const uint16_t* K, int64_t k_head_stride, int64_t k_tok_stride,
                                       int32_t Hq, int32_t Hkv, int32_t L, int32_t K1, int32_t d_h,
-                                      float softmax_scale, float* u_out, float* attn_out,
+                                      float softmax_scale, const float* lse_other, float* u_out, float* attn_out,
                                       void* workspace, size_t workspace_bytes, void* stream) {
   g_launches = 0;
   trevs_status s = validate_in_common(Hq, Hkv, d_h, 1);
@@ -1066,6 +1074,8 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + W.cnt_ts);
   a.hs_finalize = 1; a.zero_p = 0;
+  TREVS_CHECK(lse_other == nullptr || ((uintptr_t)lse_other & 3u) == 0, "lse_other must be 4-byte aligned");
+  a.lse = lse_other; a.lse_hs = L; a.lse_rs = 1;
   TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, K1, (cudaStream_t)stream)), "head_stats launch");
   return TREVS_OK;
 }

@@ -116,16 +116,22 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
   // row statistics, TPR threads per row (all rows of the chunk in parallel)
   constexpr int TPR = 128 / QC;
   __shared__ float s_inv[64];
+  __shared__ float s_mean[64];
   const int k1 = r.k1;
-  const float mean = 1.0f / (float)k1;
   {
     const int rr = tid / TPR, sub = tid % TPR;
     float* row = lg + rr * k1_ld;
+    // full-sequence variant: the row's non-visual mass joins the denominator (log2 units)
+    float other = -INFINITY;
+    if (a.lse && q0 + rr < r.l)
+      other = __ldg(a.lse + (long long)h * a.lse_hs + (long long)(r.l_off + q0 + rr) * a.lse_rs) *
+              1.4426950408889634f;
     float mx = -INFINITY;
 #pragma unroll 4
     for (int i = sub; i < k1; i += TPR) mx = fmaxf(mx, row[i]);
 #pragma unroll
     for (int o = 1; o < TPR; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    mx = fmaxf(mx, other);
     float sum = 0.f;
 #pragma unroll 4
     for (int i = sub; i < k1; i += TPR) {
@@ -135,16 +141,22 @@ __global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constan
     }
 #pragma unroll
     for (int o = 1; o < TPR; o <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (sub == 0) s_inv[rr] = 1.0f / sum;
+    if (sub == 0) {
+      const float tot = sum + exp2f(other - mx);   // + 0 without the variant
+      s_inv[rr] = 1.0f / tot;
+      // Eq. 8 takes the variance about the row's mean: 1 / K1, or its visual mass / K1
+      s_mean[rr] = a.lse ? (sum / tot) / (float)k1 : 1.0f / (float)k1;
+    }
   }
   __syncthreads();
   // A[h][q][i] = e / sum, written along i by whole warps, and the two-pass variance of the
-  // row about its mean 1/K1 (Eq. 8)
+  // row about its mean (Eq. 8)
   {
     const int rows = min(QC, r.l - q0);
     float* A = a.attn + r.attn_off + ((long long)h * r.l + q0) * k1;
     for (int rr = warp; rr < rows; rr += 4) {
       const float inv = s_inv[rr];
+      const float mean = s_mean[rr];
       const float* row = lg + rr * k1_ld;
       float* out = A + (long long)rr * k1;
       float v = 0.f;
@@ -352,8 +364,14 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
     for (int ch = 0; ch < NCH; ++ch) qk_tile<NT>(af, ks_a + ch * 64 * kRowBytes, 0, lane, acc[ch]);
   }
   const float sc = a.scale * 1.4426950408889634f;       // logits in log2 units
-  const float mean = 1.0f / (float)K1;
   const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
+  // full-sequence variant: the non-visual mass of rows ra, rb joins their denominators
+  float oa = -INFINITY, ob = -INFINITY;
+  if (a.lse) {
+    const float* lr = a.lse + (long long)h * a.lse_hs + (long long)r.l_off * a.lse_rs;
+    if (ra < L) oa = __ldg(lr + (long long)ra * a.lse_rs) * 1.4426950408889634f;
+    if (rb < L) ob = __ldg(lr + (long long)rb * a.lse_rs) * 1.4426950408889634f;
+  }
   float mxa = -INFINITY, mxb = -INFINITY;
 #pragma unroll
   for (int ch = 0; ch < NCH; ++ch)
@@ -372,6 +390,8 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
     mxa = fmaxf(mxa, __shfl_xor_sync(0xffffffffu, mxa, o));
     mxb = fmaxf(mxb, __shfl_xor_sync(0xffffffffu, mxb, o));
   }
+  mxa = fmaxf(mxa, oa);
+  mxb = fmaxf(mxb, ob);
   float sa = 0.f, sb = 0.f;
 #pragma unroll
   for (int ch = 0; ch < NCH; ++ch)
@@ -392,7 +412,11 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
     sa += __shfl_xor_sync(0xffffffffu, sa, o);
     sb += __shfl_xor_sync(0xffffffffu, sb, o);
   }
-  const float ia = 1.0f / sa, ib = 1.0f / sb;
+  const float ta = sa + exp2f(oa - mxa), tb = sb + exp2f(ob - mxb);   // + 0 without the variant
+  const float ia = 1.0f / ta, ib = 1.0f / tb;
+  // Eq. 8 takes the variance about each row's mean: 1 / K1, or its visual mass / K1
+  const float mean_a = a.lse ? (sa * ia) / (float)K1 : 1.0f / (float)K1;
+  const float mean_b = a.lse ? (sb * ib) / (float)K1 : 1.0f / (float)K1;
   float* A = a.attn + r.attn_off + (long long)h * L * K1;
   float* Aa = A + (long long)ra * K1;
   float* Ab = A + (long long)rb * K1;
@@ -408,12 +432,12 @@ __global__ void __launch_bounds__(128) in_attn_small_kernel(const __grid_constan
       const float pa0 = acc[ch][nt][0] * ia, pa1 = acc[ch][nt][1] * ia;
       const float pb0 = acc[ch][nt][2] * ib, pb1 = acc[ch][nt][3] * ib;
       if (key < K1) {
-        va = fmaf(pa0 - mean, pa0 - mean, va);
-        vb = fmaf(pb0 - mean, pb0 - mean, vb);
+        va = fmaf(pa0 - mean_a, pa0 - mean_a, va);
+        vb = fmaf(pb0 - mean_b, pb0 - mean_b, vb);
       }
       if (key + 1 < K1) {
-        va = fmaf(pa1 - mean, pa1 - mean, va);
-        vb = fmaf(pb1 - mean, pb1 - mean, vb);
+        va = fmaf(pa1 - mean_a, pa1 - mean_a, va);
+        vb = fmaf(pb1 - mean_b, pb1 - mean_b, vb);
       }
       if (pairs) {
         if (key < K1) {

@@ -64,7 +64,8 @@ class InBatchC(ctypes.Structure):
                 ("hidden", _vp), ("hidden_row_stride", _c_i64),
                 ("u", _vp), ("heads", _vp), ("p", _vp), ("kept_local", _vp),
                 ("hidden_out", _vp), ("hidden_out_row_stride", _c_i64),
-                ("K_out", _vp), ("V_out", _vp), ("out_head_stride", _c_i64), ("out_tok_stride", _c_i64)]
+                ("K_out", _vp), ("V_out", _vp), ("out_head_stride", _c_i64), ("out_tok_stride", _c_i64),
+                ("lse_other", _vp), ("lse_head_stride", _c_i64), ("lse_row_stride", _c_i64)]
 
 
 _SIGS = {
@@ -88,9 +89,12 @@ _SIGS = {
                                    _vp, _c_sz, _vp]),
     "trevs_in_llm_workspace_size": (_c_sz, [_c_i32, _c_i32, _c_i32]),
     "trevs_in_llm_head_scores": (_c_i32, [_vp, _c_i64, _c_i64, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
-                                          _c_i32, _c_i32, _c_i32, _c_f32, _vp, _vp, _vp, _c_sz, _vp]),
+                                          _c_i32, _c_i32, _c_i32, _c_f32, _vp, _vp, _vp, _vp, _c_sz, _vp]),
     "trevs_in_llm_select": (_c_i32, [_vp, _vp, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp,
                                      _vp, _c_sz, _vp]),
+    "trevs_textual_sensitivity_workspace_size": (_c_sz, [_c_i32, _c_i32]),
+    "trevs_textual_sensitivity": (_c_i32, [_vp, _c_i32, _vp, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp, _vp, _c_sz,
+                                           _vp]),
     "trevs_in_llm_select_noalloc": (_c_i32, [_vp, _vp, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _vp, _vp, _vp,
                                              _vp]),
     "trevs_in_llm_compact": (_c_i32, [_vp, _c_i64, _c_i32, _vp, _vp, _c_i64, _c_i64, _c_i32, _c_i32,
@@ -245,11 +249,12 @@ def trevs_pre_llm_fps(Z, pivots, K_d, picks, pick_dist=None, pool=0, ws=None, st
 
 
 def trevs_in_llm_head_scores(Q, K, Hq, Hkv, L, K1, u_out, attn_out, q_strides, k_strides,
-                             scale=0.0, ws=None, stream=None):
+                             scale=0.0, ws=None, stream=None, lse_other=None):
+    """lse_other: optional [Hq, L] float32 (contiguous), the full-sequence softmax variant."""
     w, nb = _ws_args(ws)
     check(load().trevs_in_llm_head_scores(_ptr(Q), q_strides[0], q_strides[1], _ptr(K), k_strides[0],
-                                          k_strides[1], Hq, Hkv, L, K1, HEAD_DIM, scale, _ptr(u_out),
-                                          _ptr(attn_out), w, nb, _stream(stream)))
+                                          k_strides[1], Hq, Hkv, L, K1, HEAD_DIM, scale, _ptr(lse_other),
+                                          _ptr(u_out), _ptr(attn_out), w, nb, _stream(stream)))
 
 
 def trevs_in_llm_select(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=None, p_out=None, ws=None,
@@ -257,6 +262,17 @@ def trevs_in_llm_select(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=No
     w, nb = _ws_args(ws)
     check(load().trevs_in_llm_select(_ptr(u), _ptr(attn), Hq, L, K1, n_keep, K2, _ptr(heads_out), _ptr(p_out),
                                      _ptr(kept_local), w, nb, _stream(stream)))
+
+
+def trevs_textual_sensitivity(attn1, attn2, ts_out, s1_out=None, s2_out=None, ws=None, stream=None):
+    """Eq. 1 for attention tensors [Hq, L1, K1] and [Hq, L2, K1] (float32, contiguous)."""
+    Hq, L1, K1 = attn1.shape
+    L2 = attn2.shape[1]
+    if ws is None:
+        ws = workspace(load().trevs_textual_sensitivity_workspace_size(Hq, K1))
+    w, nb = _ws_args(ws)
+    check(load().trevs_textual_sensitivity(_ptr(attn1), L1, _ptr(attn2), L2, Hq, K1, _ptr(ts_out), _ptr(s1_out),
+                                           _ptr(s2_out), w, nb, _stream(stream)))
 
 
 def trevs_in_llm_select_noalloc(u, attn, Hq, L, K1, n_keep, K2, kept_local, heads_out=None, p_out=None,
@@ -320,6 +336,7 @@ class InBatch:
     heads: object = None       # [B, n_keep] i32
     p: object = None           # [sum k1] f32
     softmax_scale: float = 0.0
+    lse_other: object = None   # [Hq, sum l] f32: full-sequence softmax variant (Sec. 4.2)
 
     def c(self):
         arr = (InRequest * max(1, len(self.reqs)))(*[InRequest(int(a), int(b), int(c)) for a, b, c in self.reqs])
@@ -335,7 +352,9 @@ class InBatch:
             _ptr(self.u), _ptr(self.heads), _ptr(self.p), _ptr(self.kept_local),
             _ptr(self.hidden_out), self.hidden_out.stride(0) if self.hidden_out is not None else 0,
             _ptr(self.K_out), _ptr(self.V_out),
-            ko.stride(1) if ko is not None else 0, ko.stride(0) if ko is not None else 0)
+            ko.stride(1) if ko is not None else 0, ko.stride(0) if ko is not None else 0,
+            _ptr(self.lse_other), self.lse_other.stride(0) if self.lse_other is not None else 0,
+            self.lse_other.stride(1) if self.lse_other is not None else 0)
 
 
 def trevs_pre_llm_varlen_workspace_size(pre: PreBatch) -> int:

@@ -159,8 +159,9 @@ def check_workload(w, g: DeviceRun, ref, mode="ratio", tally: Tally | None = Non
                 # H* may differ inside the band; Eq. 9 is then checked over the GPU's own H*
                 assert len(heads) == w.n_keep_heads and np.all(np.diff(heads) > 0), f"req {b}: bad H*"
                 check_band(heads, inn["u"], w.n_keep_heads, None, f"req {b} H*")
+                lse = None if w.lse_other is None else w.lse_other[:, l_off[b]:l_off[b + 1]]
                 A = O.text_to_vision_attention(O.bf16_bits_to_f64(w.Q[l_off[b]:l_off[b + 1]]),
-                                               O.bf16_bits_to_f64(w.K[k1_off[b]:k1_off[b + 1]]))
+                                               O.bf16_bits_to_f64(w.K[k1_off[b]:k1_off[b + 1]]), lse_other=lse)
                 p_ref = O.token_scores(A, heads)
             else:
                 np.testing.assert_array_equal(heads, inn["heads"], err_msg=f"req {b} heads")

@@ -520,6 +520,8 @@ def pin_textual_sensitivity():
     a, b = rng.random((4, 9)), rng.random((4, 9))
     _close(O.textual_sensitivity(a, 3.0 * b), O.textual_sensitivity(a, b))          # scale
     _close(O.textual_sensitivity(a, b), O.textual_sensitivity(b, a))                # symmetric
+    # a zero distribution has cosine 0 with anything (the reading of Eq. 4 carried over)
+    _close(O.textual_sensitivity(np.zeros((1, 3)), np.array([[0.2, 0.3, 0.5]])), [1.0])
 
 
 def pin_head_visual_attention():

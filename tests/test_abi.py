@@ -141,7 +141,7 @@ def test_cls_saliency_validation(lib):
 def test_stage2_validation(lib):
     def hs(Hq, Hkv, L, K1, dh):
         return lib.trevs_in_llm_head_scores(FAKE, 4096, 128, FAKE, 8192, 128, Hq, Hkv, L, K1, dh, 0.0,
-                                            FAKE, FAKE, FAKE, 1 << 24, None)
+                                            None, FAKE, FAKE, FAKE, 1 << 24, None)
     assert hs(32, 5, 32, 64, 128) == t.TREVS_ERR_INVALID_ARGUMENT      # Hq % Hkv
     assert hs(32, 32, 32, 64, 64) == t.TREVS_ERR_UNSUPPORTED           # d_h
     assert hs(32, 32, 32, 4096, 128) == t.TREVS_ERR_UNSUPPORTED        # K1 beyond the limit
@@ -255,3 +255,14 @@ def test_in_varlen_validation(lib):
     assert tot >= lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(pre)) + need
     assert lib.trevs_prune_varlen(ctypes.byref(pre), None, ctypes.byref(ok), FAKE, tot - 256,
                                   None) == t.TREVS_ERR_WORKSPACE
+
+
+def test_textual_sensitivity_validation(lib):
+    ts = lib.trevs_textual_sensitivity
+    need = lib.trevs_textual_sensitivity_workspace_size(28, 1024)
+    assert need > 0 and lib.trevs_textual_sensitivity_workspace_size(0, 5) == 0
+    assert ts(FAKE, 4, FAKE, 4, 0, 10, FAKE, None, None, FAKE, need, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert ts(FAKE, 0, FAKE, 4, 2, 10, FAKE, None, None, FAKE, need, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert ts(None, 4, FAKE, 4, 2, 10, FAKE, None, None, FAKE, need, None) == t.TREVS_ERR_INVALID_ARGUMENT
+    assert ts(FAKE, 4, FAKE, 4, 28, 1024, FAKE, None, None, FAKE, need - 1, None) == t.TREVS_ERR_WORKSPACE
+    assert ts(FAKE, 4, FAKE, 4, 28, 1024, FAKE, None, None, None, need, None) == t.TREVS_ERR_WORKSPACE

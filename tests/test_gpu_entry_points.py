@@ -224,3 +224,23 @@ def test_stage2_nan_u_stays_in_bounds(path):
     # request 1 has finite inputs: its results are the oracle's
     ref = O.in_llm_request(w.Q[l:], w.K[k1:], w.V[k1:], w.hidden[k1:], w.n_keep_heads, 16)
     np.testing.assert_array_equal(heads[1], ref["heads"])
+
+
+@pytest.mark.parametrize("k1,l", [(64, 32), (700, 20)])
+def test_single_request_head_scores_full_sequence(k1, l):
+    """trevs_in_llm_head_scores with lse_other: u and the attention against the oracle's
+    full-sequence variant; rows then sum to less than 1."""
+    w = synth.small_case(seed_cfg=130 + l, n=(k1,), m=(l,), d=64, hq=8, hkv=4, n_keep_heads=2,
+                         k1=(k1,), ratio=(0.5,), k2=(8,))
+    w = synth.with_full_sequence_softmax(w, seed=5)
+    Q, K = H.dev_bf16(w.Q), H.dev_bf16(w.K)
+    lse = H.dev_f32(w.lse_other)
+    ws = T.workspace(T.load().trevs_in_llm_workspace_size(w.hq, l, k1))
+    u = torch.zeros(w.hq, dtype=torch.float32, device="cuda")
+    attn = torch.zeros((w.hq, l, k1), dtype=torch.float32, device="cuda")
+    T.trevs_in_llm_head_scores(Q, K, w.hq, w.hkv, l, k1, u, attn, (128, w.hq * 128), (128, w.hkv * 128), ws=ws,
+                               lse_other=lse)
+    A = O.text_to_vision_attention(O.bf16_bits_to_f64(w.Q), O.bf16_bits_to_f64(w.K), lse_other=w.lse_other)
+    assert A.sum(axis=2).max() < 1.0
+    H.assert_close(attn.cpu().numpy(), A, H.RTOL, H.ATOL_P, "attention")
+    H.assert_close(u.cpu().numpy(), O.head_variance(A), H.RTOL, 1e-9, "u")

@@ -77,8 +77,11 @@ def test_deterministic_repeat():
 
 
 @pytest.mark.parametrize("make", [synth.llava15_single, synth.llava_next_batch8, synth.long_video_batch2,
-                                  synth.ragged_serving_batch64],
-                         ids=["llava15_576", "llava_next_2880_b8", "long_16384_gqa", "ragged_b64"])
+                                  synth.ragged_serving_batch64, synth.video_llava_batch,
+                                  lambda: synth.with_full_sequence_softmax(synth.video_llava_batch()),
+                                  lambda: synth.with_full_sequence_softmax(synth.llava15_single())],
+                         ids=["llava15_576", "llava_next_2880_b8", "long_16384_gqa", "ragged_b64",
+                              "video_llava_2048_b4", "video_llava_2048_b4_fullseq", "llava15_576_fullseq"])
 def test_full_size_workloads(make):
     w = make()
     tally, _ = _run_and_check(w)
@@ -105,3 +108,15 @@ def test_llava15_batch32_sweep(k1, k2):
 def test_fused_full_size():
     w = synth.llava_next_batch8()
     _run_and_check(w, "fused")
+
+
+@pytest.mark.parametrize("k1,l", [(40, 9), (128, 64), (300, 33), (1024, 128)])
+def test_full_sequence_softmax_stage2(k1, l):
+    """The Sec. 4.2 variant whose rows also count the non-visual keys' mass, on both stage-2
+    paths (small: L <= 64 and K1 <= 128), against the oracle's variant."""
+    w = synth.small_case(seed_cfg=120 + l, n=(k1 + 3, k1), m=(l, max(1, l // 3)), d=64, hq=8, hkv=2,
+                         n_keep_heads=3, k1=(k1, k1), ratio=(0.5, 0.5), k2=(k1 // 3, k1 // 2))
+    w = synth.with_full_sequence_softmax(w, seed=k1)
+    g, _ = H.run_gpu(w, stages="in")
+    tally = H.check_workload(w, g, O.run_workload(w, stage1=False))
+    assert tally.stage2_near_ties <= 1, tally

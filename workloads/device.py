@@ -74,7 +74,8 @@ def build_batches(w, mode=T.SELECT_RATIO, dev=None):
         V_out=torch.zeros((max(sum_k2, 1), w.hkv, w.dh), dtype=torch.bfloat16, device="cuda"),
         u=torch.zeros((w.B, w.hq), dtype=torch.float32, device="cuda"),
         heads=torch.full((w.B, w.n_keep_heads), -1, dtype=torch.int32, device="cuda"),
-        p=torch.zeros(max(sum_k1, 1), dtype=torch.float32, device="cuda"))
+        p=torch.zeros(max(sum_k1, 1), dtype=torch.float32, device="cuda"),
+        lse_other=None if w.lse_other is None else dev.get("lse_other", dev_f32(w.lse_other)))
     return pre, inb
 
 

@@ -62,6 +62,7 @@ class Workload:
     V: np.ndarray
     hidden: np.ndarray
     planted: list = dataclasses.field(default_factory=list)
+    lse_other: np.ndarray | None = None   # [hq, sum L] float32: full-sequence softmax variant
 
     @property
     def B(self) -> int:
@@ -230,6 +231,29 @@ def cls_inputs(n, heads=16, dh=64, seed=77, spikes=8):
             K[off + idx] += 4.0 * u[None, :, :]
         off += nb
     return f32_to_bf16_bits(q.astype(np.float32)), f32_to_bf16_bits(K.astype(np.float32))
+
+
+def with_full_sequence_softmax(w, seed=7, system_tokens=35):
+    """A copy of `w` with lse_other [hq, sum L] (float32): for text row q of a request, the log
+    of the summed exp-logits of the keys a causal LLM row also attends to besides the visual
+    ones (`system_tokens` system-prompt keys and the text keys up to q). Those logits are drawn
+    with the spread of the row's own visual logits, sigma = ||Q_h[q]|| / sqrt(dh), and the first
+    system key gets sigma * 4 + 2 more (the usual attention sink)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    Q = w.Q.astype(np.uint32) << np.uint32(16)
+    Qf = Q.view(np.float32).astype(np.float64)                     # [sum L, hq, dh]
+    sigma = np.sqrt((Qf * Qf).sum(axis=2)) / math.sqrt(w.dh)        # [sum L, hq]
+    lse = np.empty((w.hq, Qf.shape[0]), dtype=np.float64)
+    l_off = w.offsets("l")
+    for b in range(w.B):
+        for q in range(w.reqs[b].l):
+            row = l_off[b] + q
+            n_o = system_tokens + q + 1
+            x = rng.standard_normal((w.hq, n_o)) * sigma[row][:, None]
+            x[:, 0] += 4.0 * sigma[row] + 2.0
+            m = x.max(axis=1)
+            lse[:, row] = m + np.log(np.exp(x - m[:, None]).sum(axis=1))
+    return dataclasses.replace(w, name=w.name + "_fullseq", lse_other=lse.astype(np.float32))
 
 
 WORKLOADS = {
