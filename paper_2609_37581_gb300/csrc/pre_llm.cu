@@ -32,11 +32,13 @@ namespace trevs {
 // in the next grid.
 //
 // Operands, all by TMA in 128-byte swizzled rows. Z: one box per 8 rows (3D map, S slices of
-// 8 rows) or, when every request starts on an 8-row boundary, per 32 rows (4D map over
-// 8-row groups); either way a tile's slice c lies at c KB within each 8-row group of S KB,
-// which the UMMA descriptor states as its stride between 8-row groups. T: its own ring of
-// slots of TS slices (TS divides S), boxes of 8 rows, laid out the same way. A partial last
-// slice (d' not a multiple of 64) comes slice by slice from 2D maps that fill zeros beyond d'.
+// 8 rows; 512 contiguous bytes of each row for S = 4) or, for two tiles per stage (256 bytes
+// of each row) on 8-row boundaries, per 32 rows (4D map over 8-row groups), which streams as
+// well; either way a tile's slice c lies at c KB within each 8-row group of S KB, which the
+// UMMA descriptor states as its stride between 8-row groups. A partial last slice (d' not a
+// multiple of 64) comes slice by slice from a 2D map that fills zeros beyond d'. T: its own
+// ring of slots of TS slices (TS divides S); each slice is one 2D box of the request's M
+// rounded up to 16, 32, 64, 128 or 256 rows (zeros beyond d').
 //
 // Warp roles: 0 = Z producer, 1 = TMEM owner and MMA issuer, 2 = T producer, 4..7 =
 // epilogue (warp w reads TMEM lanes 32*(w%4) .. +31), 8..15 = Z norms (G = 1: two threads
@@ -52,6 +54,14 @@ constexpr int kZNormWarps = 8;
 constexpr int kRingBudget = 216 * 1024;        // the Z and T rings (dynamic shared memory)
 constexpr int kZ4Rows = 32;                    // rows per Z box from the 4D map
 
+constexpr int kTMaps = 5;   // T boxes of 16, 32, 64, 128 or 256 rows by one slice
+
+// The tensor maps of T, one per box height; a request's slices come from the lowest box that
+// holds its M rounded up to 16 rows.
+struct TMaps {
+  CUtensorMap m[kTMaps];
+};
+
 struct ScoreLaunch {
   int G;              // tiles per group and per Z stage (1 or 2)
   int S;              // 64-column slices per Z stage (4 / G)
@@ -59,7 +69,7 @@ struct ScoreLaunch {
   int z_stages;       // Z ring depth
   int t_slots;        // T ring depth
   int t_slot_slices;  // slices per T slot (TS, divides S)
-  int tn;             // T rows per slot slice: the largest M of the launch rounded up to 16
+  int tn;             // T rows per slot slice: the largest M of the launch rounded up to a power of two
   int acc_cols;       // TMEM columns of one tile's accumulator (power of two >= 32 and >= tn)
   int mld;            // row length of a partial G (max M rounded up to 4)
   int z4;             // Z from the 4D map in boxes of 32 rows
@@ -144,9 +154,8 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* tmap, int 
 template <bool kSeed>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     pre_score_kernel(const __grid_constant__ CUtensorMap tmZ3, const __grid_constant__ CUtensorMap tmZ2,
-                     const __grid_constant__ CUtensorMap tmZ4, const __grid_constant__ CUtensorMap tmT3,
-                     const __grid_constant__ CUtensorMap tmT2, const __grid_constant__ PreMeta meta, const PreArgs a,
-                     const ScoreLaunch L) {
+                     const __grid_constant__ CUtensorMap tmZ4, const __grid_constant__ TMaps tmT,
+                     const __grid_constant__ PreMeta meta, const PreArgs a, const ScoreLaunch L) {
   using namespace sm100;
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t zfull[kMaxZStages], zempty[kMaxZStages];
@@ -161,12 +170,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t zbase = smem_u32(smem);
   const int SZ = L.z_stages, ST = L.t_slots, TS = L.t_slot_slices, G = L.G, S = L.S;
-  const int t_slot_bytes = TS * L.tn * 128;
+  const int t_slice_bytes = L.tn * 128;
+  const int t_slot_bytes = TS * t_slice_bytes;
   const uint32_t tbase = zbase + SZ * kZStageBytes;   // after the Z stages
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int d = a.d;
   const int nk = (d + kChunk - 1) / kChunk;           // 64-column slices
-  const int full_slices = d / kChunk;                 // slices the 3D and 4D maps cover
+  const int full_slices = d / kChunk;                 // slices the 3D and 4D Z maps cover
   const long long W = (long long)meta.total_tiles * L.nst, P = gridDim.x;
   const long long w0 = W * blockIdx.x / P, w1 = W * (blockIdx.x + 1) / P;
   const int tile_bytes = kTileRows * S * 128;         // one tile's share of a Z stage
@@ -254,8 +264,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     }
   } else if (warp == 2) {
     if (lane == 0) {
-      tma_prefetch_desc(&tmT3);
-      tma_prefetch_desc(&tmT2);
+      for (int i = 0; i < kTMaps; ++i) tma_prefetch_desc(&tmT.m[i]);
       const uint64_t pt = l2_policy_evict_last();   // T is read again by every tile of its request
       int gt = 0;
       SegWalk walk(meta, L.nst, w0, w1);
@@ -263,7 +272,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       bool ok = true;
       while (ok && walk.next(meta, L, sg)) {
         const PreReq& r = meta.r[sg.b];
-        const int nb = ((r.m + 15) & ~15) / 8;       // 8-row boxes the request's MMAs read
+        int mi = 0;                                  // the lowest box holding M rounded up to 16
+        while ((16 << mi) < r.m && mi + 1 < kTMaps) ++mi;
+        const uint32_t box_bytes = (uint32_t)(16 << mi) * 128;
         for (int s = sg.s0; ok && s < sg.s1; ++s) {
           const int k0 = s * S, ns = min(S, nk - k0);
           for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
@@ -276,15 +287,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
             const uint32_t B = tbase + ts * t_slot_bytes;
             const uint32_t fb = smem_u32(&tfull[ts]);
             const int kc = k0 + c0, nsl = min(TS, ns - c0);
-            if (kc + nsl > full_slices) {
-              mbar_arrive_expect_tx(fb, (uint32_t)(nb * nsl * 1024));
-              for (int rb = 0; rb < nb; ++rb)
-                for (int c = 0; c < nsl; ++c)
-                  tma_load_2d(B + rb * TS * 1024 + c * 1024, &tmT2, (kc + c) * kChunk, r.m_off + rb * 8, fb, pt);
-            } else {
-              mbar_arrive_expect_tx(fb, (uint32_t)(nb * TS * 1024));
-              for (int rb = 0; rb < nb; ++rb) tma_load_3d(B + rb * TS * 1024, &tmT3, 0, r.m_off + rb * 8, kc, fb, pt);
-            }
+            mbar_arrive_expect_tx(fb, (uint32_t)nsl * box_bytes);
+            for (int c = 0; c < nsl; ++c) tma_load_2d(B + c * t_slice_bytes, &tmT.m[mi], (kc + c) * kChunk, r.m_off, fb, pt);
             s_tissued = gt + 1;
           }
         }
@@ -330,7 +334,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 #pragma unroll
                 for (int k = 0; k < kChunk / 16; ++k)
                   umma_bf16(dt, umma_desc_sw128(A + g * tile_bytes + (c0 + c) * 1024 + 32 * k, S * 1024),
-                            umma_desc_sw128(B + c * 1024 + 32 * k, TS * 1024), idesc,
+                            umma_desc_sw128(B + c * t_slice_bytes + 32 * k), idesc,
                             (s != sg.s0 || c0 + c != 0 || k != 0) ? 1u : 0u);
               }
             }
@@ -773,14 +777,14 @@ static ScorePlan score_plan(const PreMeta& meta, const PreArgs& a, int max_m) {
   ScorePlan p;
   ScoreLaunch& L = p.L;
   const int nk = (a.d + kChunk - 1) / kChunk;
-  L.tn = (max_m + 15) & ~15;                  // the MMA reads M rounded up to 16 rows
-  int cols = 32;
-  while (cols < L.tn) cols <<= 1;
-  L.acc_cols = cols;
+  // T rows per slot slice: the tallest box a request of the launch takes (its M rounded up to
+  // a power of two, at least 16), which the MMA's N (M rounded up to 16) never exceeds
+  L.tn = 16;
+  while (L.tn < max_m) L.tn <<= 1;
+  L.acc_cols = L.tn < 32 ? 32 : L.tn;
   L.mld = (max_m + 3) & ~3;
   bool rows8 = true;                          // every request's rows start on an 8-row boundary
   for (int b = 0; b < meta.B; ++b) rows8 = rows8 && (meta.r[b].n % 8 == 0);
-  L.z4 = rows8 ? 1 : 0;
   // grid: one CTA per SM (less the SMs left to concurrent work), at least four G = 1 stages each
   const long long W1 = (long long)meta.total_tiles * ((nk + 3) / 4);
   long long P = sm_count() - (a.score_reserve > 0 ? a.score_reserve : 0);
@@ -794,6 +798,7 @@ static ScorePlan score_plan(const PreMeta& meta, const PreArgs& a, int max_m) {
   L.G = (4 * L.acc_cols <= 512 && rows8 && meta.total_tiles >= (7 * p.P) / 4) ? 2 : 1;
   L.S = 4 / L.G;
   L.nst = (nk + L.S - 1) / L.S;
+  L.z4 = L.G == 2 ? 1 : 0;
   // rings: two Z stages and T slots of S slices when two of them fit, else narrower T slots;
   // a third Z stage when two stages' worth of T slots still fit beside it
   const int slice = L.tn * 128;
@@ -840,19 +845,18 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   if (meta.total_tiles == 0) return cudaSuccess;
   const ScorePlan p = score_plan(meta, a, max_m);
   const ScoreLaunch& L = p.L;
-  CUtensorMap tmZ3, tmZ2, tmZ4, tmT3, tmT2;
+  CUtensorMap tmZ3, tmZ2, tmZ4;
+  TMaps tmT;
   cudaError_t e = make_tmap_sliced(&tmZ3, a.Z, z_rows, a.d, a.z_stride, 8, L.S);
   if (e == cudaSuccess) e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, 8);
   if (e == cudaSuccess && L.z4) e = make_tmap_rowgroups(&tmZ4, a.Z, z_rows, a.d, a.z_stride, L.S, kZ4Rows / 8);
   if (e == cudaSuccess && !L.z4) tmZ4 = tmZ3;   // not read
-  if (e == cudaSuccess) e = make_tmap_sliced(&tmT3, a.T, a.total_m, a.d, a.t_stride, 8, L.t_slot_slices);
-  if (e == cudaSuccess) e = make_tmap(&tmT2, a.T, a.total_m, a.d, a.t_stride, 8);
+  for (int i = 0; i < kTMaps && e == cudaSuccess; ++i) e = make_tmap(&tmT.m[i], a.T, a.total_m, a.d, a.t_stride, 16 << i);
   if (e != cudaSuccess) return e;
   auto kernel = a.action == kActFpsSeed ? pre_score_kernel<true> : pre_score_kernel<false>;
   e = ensure_dynamic_smem(kernel, p.smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(kernel, dim3(p.P), dim3(kScoreThreads), p.smem, st, pdl, tmZ3, tmZ2, tmZ4, tmT3, tmT2, meta,
-                       a, L);
+  return launch_kernel(kernel, dim3(p.P), dim3(kScoreThreads), p.smem, st, pdl, tmZ3, tmZ2, tmZ4, tmT, meta, a, L);
 }
 
 // Finishing grid after the scoring grid launched just before it (same meta, d' and max M;
