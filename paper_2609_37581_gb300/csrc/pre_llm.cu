@@ -10,48 +10,52 @@ namespace trevs {
 // A persistent grid, one CTA per SM, scores the visual rows of every request against the M
 // text rows of that request. Each request is cut into tiles of 128 rows (its last tile may
 // be shorter) and the tiles into groups of G consecutive tiles (G = 1 or 2 per launch; a
-// request's last group may hold fewer). A Z stage is 64 KB: the G tiles of a group over
-// S = 4 / G slices of 64 columns, so a group takes nst = ceil(slices / S) stages. Work is
-// counted in tile-stages: the stage of a group of g' tiles weighs g', the launch weighs
-// W = tiles * nst, and CTA c owns the stages whose start falls in [W c / P, W (c + 1) / P), so
-// every CTA streams the same number of Z bytes (stream-K). A group whose stages are split
-// between CTAs leaves partial sums of G and ||z||^2 in the workspace (at most two segments
-// per CTA: where its range starts and where it ends), and pre_finish_kernel adds them up in
-// stage order.
+// request's last group may hold fewer). A group stage covers S = 4 / G slices of 64 columns
+// of its tiles (64 KB of Z), so a group takes nst = ceil(slices / S) stages. Work is counted
+// in tile-stages: the stage of a group of g' tiles weighs g', the launch weighs W = tiles *
+// nst, and CTA c owns the stages whose start falls in [W c / P, W (c + 1) / P), so every CTA
+// streams the same number of Z bytes (stream-K). A group whose stages are split between
+// CTAs leaves partial sums of G and ||z||^2 in the workspace (at most two segments per CTA:
+// where its range starts and where it ends), and pre_finish_kernel adds them up in stage
+// order.
 //
-// Each stage's slices of T serve the G tiles of the stage, so the SM takes in T once per G
-// tiles: the SM's intake (about 55 GB/s) is shared by Z from HBM and T from L2, and with
-// M = 128 text rows T is as large as Z per tile.
+// Z arrives in sub-stages of 32 KB: one tile's 128 rows over a pair of slices (256
+// contiguous bytes of each row), each with its own barriers, in a ring of four to six. The
+// tensor cores start on a sub-stage as soon as it lands and release it about 0.25 us later,
+// so the SM keeps well over 100 KB of Z in flight (with 64 KB stages, two in a ring, the
+// wait for their MMAs held the rate far below the HBM share). The slices of T for a pair
+// serve the G tiles of the group: the SM takes in T once per G tiles (its intake, about
+// 55 GB/s, is shared by Z from HBM and T from L2, and with M = 128 text rows T is as large
+// as Z per tile).
 //
 // For each group the 5th-generation tensor cores compute G = Z_tile . T^T per tile (UMMA
 // M = 128, N = M_b rounded up to 16) into G TMEM accumulators (two buffers of G), while eight
-// warps sum the squares ||z_i||^2 from the same shared-memory stages. Four epilogue warps
+// warps sum the squares ||z_i||^2 from the same shared-memory sub-stages. Four epilogue warps
 // read a finished group's accumulators while the next group streams into the other buffer,
 // and form m_ji = max(G_ji / (||t_j|| ||z_i||), 0) and s^t_i = sqrt(sum_j m_ji^2 / M) with
 // 1 / ||t_j|| from the pre-pass; the [M, N] similarity never reaches memory. Selection runs
 // in the next grid.
 //
-// Operands, all by TMA in 128-byte swizzled rows. Z: one box per 8 rows (3D map, S slices of
-// 8 rows; 512 contiguous bytes of each row for S = 4) or, for two tiles per stage (256 bytes
-// of each row) on 8-row boundaries, per 32 rows (4D map over 8-row groups), which streams as
-// well; either way a tile's slice c lies at c KB within each 8-row group of S KB, which the
-// UMMA descriptor states as its stride between 8-row groups. A partial last slice (d' not a
-// multiple of 64) comes slice by slice from a 2D map that fills zeros beyond d'. T: its own
-// ring of slots of TS slices (TS divides S); each slice is one 2D box of the request's M
-// rounded up to 16, 32, 64, 128 or 256 rows (zeros beyond d').
+// Operands, all by TMA in 128-byte swizzled rows. Z: boxes of 32 rows x two slices from a 4D
+// map over 8-row groups when every request starts on an 8-row boundary, else of 8 rows from
+// a 3D map; either way slice c of a sub-stage lies at c KB within each 8-row group of 2 KB,
+// which the UMMA descriptor states as its stride between 8-row groups. A partial last slice
+// (d' not a multiple of 64) comes slice by slice from a 2D map that fills zeros beyond d'.
+// T: its own ring of slots of one or two slices; each slice is the request's M rounded up to
+// 16 rows, as boxes of 256, 128, 64, 32 and 16 rows from 2D maps (zeros beyond d').
 //
 // Warp roles: 0 = Z producer, 1 = TMEM owner and MMA issuer, 2 = T producer, 4..7 =
-// epilogue (warp w reads TMEM lanes 32*(w%4) .. +31), 8..15 = Z norms (G = 1: two threads
-// per row, two slices each; G = 2: one thread per row of the two tiles).
+// epilogue (warp w reads TMEM lanes 32*(w%4) .. +31), 8..15 = Z norms (a thread per row and
+// slice of each sub-stage).
 
 constexpr int kTileRows = kScoreTileRows;
 constexpr int kChunk = 64;                     // d' columns per slice (one 128-byte swizzle row)
-constexpr int kZStageBytes = 64 * 1024;        // Z bytes per stage
-constexpr int kMaxZStages = 3;
+constexpr int kSubBytes = 32 * 1024;           // one Z sub-stage: a tile's 128 rows x two slices
+constexpr int kMaxZSubs = 6;
 constexpr int kMaxTSlots = 8;
 constexpr int kScoreThreads = 512;
 constexpr int kZNormWarps = 8;
-constexpr int kRingBudget = 216 * 1024;        // the Z and T rings (dynamic shared memory)
+constexpr int kRingBudget = 208 * 1024;        // the Z and T rings (dynamic shared memory)
 constexpr int kZ4Rows = 32;                    // rows per Z box from the 4D map
 
 constexpr int kTMaps = 5;   // T boxes of 16, 32, 64, 128 or 256 rows by one slice
@@ -63,16 +67,16 @@ struct TMaps {
 };
 
 struct ScoreLaunch {
-  int G;              // tiles per group and per Z stage (1 or 2)
-  int S;              // 64-column slices per Z stage (4 / G)
-  int nst;            // Z stages per group: ceil(slices / S)
-  int z_stages;       // Z ring depth
+  int G;              // tiles per group (1 or 2)
+  int S;              // 64-column slices per group stage (4 / G): G * S / 2 sub-stages of 32 KB
+  int nst;            // stages per group: ceil(slices / S)
+  int z_subs;         // Z ring depth in sub-stages
   int t_slots;        // T ring depth
-  int t_slot_slices;  // slices per T slot (TS, divides S)
+  int t_slot_slices;  // slices per T slot (2, or 1 for tall T)
   int tn;             // T rows per slot slice: the largest M of the launch rounded up to a power of two
   int acc_cols;       // TMEM columns of one tile's accumulator (power of two >= 32 and >= tn)
   int mld;            // row length of a partial G (max M rounded up to 4)
-  int z4;             // Z from the 4D map in boxes of 32 rows
+  int z4;             // Z from the 4D map in boxes of 32 rows (every request on 8-row boundaries)
 };
 
 // Floats of one tile's partial sums: G [128][mld], then ||z||^2 [128]; a slot holds G tiles.
@@ -158,32 +162,31 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
                      const __grid_constant__ PreMeta meta, const PreArgs a, const ScoreLaunch L) {
   using namespace sm100;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t zfull[kMaxZStages], zempty[kMaxZStages];
+  __shared__ __align__(8) uint64_t zfull[kMaxZSubs], zempty[kMaxZSubs];
   __shared__ __align__(8) uint64_t tfull[kMaxTSlots], tempty[kMaxTSlots];
   __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], norm_full[2], norm_empty[2];
   __shared__ uint32_t tmem_base_s;
-  __shared__ float rinv_s[4][256];   // one row per epilogue warp (no cross-warp barrier)
-  __shared__ float zsq_s[2][2][kTileRows];   // [buffer][tile (G = 2) or column half (G = 1)][row]
+  __shared__ float rinv_s[4][256];              // one row per epilogue warp (no cross-warp barrier)
+  __shared__ float zsq_s[2][2][2][kTileRows];   // [buffer][tile][slice of the pair][row]
   __shared__ volatile int s_abort;
   __shared__ volatile int s_zissued, s_tissued;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t zbase = smem_u32(smem);
-  const int SZ = L.z_stages, ST = L.t_slots, TS = L.t_slot_slices, G = L.G, S = L.S;
+  const int NZ = L.z_subs, ST = L.t_slots, TS = L.t_slot_slices, G = L.G, S = L.S;
   const int t_slice_bytes = L.tn * 128;
   const int t_slot_bytes = TS * t_slice_bytes;
-  const uint32_t tbase = zbase + SZ * kZStageBytes;   // after the Z stages
+  const uint32_t tbase = zbase + NZ * kSubBytes;      // after the Z sub-stages
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int d = a.d;
   const int nk = (d + kChunk - 1) / kChunk;           // 64-column slices
   const int full_slices = d / kChunk;                 // slices the 3D and 4D Z maps cover
   const long long W = (long long)meta.total_tiles * L.nst, P = gridDim.x;
   const long long w0 = W * blockIdx.x / P, w1 = W * (blockIdx.x + 1) / P;
-  const int tile_bytes = kTileRows * S * 128;         // one tile's share of a Z stage
   const long long tf = score_tile_floats(L.mld);
 
   if (tid == 0) {
-    for (int s = 0; s < SZ; ++s) {
+    for (int s = 0; s < NZ; ++s) {
       mbar_init(smem_u32(&zfull[s]), 1);
       mbar_init(smem_u32(&zempty[s]), 1 + kZNormWarps);   // MMA commit + the Z-norm warps
     }
@@ -212,6 +215,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   const uint32_t tmem = tmem_base_s;
   pdl_launch_dependents();   // the selection grid may start launching
 
+  // A group's stage s covers slices [s S, s S + ns); its sub-stages, in order, are the slice
+  // pairs h of the stage and, within a pair, the tiles g of the group: one tile x two slices.
   if (warp == 0) {
     if (lane == 0) {
       tma_prefetch_desc(L.z4 ? &tmZ4 : &tmZ3);
@@ -223,42 +228,39 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       bool ok = true;
       while (ok && walk.next(meta, L, sg)) {
         const PreReq& r = meta.r[sg.b];
-        for (int s = sg.s0; s < sg.s1; ++s, ++gz) {
-          const int st = gz % SZ, ph = gz / SZ;
-          if (gz >= SZ && !mbar_wait(smem_u32(&zempty[st]), (ph - 1) & 1, &s_abort)) {
-            s_abort = 1;
-            ok = false;
-            break;
-          }
-          const uint32_t A = zbase + st * kZStageBytes;
-          const uint32_t fb = smem_u32(&zfull[st]);
-          const int k0 = s * S;
-          const int ns = min(S, nk - k0);
-          const bool ragged = k0 + ns > full_slices;   // a partial slice: slice by slice from the 2D map
-          uint32_t bytes = 0;
-          for (int g = 0; g < sg.gp; ++g) {
-            const int h = sg.h[g];
-            if (ragged) bytes += (uint32_t)(((h + 7) / 8) * ns * 1024);
-            else if (L.z4) bytes += (uint32_t)(((h + kZ4Rows - 1) / kZ4Rows) * kZ4Rows * S * 128);
-            else bytes += (uint32_t)(((h + 7) / 8) * S * 1024);
-          }
-          mbar_arrive_expect_tx(fb, bytes);
-          for (int g = 0; g < sg.gp; ++g) {
-            const int h = sg.h[g];
-            const int y0 = r.n_off + sg.row0 + g * kTileRows;
-            const uint32_t At = A + g * tile_bytes;
-            if (ragged) {
-              for (int zb = 0; zb < (h + 7) / 8; ++zb)
-                for (int c = 0; c < ns; ++c)
-                  tma_load_2d(At + zb * S * 1024 + c * 1024, &tmZ2, (k0 + c) * kChunk, y0 + zb * 8, fb, pz);
-            } else if (L.z4) {
-              for (int i = 0; i < (h + kZ4Rows - 1) / kZ4Rows; ++i)
-                tma_load_4d(At + i * kZ4Rows * S * 128, &tmZ4, 0, 0, k0, (y0 >> 3) + i * (kZ4Rows / 8), fb, pz);
-            } else {
-              for (int zb = 0; zb < (h + 7) / 8; ++zb) tma_load_3d(At + zb * S * 1024, &tmZ3, 0, y0 + zb * 8, k0, fb, pz);
+        for (int s = sg.s0; ok && s < sg.s1; ++s) {
+          const int k0 = s * S, ns = min(S, nk - k0);
+          for (int hp = 0; ok && 2 * hp < ns; ++hp) {
+            const int kc = k0 + 2 * hp, nps = min(2, ns - 2 * hp);
+            const bool ragged = kc + nps > full_slices;   // a partial slice: slice by slice from the 2D map
+            for (int g = 0; g < sg.gp; ++g, ++gz) {
+              const int st = gz % NZ, ph = gz / NZ;
+              if (gz >= NZ && !mbar_wait(smem_u32(&zempty[st]), (ph - 1) & 1, &s_abort)) {
+                s_abort = 1;
+                ok = false;
+                break;
+              }
+              const uint32_t A = zbase + st * kSubBytes;
+              const uint32_t fb = smem_u32(&zfull[st]);
+              const int h = sg.h[g];
+              const int y0 = r.n_off + sg.row0 + g * kTileRows;
+              if (ragged) {
+                mbar_arrive_expect_tx(fb, (uint32_t)(((h + 7) / 8) * nps * 1024));
+                for (int zb = 0; zb < (h + 7) / 8; ++zb)
+                  for (int c = 0; c < nps; ++c)
+                    tma_load_2d(A + zb * 2048 + c * 1024, &tmZ2, (kc + c) * kChunk, y0 + zb * 8, fb, pz);
+              } else if (L.z4) {
+                const int nb = (h + kZ4Rows - 1) / kZ4Rows;
+                mbar_arrive_expect_tx(fb, (uint32_t)(nb * kZ4Rows * 2 * 128));
+                for (int i = 0; i < nb; ++i)
+                  tma_load_4d(A + i * kZ4Rows * 2 * 128, &tmZ4, 0, 0, kc, (y0 >> 3) + i * (kZ4Rows / 8), fb, pz);
+              } else {
+                mbar_arrive_expect_tx(fb, (uint32_t)(((h + 7) / 8) * 2048));
+                for (int zb = 0; zb < (h + 7) / 8; ++zb) tma_load_3d(A + zb * 2048, &tmZ3, 0, y0 + zb * 8, kc, fb, pz);
+              }
+              s_zissued = gz + 1;
             }
           }
-          s_zissued = gz + 1;
         }
       }
     }
@@ -272,24 +274,34 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       bool ok = true;
       while (ok && walk.next(meta, L, sg)) {
         const PreReq& r = meta.r[sg.b];
-        int mi = 0;                                  // the lowest box holding M rounded up to 16
-        while ((16 << mi) < r.m && mi + 1 < kTMaps) ++mi;
-        const uint32_t box_bytes = (uint32_t)(16 << mi) * 128;
+        const int np16 = (r.m + 15) & ~15;           // the rows of T the request's MMAs read
         for (int s = sg.s0; ok && s < sg.s1; ++s) {
           const int k0 = s * S, ns = min(S, nk - k0);
-          for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
-            const int ts = gt % ST, ph = gt / ST;
-            if (gt >= ST && !mbar_wait(smem_u32(&tempty[ts]), (ph - 1) & 1, &s_abort)) {
-              s_abort = 1;
-              ok = false;
-              break;
+          for (int hp = 0; ok && 2 * hp < ns; ++hp) {
+            const int kc = k0 + 2 * hp, nps = min(2, ns - 2 * hp);
+            const int nslots = TS == 2 ? 1 : nps;
+            for (int q = 0; q < nslots; ++q, ++gt) {
+              const int ts = gt % ST, ph = gt / ST;
+              if (gt >= ST && !mbar_wait(smem_u32(&tempty[ts]), (ph - 1) & 1, &s_abort)) {
+                s_abort = 1;
+                ok = false;
+                break;
+              }
+              const uint32_t B = tbase + ts * t_slot_bytes;
+              const uint32_t fb = smem_u32(&tfull[ts]);
+              const int c0 = TS == 2 ? 0 : q, c1 = TS == 2 ? nps : q + 1;
+              mbar_arrive_expect_tx(fb, (uint32_t)((c1 - c0) * np16 * 128));
+              for (int c = c0; c < c1; ++c) {
+                // np16 rows as boxes of 256, 128, 64, 32 and 16 rows, one after the other
+                for (int rr = 0, mi = kTMaps - 1; rr < np16; --mi) {
+                  if ((16 << mi) > np16 - rr) continue;
+                  tma_load_2d(B + (c - c0) * t_slice_bytes + rr * 128, &tmT.m[mi], (kc + c) * kChunk, r.m_off + rr, fb,
+                              pt);
+                  rr += 16 << mi;
+                }
+              }
+              s_tissued = gt + 1;
             }
-            const uint32_t B = tbase + ts * t_slot_bytes;
-            const uint32_t fb = smem_u32(&tfull[ts]);
-            const int kc = k0 + c0, nsl = min(TS, ns - c0);
-            mbar_arrive_expect_tx(fb, (uint32_t)nsl * box_bytes);
-            for (int c = 0; c < nsl; ++c) tma_load_2d(B + c * t_slice_bytes, &tmT.m[mi], (kc + c) * kChunk, r.m_off, fb, pt);
-            s_tissued = gt + 1;
           }
         }
       }
@@ -309,39 +321,41 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         tc_fence_after();
         const uint32_t dg = tmem + (uint32_t)(buf * G * L.acc_cols);
         const uint32_t idesc = umma_idesc_bf16(kTileRows, (meta.r[sg.b].m + 15) & ~15);
-        for (int s = sg.s0; s < sg.s1; ++s, ++gz) {
-          const int st = gz % SZ, ph = gz / SZ;
-          if (!mbar_wait(smem_u32(&zfull[st]), ph & 1, &s_abort)) {
-            s_abort = 1;
-            ok = false;
-            break;
-          }
-          const uint32_t A = zbase + st * kZStageBytes;
-          const int ns = min(S, nk - s * S);
-          for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
-            const int ts = gt % ST, tph = gt / ST;
-            if (!mbar_wait(smem_u32(&tfull[ts]), tph & 1, &s_abort)) {
+        for (int s = sg.s0; ok && s < sg.s1; ++s) {
+          const int k0 = s * S, ns = min(S, nk - k0);
+          for (int hp = 0; ok && 2 * hp < ns; ++hp) {
+            const int nps = min(2, ns - 2 * hp);
+            const int nslots = TS == 2 ? 1 : nps;
+            for (int q = 0; ok && q < nslots; ++q)
+              if (!mbar_wait(smem_u32(&tfull[(gt + q) % ST]), ((gt + q) / ST) & 1, &s_abort)) ok = false;
+            if (!ok) {
               s_abort = 1;
-              ok = false;
               break;
             }
-            tc_fence_after();
-            const uint32_t B = tbase + ts * t_slot_bytes;
-            const int nsl = min(TS, ns - c0);
-            for (int g = 0; g < sg.gp; ++g) {
+            for (int g = 0; g < sg.gp; ++g, ++gz) {
+              const int st = gz % NZ, ph = gz / NZ;
+              if (!mbar_wait(smem_u32(&zfull[st]), ph & 1, &s_abort)) {
+                s_abort = 1;
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t A = zbase + st * kSubBytes;
               const uint32_t dt = dg + (uint32_t)(g * L.acc_cols);
-              for (int c = 0; c < nsl; ++c) {
+              for (int c = 0; c < nps; ++c) {
+                const uint32_t B = TS == 2 ? tbase + (gt % ST) * t_slot_bytes + c * t_slice_bytes
+                                           : tbase + ((gt + c) % ST) * t_slot_bytes;
 #pragma unroll
                 for (int k = 0; k < kChunk / 16; ++k)
-                  umma_bf16(dt, umma_desc_sw128(A + g * tile_bytes + (c0 + c) * 1024 + 32 * k, S * 1024),
-                            umma_desc_sw128(B + c * t_slice_bytes + 32 * k), idesc,
-                            (s != sg.s0 || c0 + c != 0 || k != 0) ? 1u : 0u);
+                  umma_bf16(dt, umma_desc_sw128(A + c * 1024 + 32 * k, 2048), umma_desc_sw128(B + 32 * k), idesc,
+                            (s != sg.s0 || hp != 0 || c != 0 || k != 0) ? 1u : 0u);
               }
+              umma_commit(smem_u32(&zempty[st]));   // frees the Z sub-stage once these MMAs have read it
             }
-            umma_commit(smem_u32(&tempty[ts]));   // frees the T slot once these MMAs have read it
+            if (!ok) break;
+            for (int q = 0; q < nslots; ++q) umma_commit(smem_u32(&tempty[(gt + q) % ST]));   // and the T slots
+            gt += nslots;
           }
-          if (!ok) break;
-          umma_commit(smem_u32(&zempty[st]));      // and the Z stage
         }
         if (!ok) break;
         umma_commit(smem_u32(&acc_full[buf]));    // this group's accumulators are complete
@@ -349,48 +363,49 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       }
     }
   } else if (warp >= 8) {
-    // Z norms. G = 1: thread zt owns row zt % 128 and slices 2 (zt / 128), + 1 of every stage;
-    // G = 2: row zt % 128 of tile zt / 128, both slices of every stage.
+    // Z norms: thread zt owns row zt % 128 and slice zt / 128 of every sub-stage's pair
     const int zt = tid - 256;
-    const int row = zt & (kTileRows - 1), part = zt >> 7;
-    const int g = G == 1 ? 0 : part;
-    const int cbeg = G == 1 ? 2 * part : 0;
+    const int row = zt & (kTileRows - 1), cs = zt >> 7;
     int gz = 0, j = 0;
     SegWalk walk(meta, L.nst, w0, w1);
     Segment sg;
     bool ok = true;
     while (ok && walk.next(meta, L, sg)) {
       const int buf = j & 1, use = j >> 1;
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
-      const bool mine = g < sg.gp && row < sg.h[g];
-      for (int s = sg.s0; s < sg.s1; ++s, ++gz) {
-        const int st = gz % SZ, ph = gz / SZ;
-        if (!mbar_wait(smem_u32(&zfull[st]), ph & 1, &s_abort)) {
-          s_abort = 1;
-          ok = false;
-          break;
-        }
-        if (mine) {
-          const uint8_t* rowp = smem + st * kZStageBytes + g * tile_bytes + (row >> 3) * S * 1024 + (row & 7) * 128;
-          const int ncols = min(S * kChunk, d - s * S * kChunk);   // columns of this stage
-#pragma unroll
-          for (int c = cbeg; c < cbeg + 2; ++c) {
-#pragma unroll
-            for (int qq = 0; qq < 8; ++qq) {
-              if (c * kChunk + qq * 8 < ncols)   // d' is a multiple of 8: whole 16-byte pieces
-                bf16_sq_acc8(*reinterpret_cast<const uint4*>(rowp + c * 1024 + (swz(row, qq) << 4)), acc);
+      float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};   // tiles 0 and 1 of the group
+      for (int s = sg.s0; ok && s < sg.s1; ++s) {
+        const int k0 = s * S, ns = min(S, nk - k0);
+        for (int hp = 0; ok && 2 * hp < ns; ++hp) {
+          const int kc = k0 + 2 * hp, nps = min(2, ns - 2 * hp);
+          const int ncols = min(kChunk, d - (kc + cs) * kChunk);   // columns of this thread's slice
+          for (int g = 0; g < sg.gp; ++g, ++gz) {
+            const int st = gz % NZ, ph = gz / NZ;
+            if (!mbar_wait(smem_u32(&zfull[st]), ph & 1, &s_abort)) {
+              s_abort = 1;
+              ok = false;
+              break;
             }
+            if (cs < nps && row < sg.h[g]) {
+              const uint8_t* rowp = smem + st * kSubBytes + (row >> 3) * 2048 + cs * 1024 + (row & 7) * 128;
+#pragma unroll
+              for (int qq = 0; qq < 8; ++qq)
+                if (qq * 8 < ncols) {   // d' is a multiple of 8: whole 16-byte pieces
+                  const uint4 v = *reinterpret_cast<const uint4*>(rowp + (swz(row, qq) << 4));
+                  if (g == 0) bf16_sq_acc8(v, acc0); else bf16_sq_acc8(v, acc1);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&zempty[st]));
           }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&zempty[st]));
       }
       if (!ok) break;
       if (j >= 2 && !mbar_wait(smem_u32(&norm_empty[buf]), (use - 1) & 1, &s_abort)) {
         s_abort = 1;
         break;
       }
-      zsq_s[buf][part][row] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      zsq_s[buf][0][cs][row] = (acc0[0] + acc0[1]) + (acc0[2] + acc0[3]);
+      zsq_s[buf][1][cs][row] = (acc1[0] + acc1[1]) + (acc1[2] + acc1[3]);
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&norm_full[buf]));
       ++j;
@@ -418,11 +433,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         break;
       }
       tc_fence_after();
-      float out[2];
+      float out0 = 0.f, out1 = 0.f;
       for (int g = 0; g < sg.gp; ++g) {
         const uint32_t lane_base =
             tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * G * L.acc_cols) + (uint32_t)(g * L.acc_cols);
-        const float zsq = G == 1 ? zsq_s[buf][0][row] + zsq_s[buf][1][row] : zsq_s[buf][g][row];
+        const float zsq = zsq_s[buf][g][0][row] + zsq_s[buf][g][1][row];
         const float rz = zsq > 0.f ? 1.0f / sqrtf(zsq) : 0.f;
         float sum = 0.f, mx = -INFINITY;
         if (sg.slot < 0) {
@@ -441,7 +456,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
               }
             }
           }
-          out[g] = kSeed ? mx : sqrtf(sum / (float)m);
+          const float o = kSeed ? mx : sqrtf(sum / (float)m);
+          if (g == 0) out0 = o; else out1 = o;
         } else {
           // a group split between CTAs: leave this CTA's partial sums (G row, columns
           // 0 .. round_up(m, 4), and ||z||^2) of tile g in its slot for pre_finish_kernel
@@ -463,9 +479,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         mbar_arrive(smem_u32(&acc_empty[buf]));
         mbar_arrive(smem_u32(&norm_empty[buf]));
       }
-      if (sg.slot < 0)
-        for (int g = 0; g < sg.gp; ++g)
-          if (row < sg.h[g]) a.s_t[r.n_off + sg.row0 + g * kTileRows + row] = out[g];
+      if (sg.slot < 0) {
+        float* out = a.s_t + r.n_off + sg.row0 + row;
+        if (row < sg.h[0]) out[0] = out0;
+        if (sg.gp > 1 && row < sg.h[1]) out[kTileRows] = out1;
+      }
       ++j;
     }
   }
@@ -479,8 +497,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     if (tid == 0) {
       const volatile int no_abort = 0;
       const int zi = s_zissued, ti = s_tissued;
-      for (int x = zi - SZ > 0 ? zi - SZ : 0; x < zi; ++x)
-        mbar_wait(smem_u32(&zfull[x % SZ]), (x / SZ) & 1, &no_abort, 500000000ull);
+      for (int x = zi - NZ > 0 ? zi - NZ : 0; x < zi; ++x)
+        mbar_wait(smem_u32(&zfull[x % NZ]), (x / NZ) & 1, &no_abort, 500000000ull);
       for (int x = ti - ST > 0 ? ti - ST : 0; x < ti; ++x)
         mbar_wait(smem_u32(&tfull[x % ST]), (x / ST) & 1, &no_abort, 500000000ull);
       atomicOr(a.err, 1u);
@@ -798,25 +816,25 @@ static ScorePlan score_plan(const PreMeta& meta, const PreArgs& a, int max_m) {
   L.G = (4 * L.acc_cols <= 512 && rows8 && meta.total_tiles >= (7 * p.P) / 4) ? 2 : 1;
   L.S = 4 / L.G;
   L.nst = (nk + L.S - 1) / L.S;
-  L.z4 = L.G == 2 ? 1 : 0;
-  // rings: two Z stages and T slots of S slices when two of them fit, else narrower T slots;
-  // a third Z stage when two stages' worth of T slots still fit beside it
+  L.z4 = rows8 ? 1 : 0;
+  // rings: the deepest Z ring (in 32 KB sub-stages) beside a T ring of at least two slots
+  // and three slices (T comes from L2 and runs ahead by a pair or more), with T slots of two
+  // slices when that costs no Z depth, else of one
   const int slice = L.tn * 128;
-  L.z_stages = 2;
-  L.t_slot_slices = 1;
-  for (int ts = L.S; ts >= 1; ts >>= 1)
-    if ((kRingBudget - 2 * kZStageBytes) / (ts * slice) >= 2) {
-      L.t_slot_slices = ts;
-      break;
+  L.z_subs = 0;
+  for (int ts = 2; ts >= 1; --ts)
+    for (int nz = kMaxZSubs; nz >= 2; --nz) {
+      const int slots = (kRingBudget - nz * kSubBytes) / (ts * slice);
+      if (slots >= 2 && slots * ts >= 3) {
+        if (nz > L.z_subs) {
+          L.z_subs = nz;
+          L.t_slot_slices = ts;
+          L.t_slots = slots > kMaxTSlots ? kMaxTSlots : slots;
+        }
+        break;
+      }
     }
-  int slots = (kRingBudget - 2 * kZStageBytes) / (L.t_slot_slices * slice);
-  const int need3 = 2 * (L.S / L.t_slot_slices);
-  if ((kRingBudget - 3 * kZStageBytes) / (L.t_slot_slices * slice) >= need3) {
-    L.z_stages = 3;
-    slots = (kRingBudget - 3 * kZStageBytes) / (L.t_slot_slices * slice);
-  }
-  L.t_slots = slots > kMaxTSlots ? kMaxTSlots : slots;
-  p.smem = L.z_stages * kZStageBytes + L.t_slots * L.t_slot_slices * slice + 1024;
+  p.smem = L.z_subs * kSubBytes + L.t_slots * L.t_slot_slices * slice + 1024;
   return p;
 }
 
@@ -847,9 +865,9 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   const ScoreLaunch& L = p.L;
   CUtensorMap tmZ3, tmZ2, tmZ4;
   TMaps tmT;
-  cudaError_t e = make_tmap_sliced(&tmZ3, a.Z, z_rows, a.d, a.z_stride, 8, L.S);
+  cudaError_t e = make_tmap_sliced(&tmZ3, a.Z, z_rows, a.d, a.z_stride, 8, 2);
   if (e == cudaSuccess) e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, 8);
-  if (e == cudaSuccess && L.z4) e = make_tmap_rowgroups(&tmZ4, a.Z, z_rows, a.d, a.z_stride, L.S, kZ4Rows / 8);
+  if (e == cudaSuccess && L.z4) e = make_tmap_rowgroups(&tmZ4, a.Z, z_rows, a.d, a.z_stride, 2, kZ4Rows / 8);
   if (e == cudaSuccess && !L.z4) tmZ4 = tmZ3;   // not read
   for (int i = 0; i < kTMaps && e == cudaSuccess; ++i) e = make_tmap(&tmT.m[i], a.T, a.total_m, a.d, a.t_stride, 16 << i);
   if (e != cudaSuccess) return e;
