@@ -123,10 +123,9 @@ def test_full_sequence_softmax_stage2(k1, l):
 
 
 @pytest.mark.parametrize("d,m", [(200, (5, 17, 128, 64)), (512, (128, 100, 1, 33)), (576, (64, 64, 64, 64))])
-def test_two_tiles_per_stage(d, m):
-    """Requests on 8-row boundaries with about two tiles per scoring CTA take the layout with
-    two tiles per Z stage (one T stage for both): odd tile counts (a group of one tile), groups
-    split between CTAs, and a partial last slice of d'."""
+def test_tiles_split_between_scoring_ctas(d, m):
+    """Several 128-row tiles per scoring CTA, tiles split between CTAs, odd tile counts, text
+    lengths from 1 to 128 and a partial last slice of d'."""
     w = synth.small_case(seed_cfg=150 + d, n=(1000, 512, 1536, 264), m=m, d=d, k1=(100, 64, 200, 8),
                          ratio=(0.5, 0.25, 0.75, 1.0), k2=(0, 0, 0, 0))
     for mode in ("ratio", "fused"):
