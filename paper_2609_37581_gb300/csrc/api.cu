@@ -22,8 +22,9 @@ cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool 
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
 cudaError_t launch_cls_saliency(const ClsMeta&, const ClsArgs&, int dh, int max_n, cudaStream_t);
-cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_l, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
+cudaError_t launch_in_token_score_qk(const InMeta&, const InArgs&, int max_l, int max_k1, cudaStream_t);
 bool in_small_fits(int Hq, int max_l, int max_k1);
 cudaError_t launch_in_small(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
@@ -181,17 +182,20 @@ PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1
 }
 
 struct InWs {
-  size_t cnt_hs, cnt_ts, attn, row_var, u, p, keys, flags, end;
+  size_t cnt_hs, cnt_ts, attn, row_var, rstat, u, p, keys, flags, end;
 };
 
-// total_lk1 = sum over requests of l * k1 (attention probabilities per head).
-InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, int B) {
+// total_lk1 = sum over requests of l * k1 (attention probabilities per head), kept only for
+// the small path (`small`), whose two grids pass the probabilities through the workspace; the
+// larger path keeps each row's max and 1 / sum (rstat) and recomputes.
+InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, int B, bool small = true) {
   InWs w;
   size_t o = kStatusBytes;
   w.cnt_hs = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
-  w.attn = o;      o = al256(o + 4 * (size_t)Hq * (size_t)total_lk1);
+  w.attn = o;      o = al256(o + (small ? 4 * (size_t)Hq * (size_t)total_lk1 : 0));
   w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
+  w.rstat = o;     o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
   w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
   w.p = o;         o = al256(o + 4 * (size_t)total_k1);
   const size_t padded = (size_t)total_k1 + 4 * (size_t)kMaxChunk + 4;   // per-request 16-byte alignment
@@ -500,7 +504,7 @@ trevs_status run_pre_batch(const trevs_pre_batch* bt, const trevs_pre_params& pr
 
 struct InTotals {
   long long l = 0, k1 = 0, k2 = 0, lk1 = 0;
-  int max_k1 = 0;
+  int max_k1 = 0, max_l = 0;
 };
 
 trevs_status validate_in_common(int Hq, int Hkv, int d_h, int n_keep) {
@@ -537,6 +541,7 @@ trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
     TREVS_CHECK(r.k2 >= 0 && r.k2 <= r.k1, "request %d: k2 = %d outside [0, k1 = %d]", b, r.k2, r.k1);
     t.l += r.l; t.k1 += r.k1; t.k2 += r.k2; t.lk1 += (long long)r.l * r.k1;
     t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
+    t.max_l = r.l > t.max_l ? r.l : t.max_l;
   }
   TREVS_CHECK(t.l < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
   s = validate_qk(bt->Q, bt->q_head_stride, bt->q_tok_stride, bt->K, bt->kv_head_stride, bt->kv_tok_stride);
@@ -620,14 +625,14 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     max_l = q.l > max_l ? q.l : max_l;
   }
   // block counts per request: text chunks of the head-statistics and token-score grids
-  const int qc = stats_text_rows(max_k1);
+  const int qc = stats_rows(max_l);
   for (int b = b0; b < b1; ++b) {
     const trevs_in_request& q = bt->reqs[b];
     InReq& r = meta.r[b - b0];
     r.hs_off = hs;
     r.ts_off = ts;
     hs += bt->Hq * ((q.l + qc - 1) / qc);
-    ts += ((q.l + kScoreTextRows - 1) / kScoreTextRows) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
+    ts += ((q.l + qc - 1) / qc) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
   }
   meta.total_hs = hs;
   meta.total_ts = ts;
@@ -641,6 +646,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.scale = bt->softmax_scale > 0.f ? bt->softmax_scale : 1.0f / sqrtf((float)bt->d_h);
   a.attn = reinterpret_cast<float*>(ws + L.attn);
   a.row_var = reinterpret_cast<float*>(ws + L.row_var);
+  a.rstat = reinterpret_cast<float*>(ws + L.rstat);
   a.stats_ld = lo;
   a.u = (bt->u ? bt->u : reinterpret_cast<float*>(ws + L.u)) + (long long)b0 * bt->Hq;
   a.u_ld = bt->Hq;
@@ -664,8 +670,8 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
     ++g_launches;   // two grids
   } else {
-    TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
-    TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
+    TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_l, st)), "head_stats launch");
+    TREVS_TRY_CUDA(counted(launch_in_token_score_qk(meta, a, max_l, max_k1, st)), "token_score launch");
   }
   if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
     fill_compaction(gm, meta,
@@ -1059,7 +1065,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   static thread_local InMeta meta;
   meta.B = 1;
   meta.r[0] = InReq{0, 0, L, 0, K1, 0, 0, 0, 0};
-  meta.total_hs = Hq * ((L + stats_text_rows(K1) - 1) / stats_text_rows(K1));
+  meta.total_hs = Hq * ((L + stats_rows(L) - 1) / stats_rows(L));
   meta.total_ts = 0;
   InArgs a;
   memset(&a, 0, sizeof(a));
@@ -1068,7 +1074,9 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.Hq = Hq; a.Hkv = Hkv; a.n_keep = 1;
   a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
   a.attn = attn_out;
+  a.write_attn = 1;
   a.row_var = reinterpret_cast<float*>(ws + W.row_var);
+  a.rstat = reinterpret_cast<float*>(ws + W.rstat);
   a.stats_ld = L;
   a.u = u_out; a.u_ld = Hq;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
@@ -1076,7 +1084,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.hs_finalize = 1; a.zero_p = 0;
   TREVS_CHECK(lse_other == nullptr || ((uintptr_t)lse_other & 3u) == 0, "lse_other must be 4-byte aligned");
   a.lse = lse_other; a.lse_hs = L; a.lse_rs = 1;
-  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, K1, (cudaStream_t)stream)), "head_stats launch");
+  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, L, (cudaStream_t)stream)), "head_stats launch");
   return TREVS_OK;
 }
 
@@ -1178,12 +1186,16 @@ size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
   long long l = 0, k1 = 0, lk1 = 0;
+  int max_l = 0, max_k1 = 0;
   for (int b = 0; b < batch->B; ++b) {
     const long long lb = batch->reqs[b].l > 0 ? batch->reqs[b].l : 0;
     const long long kb = batch->reqs[b].k1 > 0 ? batch->reqs[b].k1 : 0;
     l += lb; k1 += kb; lk1 += lb * kb;
+    max_l = lb > max_l ? (int)lb : max_l;
+    max_k1 = kb > max_k1 ? (int)kb : max_k1;
   }
-  return in_ws(l, k1, lk1, batch->Hq > 0 ? batch->Hq : 0, batch->B).end;
+  const int Hq = batch->Hq > 0 ? batch->Hq : 0;
+  return in_ws(l, k1, lk1, Hq, batch->B, in_small_fits(Hq, max_l, max_k1)).end;
 }
 
 size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in) {
@@ -1235,7 +1247,7 @@ trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch, void* workspace, s
   InTotals t;
   trevs_status s = validate_in_batch(batch, t);
   if (s != TREVS_OK || batch->B == 0) return s;
-  const InWs L = in_ws(t.l, t.k1, t.lk1, batch->Hq, batch->B);
+  const InWs L = in_ws(t.l, t.k1, t.lk1, batch->Hq, batch->B, in_small_fits(batch->Hq, t.max_l, t.max_k1));
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_in_batch(batch, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -1257,7 +1269,8 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1, pre->d);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
-  const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
+  const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B,
+                       in->B > 0 && in_small_fits(in->Hq, ti.max_l, ti.max_k1));
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);
   s = check_ws(workspace, workspace_bytes, need);
   if (s != TREVS_OK) return s;
