@@ -25,6 +25,7 @@ cudaError_t launch_cls_saliency(const ClsMeta&, const ClsArgs&, int dh, int max_
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_l, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score_qk(const InMeta&, const InArgs&, int max_l, int max_k1, cudaStream_t);
+cudaError_t launch_in_head_stats_tc(const InMeta&, const InArgs&, cudaStream_t);
 bool in_small_fits(int Hq, int max_l, int max_k1);
 cudaError_t launch_in_small(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
@@ -606,7 +607,8 @@ void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden,
 // `merged`: gather jobs of stage 1 to launch together with the compaction.
 trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
                           long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st, bool overlap,
-                          GatherMeta* merged, bool launch_gather_here = true, bool independent = false) {
+                          GatherMeta* merged, bool launch_gather_here = true, bool independent = false,
+                          uint32_t* status = nullptr) {
   static thread_local InMeta meta;
   static thread_local GatherMeta gm_own;
   GatherMeta& gm = merged ? *merged : gm_own;
@@ -624,14 +626,15 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
     max_l = q.l > max_l ? q.l : max_l;
   }
-  // block counts per request: text chunks of the head-statistics and token-score grids
+  // block counts per request: the head-statistics grid takes 128 text rows per block (one
+  // per TMEM lane), the token-score grid stats_rows(max_l)
   const int qc = stats_rows(max_l);
   for (int b = b0; b < b1; ++b) {
     const trevs_in_request& q = bt->reqs[b];
     InReq& r = meta.r[b - b0];
     r.hs_off = hs;
     r.ts_off = ts;
-    hs += bt->Hq * ((q.l + qc - 1) / qc);
+    hs += bt->Hq * ((q.l + 127) / 128);
     ts += ((q.l + qc - 1) / qc) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
   }
   meta.total_hs = hs;
@@ -657,6 +660,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.flags = ws + L.flags;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + L.cnt_hs);
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + L.cnt_ts);
+  a.err = status ? status : reinterpret_cast<uint32_t*>(ws);
   a.hs_finalize = 1;
   a.zero_p = 1;
   if (bt->lse_other) {
@@ -670,7 +674,7 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
     ++g_launches;   // two grids
   } else {
-    TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_l, st)), "head_stats launch");
+    TREVS_TRY_CUDA(counted(launch_in_head_stats_tc(meta, a, st)), "head_stats launch");
     TREVS_TRY_CUDA(counted(launch_in_token_score_qk(meta, a, max_l, max_k1, st)), "token_score launch");
   }
   if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
@@ -722,11 +726,13 @@ int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const 
   return r;
 }
 
-trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st) {
+trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st,
+                          uint32_t* status = nullptr) {
   long long l_base = 0, k1_base = 0, k2_base = 0;
   for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
     const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
-    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st, false, nullptr);
+    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st, false, nullptr, true, false,
+                                  status);
     if (s != TREVS_OK) return s;
     for (int b = b0; b < b1; ++b) {
       l_base += bt->reqs[b].l; k1_base += bt->reqs[b].k1; k2_base += bt->reqs[b].k2;
@@ -1305,7 +1311,8 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
       s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork, nullptr, aux->stream,
                         reserve, &forked);
       if (s != TREVS_OK) return joined(s);
-      s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true);
+      s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true,
+                       reinterpret_cast<uint32_t*>(ws));
       return joined(s);
     }
     // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
@@ -1315,14 +1322,15 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
     if (s != TREVS_OK) return s;
     TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
     forked = true;
-    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true);
+    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true, false,
+                     reinterpret_cast<uint32_t*>(ws));
     return joined(s);
   }
   if (pre->B > 0) {
     s = run_pre_batch(pre, prm, ws, LP, st);
     if (s != TREVS_OK) return s;
   }
-  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, st);
+  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, st, reinterpret_cast<uint32_t*>(ws));
   return TREVS_OK;
 }
 

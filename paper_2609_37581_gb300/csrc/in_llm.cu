@@ -1,6 +1,7 @@
 // Stage 2 (in-LLM at layer l*, Sec. 4.2): text-to-vision attention statistics, head
 // variance (Eq. 8), high-variance head set H*, token scores (Eq. 9), TopK and compaction.
 #include "in_llm.cuh"
+#include "sm100.cuh"
 
 namespace trevs {
 
@@ -225,6 +226,231 @@ __global__ void __launch_bounds__(32 * NW) in_head_stats_kernel(const __grid_con
   }
   if (a.zero_p)
     for (int i = tid; i < K1; i += NTH) a.p_bits[r.k1_off + i] = 0u;
+}
+
+// ------------------------------------------------------------------ attention statistics on tcgen05
+//
+// Block (request, head h, 128 text rows): the 5th-generation tensor cores form the logits
+// S = Q_h . K_g^T of the block's rows (UMMA M = 128 rows, N = 128 keys, K = 128 dims) chunk by
+// chunk into a double-buffered TMEM accumulator, twice over the K1 keys: pass 1 for each row's
+// running max and sum of exp (online softmax; with the full-sequence variant the row's
+// non-visual mass joins at the end), pass 2 for the probabilities and the two-pass Eq. 8
+// variance about the row's mean. TMEM lane r holds text row r, so each epilogue thread owns a
+// whole row and its reductions need no shuffles. Q_h is copied once and K_g streams in
+// 128-key chunks through a two-stage ring (cp.async by one warp, into the 128-byte swizzled
+// K-major layout the UMMA descriptors state). Each row's max and 1 / sum go to the workspace
+// for the token scores. The last block of a request averages the row variances into u_h and
+// clears p.
+//
+// Warps: 0 = loader, 1 = TMEM owner and MMA issuer, 2..5 = epilogue (warp w reads TMEM lanes
+// 32*(w%4) .. +31, so the four cover the 128 rows).
+constexpr int kTcKeys = 128;                       // keys per chunk (UMMA N)
+constexpr int kTcThreads = 192;
+constexpr int kTcTileBytes = 128 * kRowBytes;      // 128 rows x 128 dims, two 64-dim slices
+constexpr int kTcStages = 2;
+constexpr int kTcSmem = (1 + kTcStages) * kTcTileBytes + 1024;
+
+// 16-byte pieces of `rows` rows (128 bf16 each) into a 128-byte swizzled, slice-major tile:
+// slice c (64 dims) of row r at c * rows * 128 + r * 128, piece q at (q ^ (r & 7)) * 16.
+__device__ __forceinline__ void load_rows_sw128(uint32_t dst, const __nv_bfloat16* base, long long row_stride,
+                                                int row0, int rows, int valid, int lane) {
+  for (int idx = lane; idx < rows * 16; idx += 32) {
+    const int rr = idx >> 4, p = idx & 15, c = p >> 3, q = p & 7;
+    const bool ok = row0 + rr < valid;
+    const void* src = ok ? (const void*)(base + (long long)(row0 + rr) * row_stride + p * 8) : (const void*)base;
+    cp_async16(dst + c * rows * 128 + rr * 128 + (swz(rr, q) << 4), src, ok ? 16 : 0);
+  }
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1) in_head_stats_tc_kernel(const __grid_constant__ InMeta meta,
+                                                                          const InArgs a) {
+  using namespace sm100;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t qfull, kfull[kTcStages], kempty[kTcStages];
+  __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
+  __shared__ uint32_t tmem_base_s;
+  __shared__ volatile int s_abort;
+  __shared__ int s_last;
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t qs = smem_u32(smem), ks = qs + kTcTileBytes;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
+  const InReq r = meta.r[b];
+  const int nqc = (r.l + 127) / 128;
+  const int t = blockIdx.x - r.hs_off;
+  const int h = t / nqc, qc = t - h * nqc;
+  const int g = (h * a.Hkv) / a.Hq;
+  const int q0 = qc * 128;
+  const int K1 = r.k1, L = r.l, nkc = (K1 + kTcKeys - 1) / kTcKeys;
+  const int nj = 2 * nkc;                          // pass 1 and pass 2 over the key chunks
+
+  if (tid == 0) {
+    mbar_init(smem_u32(&qfull), 32);
+    for (int s = 0; s < kTcStages; ++s) {
+      mbar_init(smem_u32(&kfull[s]), 32);          // the loader's lanes, once their copies land
+      mbar_init(smem_u32(&kempty[s]), 1);          // MMA commit
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&acc_full[i]), 1);
+      mbar_init(smem_u32(&acc_empty[i]), 4);       // the epilogue warps
+    }
+    s_abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&tmem_base_s), 2 * kTcKeys);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  if (!a.overlap && !a.independent) pdl_wait();   // Q, K may come from the preceding grid
+  pdl_launch_dependents();
+
+  if (warp == 0) {
+    const __nv_bfloat16* Qb = a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs;
+    const __nv_bfloat16* Kb = a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs;
+    load_rows_sw128(qs, Qb, a.q_ts, q0, 128, L, lane);
+    cp_async_arrive_noinc(smem_u32(&qfull));
+    for (int j = 0; j < nj; ++j) {
+      const int s = j % kTcStages, ph = j / kTcStages;
+      if (j >= kTcStages && !mbar_wait(smem_u32(&kempty[s]), (ph - 1) & 1, &s_abort)) {
+        s_abort = 1;
+        break;
+      }
+      const int kc = j < nkc ? j : j - nkc;
+      load_rows_sw128(ks + s * kTcTileBytes, Kb, a.k_ts, kc * kTcKeys, kTcKeys, K1, lane);
+      cp_async_arrive_noinc(smem_u32(&kfull[s]));
+    }
+    cp_async_wait_all();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(128, kTcKeys);
+      bool ok = mbar_wait(smem_u32(&qfull), 0, &s_abort);
+      for (int j = 0; ok && j < nj; ++j) {
+        const int s = j % kTcStages, ph = j / kTcStages, buf = j & 1, use = j >> 1;
+        if (!mbar_wait(smem_u32(&kfull[s]), ph & 1, &s_abort)) ok = false;
+        if (ok && j >= 2 && !mbar_wait(smem_u32(&acc_empty[buf]), (use - 1) & 1, &s_abort)) ok = false;
+        if (!ok) break;
+        fence_proxy_async_smem();   // the stages were written by cp.async (generic proxy)
+        tc_fence_after();
+        const uint32_t kst = ks + s * kTcTileBytes, dt = tmem + (uint32_t)(buf * kTcKeys);
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(dt, umma_desc_sw128(qs + c * kTcTileBytes / 2 + 32 * k),
+                      umma_desc_sw128(kst + c * kTcTileBytes / 2 + 32 * k), idesc, (c | k) != 0 ? 1u : 0u);
+        umma_commit(smem_u32(&kempty[s]));   // frees the K stage once these MMAs have read it
+        umma_commit(smem_u32(&acc_full[buf]));
+      }
+      if (!ok) s_abort = 1;
+    }
+  } else {
+    const int q = warp & 3, row = 32 * q + lane;   // TMEM lane quarter; the block's text row
+    const int rq = q0 + row;                       // request-local text row
+    const float sc = a.scale * kLog2e;            // logits in log2 units
+    float m = -INFINITY, ssum = 0.f, inv = 0.f, mean = 0.f, var = 0.f;
+    for (int j = 0; j < nj; ++j) {
+      const int buf = j & 1, use = j >> 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[buf]), use & 1, &s_abort) && !s_abort);
+      if (!ok) {
+        s_abort = 1;
+        break;
+      }
+      tc_fence_after();
+      const int kc = j < nkc ? j : j - nkc;
+      const int nv = min(kTcKeys, K1 - kc * kTcKeys);   // valid keys of the chunk
+      const uint32_t lb = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kTcKeys);
+      if (j < nkc) {
+        float cm = -INFINITY;
+        float v[32];
+        for (int c0 = 0; c0 < nv; c0 += 32) {
+          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (c0 + e < nv) cm = fmaxf(cm, v[e] * sc);
+        }
+        const float nm = fmaxf(m, cm);
+        float cs = 0.f;
+        for (int c0 = 0; c0 < nv; c0 += 32) {
+          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (c0 + e < nv) cs += exp2f(v[e] * sc - nm);
+        }
+        ssum = ssum * exp2f(m - nm) + cs;   // exp2(-inf) = 0 on the first chunk
+        m = nm;
+        if (j == nkc - 1) {
+          // full-sequence variant: the row's non-visual mass joins the denominator
+          const float o = (a.lse && rq < L)
+                              ? __ldg(a.lse + (long long)h * a.lse_hs + (long long)(r.l_off + rq) * a.lse_rs) * kLog2e
+                              : -INFINITY;
+          const float tm = fmaxf(m, o);
+          const float sv = ssum * exp2f(m - tm);   // visual mass, rescaled
+          inv = 1.0f / (sv + exp2f(o - tm));
+          m = tm;
+          // Eq. 8 takes the variance about the row's mean: 1 / K1, or its visual mass / K1
+          mean = a.lse ? (sv * inv) / (float)K1 : 1.0f / (float)K1;
+          if (rq < L) {
+            float* st = a.rstat + 2 * ((long long)h * a.stats_ld + r.l_off + rq);
+            st[0] = m;
+            st[1] = inv;
+          }
+        }
+      } else {
+        float v[32];
+        for (int c0 = 0; c0 < nv; c0 += 32) {
+          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (c0 + e < nv) {
+              const float p = exp2f(v[e] * sc - m) * inv;
+              var = fmaf(p - mean, p - mean, var);
+            }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
+    }
+    if (!s_abort && rq < L) a.row_var[(long long)h * a.stats_ld + r.l_off + rq] = var / (float)K1;
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * kTcKeys);
+  }
+  if (s_abort) {
+    if (tid == 0) atomicOr(a.err, 1u);   // the loader's copies have landed (cp.async.wait_all)
+    return;
+  }
+
+  // completion of this grid implies completion of the preceding one
+  if (a.overlap && !a.independent) pdl_wait();
+  if (!a.hs_finalize) return;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) {
+    const unsigned prev = atomicAdd(&a.cnt_hs[b], 1u);
+    s_last = (prev == (unsigned)(a.Hq * nqc) - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (tid == 0) a.cnt_hs[b] = 0u;
+  // u_h = mean over text rows of the row variances: one warp per head, lanes over rows
+  for (int hh = warp; hh < a.Hq; hh += kTcThreads / 32) {
+    const float* rv = a.row_var + (long long)hh * a.stats_ld + r.l_off;
+    float s = 0.f;
+    for (int x = lane; x < L; x += 32) s += __ldcg(rv + x);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) a.u[(long long)b * a.u_ld + hh] = s / (float)L;
+  }
+  if (a.zero_p)
+    for (int i = tid; i < K1; i += kTcThreads) a.p_bits[r.k1_off + i] = 0u;
 }
 
 // ------------------------------------------------------------------ token scores by recomputation
@@ -768,6 +994,12 @@ cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_l,
   const int smem = 16 * nw * kRowBytes + 2 * kKB * kRowBytes;   // Q rows and two K chunks
   return nw == 8 ? launch_kernel(in_head_stats_kernel<8>, dim3(meta.total_hs), dim3(256), smem, st, true, meta, a)
                  : launch_kernel(in_head_stats_kernel<4>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a);
+}
+
+// The statistics of the batched path on tcgen05: one block per (request, head, 128 text rows).
+cudaError_t launch_in_head_stats_tc(const InMeta& meta, const InArgs& a, cudaStream_t st) {
+  if (meta.total_hs == 0) return cudaSuccess;
+  return launch_kernel(in_head_stats_tc_kernel, dim3(meta.total_hs), dim3(kTcThreads), kTcSmem, st, true, meta, a);
 }
 
 cudaError_t launch_in_token_score_qk(const InMeta& meta, const InArgs& a, int max_l, int max_k1, cudaStream_t st) {

@@ -40,6 +40,7 @@ struct InArgs {
   int overlap;              // head statistics need not wait for the preceding grid at start
   int independent;          // Q and K do not come from the preceding grid: the first
                             // stage-2 grid never waits for it (it may run beside it)
+  uint32_t* err;            // device status word: bit 0 = a bounded wait gave up
   const float* lse;         // full-sequence variant: log of the non-visual mass of row (h, q),
                             // at lse + h * lse_hs + (launch text row) * lse_rs; null: off
   long long lse_hs, lse_rs;
