@@ -22,10 +22,8 @@ cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool 
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
 cudaError_t launch_cls_saliency(const ClsMeta&, const ClsArgs&, int dh, int max_n, cudaStream_t);
-cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_l, cudaStream_t);
+cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
-cudaError_t launch_in_token_score_qk(const InMeta&, const InArgs&, int max_l, int max_k1, cudaStream_t);
-cudaError_t launch_in_head_stats_tc(const InMeta&, const InArgs&, cudaStream_t);
 bool in_small_fits(int Hq, int max_l, int max_k1);
 cudaError_t launch_in_small(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 }  // namespace trevs
@@ -86,7 +84,11 @@ cudaError_t aux_stream(AuxStream*& out) {
     }
   for (AuxStream& x : aux)
     if (x.device < 0) {
-      e = cudaStreamCreateWithFlags(&x.stream, cudaStreamNonBlocking);
+      // the stage-1 tail runs here: at the highest priority, so that its blocks take the SMs
+      // the scoring grid frees ahead of the stage-2 blocks still waiting on the caller's stream
+      int least = 0, greatest = 0;
+      e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
+      if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&x.stream, cudaStreamNonBlocking, greatest);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.fork, cudaEventDisableTiming);
       if (e == cudaSuccess) e = cudaEventCreateWithFlags(&x.join, cudaEventDisableTiming);
       if (e != cudaSuccess) return e;
@@ -183,20 +185,17 @@ PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1
 }
 
 struct InWs {
-  size_t cnt_hs, cnt_ts, attn, row_var, rstat, u, p, keys, flags, end;
+  size_t cnt_hs, cnt_ts, attn, row_var, u, p, keys, flags, end;
 };
 
-// total_lk1 = sum over requests of l * k1 (attention probabilities per head), kept only for
-// the small path (`small`), whose two grids pass the probabilities through the workspace; the
-// larger path keeps each row's max and 1 / sum (rstat) and recomputes.
-InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, int B, bool small = true) {
+// total_lk1 = sum over requests of l * k1 (attention probabilities per head).
+InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, int B) {
   InWs w;
   size_t o = kStatusBytes;
   w.cnt_hs = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
-  w.attn = o;      o = al256(o + (small ? 4 * (size_t)Hq * (size_t)total_lk1 : 0));
+  w.attn = o;      o = al256(o + 4 * (size_t)Hq * (size_t)total_lk1);
   w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
-  w.rstat = o;     o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
   w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
   w.p = o;         o = al256(o + 4 * (size_t)total_k1);
   const size_t padded = (size_t)total_k1 + 4 * (size_t)kMaxChunk + 4;   // per-request 16-byte alignment
@@ -505,7 +504,7 @@ trevs_status run_pre_batch(const trevs_pre_batch* bt, const trevs_pre_params& pr
 
 struct InTotals {
   long long l = 0, k1 = 0, k2 = 0, lk1 = 0;
-  int max_k1 = 0, max_l = 0;
+  int max_k1 = 0;
 };
 
 trevs_status validate_in_common(int Hq, int Hkv, int d_h, int n_keep) {
@@ -542,7 +541,6 @@ trevs_status validate_in_batch(const trevs_in_batch* bt, InTotals& t) {
     TREVS_CHECK(r.k2 >= 0 && r.k2 <= r.k1, "request %d: k2 = %d outside [0, k1 = %d]", b, r.k2, r.k1);
     t.l += r.l; t.k1 += r.k1; t.k2 += r.k2; t.lk1 += (long long)r.l * r.k1;
     t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
-    t.max_l = r.l > t.max_l ? r.l : t.max_l;
   }
   TREVS_CHECK(t.l < (1ll << 31) && t.k1 < (1ll << 31), "batch too large for int32 offsets");
   s = validate_qk(bt->Q, bt->q_head_stride, bt->q_tok_stride, bt->K, bt->kv_head_stride, bt->kv_tok_stride);
@@ -607,8 +605,7 @@ void fill_compaction(GatherMeta& gm, const InMeta& meta, const uint16_t* hidden,
 // `merged`: gather jobs of stage 1 to launch together with the compaction.
 trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_base, long long k1_base,
                           long long k2_base, uint8_t* ws, const InWs& L, cudaStream_t st, bool overlap,
-                          GatherMeta* merged, bool launch_gather_here = true, bool independent = false,
-                          uint32_t* status = nullptr) {
+                          GatherMeta* merged, bool launch_gather_here = true, bool independent = false) {
   static thread_local InMeta meta;
   static thread_local GatherMeta gm_own;
   GatherMeta& gm = merged ? *merged : gm_own;
@@ -626,16 +623,15 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
     max_l = q.l > max_l ? q.l : max_l;
   }
-  // block counts per request: the head-statistics grid takes 128 text rows per block (one
-  // per TMEM lane), the token-score grid stats_rows(max_l)
-  const int qc = stats_rows(max_l);
+  // block counts per request: text chunks of the head-statistics and token-score grids
+  const int qc = stats_text_rows(max_k1);
   for (int b = b0; b < b1; ++b) {
     const trevs_in_request& q = bt->reqs[b];
     InReq& r = meta.r[b - b0];
     r.hs_off = hs;
     r.ts_off = ts;
-    hs += bt->Hq * ((q.l + 127) / 128);
-    ts += ((q.l + qc - 1) / qc) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
+    hs += bt->Hq * ((q.l + qc - 1) / qc);
+    ts += ((q.l + kScoreTextRows - 1) / kScoreTextRows) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
   }
   meta.total_hs = hs;
   meta.total_ts = ts;
@@ -649,7 +645,6 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.scale = bt->softmax_scale > 0.f ? bt->softmax_scale : 1.0f / sqrtf((float)bt->d_h);
   a.attn = reinterpret_cast<float*>(ws + L.attn);
   a.row_var = reinterpret_cast<float*>(ws + L.row_var);
-  a.rstat = reinterpret_cast<float*>(ws + L.rstat);
   a.stats_ld = lo;
   a.u = (bt->u ? bt->u : reinterpret_cast<float*>(ws + L.u)) + (long long)b0 * bt->Hq;
   a.u_ld = bt->Hq;
@@ -660,7 +655,6 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.flags = ws + L.flags;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + L.cnt_hs);
   a.cnt_ts = reinterpret_cast<uint32_t*>(ws + L.cnt_ts);
-  a.err = status ? status : reinterpret_cast<uint32_t*>(ws);
   a.hs_finalize = 1;
   a.zero_p = 1;
   if (bt->lse_other) {
@@ -674,8 +668,8 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
     ++g_launches;   // two grids
   } else {
-    TREVS_TRY_CUDA(counted(launch_in_head_stats_tc(meta, a, st)), "head_stats launch");
-    TREVS_TRY_CUDA(counted(launch_in_token_score_qk(meta, a, max_l, max_k1, st)), "token_score launch");
+    TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
+    TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");
   }
   if (k2o > 0 && (bt->hidden || bt->K_out || bt->V)) {
     fill_compaction(gm, meta,
@@ -726,13 +720,11 @@ int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const 
   return r;
 }
 
-trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st,
-                          uint32_t* status = nullptr) {
+trevs_status run_in_batch(const trevs_in_batch* bt, uint8_t* ws, const InWs& L, cudaStream_t st) {
   long long l_base = 0, k1_base = 0, k2_base = 0;
   for (int b0 = 0; b0 < bt->B; b0 += kMaxChunk) {
     const int b1 = b0 + kMaxChunk < bt->B ? b0 + kMaxChunk : bt->B;
-    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st, false, nullptr, true, false,
-                                  status);
+    trevs_status s = run_in_chunk(bt, b0, b1, l_base, k1_base, k2_base, ws, L, st, false, nullptr);
     if (s != TREVS_OK) return s;
     for (int b = b0; b < b1; ++b) {
       l_base += bt->reqs[b].l; k1_base += bt->reqs[b].k1; k2_base += bt->reqs[b].k2;
@@ -1071,7 +1063,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   static thread_local InMeta meta;
   meta.B = 1;
   meta.r[0] = InReq{0, 0, L, 0, K1, 0, 0, 0, 0};
-  meta.total_hs = Hq * ((L + stats_rows(L) - 1) / stats_rows(L));
+  meta.total_hs = Hq * ((L + stats_text_rows(K1) - 1) / stats_text_rows(K1));
   meta.total_ts = 0;
   InArgs a;
   memset(&a, 0, sizeof(a));
@@ -1080,9 +1072,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.Hq = Hq; a.Hkv = Hkv; a.n_keep = 1;
   a.scale = softmax_scale > 0.f ? softmax_scale : 1.0f / sqrtf((float)d_h);
   a.attn = attn_out;
-  a.write_attn = 1;
   a.row_var = reinterpret_cast<float*>(ws + W.row_var);
-  a.rstat = reinterpret_cast<float*>(ws + W.rstat);
   a.stats_ld = L;
   a.u = u_out; a.u_ld = Hq;
   a.cnt_hs = reinterpret_cast<uint32_t*>(ws + W.cnt_hs);
@@ -1090,7 +1080,7 @@ trevs_status trevs_in_llm_head_scores(const uint16_t* Q, int64_t q_head_stride, 
   a.hs_finalize = 1; a.zero_p = 0;
   TREVS_CHECK(lse_other == nullptr || ((uintptr_t)lse_other & 3u) == 0, "lse_other must be 4-byte aligned");
   a.lse = lse_other; a.lse_hs = L; a.lse_rs = 1;
-  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, L, (cudaStream_t)stream)), "head_stats launch");
+  TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, K1, (cudaStream_t)stream)), "head_stats launch");
   return TREVS_OK;
 }
 
@@ -1192,16 +1182,12 @@ size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
   long long l = 0, k1 = 0, lk1 = 0;
-  int max_l = 0, max_k1 = 0;
   for (int b = 0; b < batch->B; ++b) {
     const long long lb = batch->reqs[b].l > 0 ? batch->reqs[b].l : 0;
     const long long kb = batch->reqs[b].k1 > 0 ? batch->reqs[b].k1 : 0;
     l += lb; k1 += kb; lk1 += lb * kb;
-    max_l = lb > max_l ? (int)lb : max_l;
-    max_k1 = kb > max_k1 ? (int)kb : max_k1;
   }
-  const int Hq = batch->Hq > 0 ? batch->Hq : 0;
-  return in_ws(l, k1, lk1, Hq, batch->B, in_small_fits(Hq, max_l, max_k1)).end;
+  return in_ws(l, k1, lk1, batch->Hq > 0 ? batch->Hq : 0, batch->B).end;
 }
 
 size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, const trevs_in_batch* in) {
@@ -1253,7 +1239,7 @@ trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch, void* workspace, s
   InTotals t;
   trevs_status s = validate_in_batch(batch, t);
   if (s != TREVS_OK || batch->B == 0) return s;
-  const InWs L = in_ws(t.l, t.k1, t.lk1, batch->Hq, batch->B, in_small_fits(batch->Hq, t.max_l, t.max_k1));
+  const InWs L = in_ws(t.l, t.k1, t.lk1, batch->Hq, batch->B);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_in_batch(batch, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -1275,8 +1261,7 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1, pre->d);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
-  const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B,
-                       in->B > 0 && in_small_fits(in->Hq, ti.max_l, ti.max_k1));
+  const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);
   s = check_ws(workspace, workspace_bytes, need);
   if (s != TREVS_OK) return s;
@@ -1311,8 +1296,7 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
       s = run_pre_chunk(pre, prm, 0, pre->B, 0, 0, 0, ws, LP, st, nullptr, aux->fork, nullptr, aux->stream,
                         reserve, &forked);
       if (s != TREVS_OK) return joined(s);
-      s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true,
-                       reinterpret_cast<uint32_t*>(ws));
+      s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, st, false, nullptr, true, true);
       return joined(s);
     }
     // One chunk each. The stages are independent, but the scoring grid fills every SM; stage
@@ -1322,15 +1306,14 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
     if (s != TREVS_OK) return s;
     TREVS_TRY_CUDA(cudaStreamWaitEvent(aux->stream, aux->fork, 0), "fork");
     forked = true;
-    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true, false,
-                     reinterpret_cast<uint32_t*>(ws));
+    s = run_in_chunk(in, 0, in->B, 0, 0, 0, ws + pre_bytes, LI, aux->stream, false, nullptr, true);
     return joined(s);
   }
   if (pre->B > 0) {
     s = run_pre_batch(pre, prm, ws, LP, st);
     if (s != TREVS_OK) return s;
   }
-  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, st, reinterpret_cast<uint32_t*>(ws));
+  if (in->B > 0) return run_in_batch(in, ws + pre_bytes, LI, st);
   return TREVS_OK;
 }
 

@@ -1,14 +1,12 @@
 // Stage 2 (in-LLM at layer l*, Sec. 4.2): text-to-vision attention statistics, head
 // variance (Eq. 8), high-variance head set H*, token scores (Eq. 9), TopK and compaction.
 #include "in_llm.cuh"
-#include "sm100.cuh"
 
 namespace trevs {
 
 constexpr int kKB = kKeyBlock;
 constexpr int kDh = 128;       // head width
 constexpr int kRowBytes = kDh * 2;
-constexpr float kLog2e = 1.4426950408889634f;
 
 // Row q of a [rows][128] bf16 tile: 16 chunks of 16 bytes, XOR-swizzled on the low 3 bits.
 __device__ __forceinline__ uint32_t tile_addr(uint32_t base, int row, int chunk) {
@@ -57,24 +55,18 @@ __device__ __forceinline__ void qk_tile(const uint32_t (&af)[8][4], uint32_t ks_
 
 // ------------------------------------------------------------------ attention statistics
 //
-// Block (request, head h, chunk of QR = 16 NW text rows), NW warps of 16 rows each. The
-// logits Q_h . K_g^T * scale of the chunk's rows against the K1 visual keys are formed twice
-// on the tensor cores (mma.sync, fragments in registers), with K streamed in 64-key chunks
-// through a two-buffer cp.async ring: pass 1 keeps each row's running max and sum of exp
-// (online softmax; with the full-sequence variant the row's non-visual mass joins at the
-// end); pass 2 forms the probabilities and the two-pass Eq. 8 variance about the row's mean.
-// A quad of lanes holds two rows, so row reductions take quad shuffles. Each row's max and
-// 1 / sum go to the workspace: the token scores recompute the probabilities of the heads of
-// H* only, so the [Hq, L, K1] probabilities never reach memory unless the caller asks for
-// them (write_attn). One K_g chunk serves 64 or 128 text rows, where a block that kept the
-// logits of a whole row range in shared memory fitted only 16 rows at K1 = 1024, and read
-// each K_g once per 16 rows. The last block of a request averages the row variances into u_h
-// and clears p for the token scores.
-template <int NW>
-__global__ void __launch_bounds__(32 * NW) in_head_stats_kernel(const __grid_constant__ InMeta meta, const InArgs a) {
-  constexpr int QR = 16 * NW;
-  constexpr int NT = kKB / 8;          // n-tiles of a 64-key chunk
-  constexpr int NTH = 32 * NW;
+// Block (request, head h, chunk of QC = 16*MT text rows): logits Q_h . K_g^T * scale for all
+// K1 keys into shared memory (tensor cores; K streamed once in 64-key chunks through a
+// two-buffer cp.async ring), then per row the max, the sum of exp and the two-pass
+// variance of the softmax row about its mean 1/K1 (Eq. 8). The last block of a request
+// averages the row variances into u_h and clears p for the token-score pass.
+// Warp w computes m-tile (w % MT) against key slice (w / MT) of each chunk.
+template <int MT>
+__global__ void __launch_bounds__(128) in_head_stats_kernel(const __grid_constant__ InMeta meta,
+                                                            const InArgs a, int k1_ld) {
+  constexpr int QC = 16 * MT;
+  constexpr int KW = 16 * MT;          // keys per warp in a 64-key chunk
+  constexpr int NT = KW / 8;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_last;
   if (!a.overlap && !a.independent) pdl_wait();   // Q, K may come from the preceding grid
@@ -82,124 +74,103 @@ __global__ void __launch_bounds__(32 * NW) in_head_stats_kernel(const __grid_con
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
   const InReq r = meta.r[b];
-  const int nqc = (r.l + QR - 1) / QR;
+  const int nqc = (r.l + QC - 1) / QC;
   const int t = blockIdx.x - r.hs_off;
   const int h = t / nqc, qc = t - h * nqc;
   const int g = (h * a.Hkv) / a.Hq;
-  const int q0 = qc * QR;
-  const int K1 = r.k1, L = r.l, nkc = (K1 + kKB - 1) / kKB;
-  const uint32_t qs_a = smem_u32(smem), kb_a = qs_a + QR * kRowBytes;
+  const int q0 = qc * QC;
+
+  uint8_t* qs = smem;                              // QC x 256 B
+  uint8_t* kbuf = smem + QC * kRowBytes;           // 2 x 64 x 256 B
+  float* lg = reinterpret_cast<float*>(kbuf + 2 * kKB * kRowBytes);   // [QC][k1_ld]
+  const uint32_t qs_a = smem_u32(qs), kb_a = smem_u32(kbuf);
+
   const __nv_bfloat16* Qb = a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs;
   const __nv_bfloat16* Kb = a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs;
-  const float sc = a.scale * kLog2e;   // logits in log2 units: exp(x) = exp2(x * log2 e)
-  const int ra = q0 + 16 * warp + (lane >> 2), rb = ra + 8;   // this thread's text rows
+  const int nkc = (r.k1 + kKB - 1) / kKB;
+  const int mt = warp % MT, kslice = warp / MT;
+  const float sc = a.scale * 1.4426950408889634f;   // logits in log2 units: exp(x) = exp2(x * log2 e)
 
-  load_rows(qs_a, Qb, a.q_ts, q0, QR, L, tid, NTH);
-  load_rows(kb_a, Kb, a.k_ts, 0, kKB, K1, tid, NTH);
+  load_rows(qs_a, Qb, a.q_ts, q0, QC, r.l, tid, 128);
+  load_rows(kb_a, Kb, a.k_ts, 0, kKB, r.k1, tid, 128);
   cp_async_commit();
   uint32_t af[8][4];
-  float ma = -INFINITY, mb = -INFINITY, sa = 0.f, sb = 0.f;   // running max and sum (log2 units)
-  float ia = 0.f, ib = 0.f, mna = 0.f, mnb = 0.f;             // 1 / sum and row mean (pass 2)
-  float va = 0.f, vb = 0.f;                                   // sums of squared deviations
-  float* A = a.write_attn ? a.attn + r.attn_off + (long long)h * L * K1 : nullptr;
-  for (int it = 0; it < 2 * nkc; ++it) {          // pass 1: chunks 0..nkc-1; pass 2: again
-    const int kc = it < nkc ? it : it - nkc;
-    if (it + 1 < 2 * nkc) {
-      const int nc = it + 1 < nkc ? it + 1 : it + 1 - nkc;
-      load_rows(kb_a + ((it + 1) & 1) * kKB * kRowBytes, Kb, a.k_ts, nc * kKB, kKB, K1, tid, NTH);
-    }
+  for (int kc = 0; kc < nkc; ++kc) {
+    if (kc + 1 < nkc) load_rows(kb_a + ((kc + 1) & 1) * kKB * kRowBytes, Kb, a.k_ts, (kc + 1) * kKB, kKB, r.k1, tid, 128);
     cp_async_commit();
     cp_async_wait<1>();
     __syncthreads();
-    if (it == 0) load_afrag(qs_a, 16 * warp, lane, af);
+    if (kc == 0) load_afrag(qs_a, 16 * mt, lane, af);
     float acc[NT][4];
-    qk_tile<NT>(af, kb_a + (it & 1) * kKB * kRowBytes, 0, lane, acc);
-    if (it < nkc) {
-      float ca = -INFINITY, cb = -INFINITY;
+    qk_tile<NT>(af, kb_a + (kc & 1) * kKB * kRowBytes, kslice * KW, lane, acc);
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e)
-          if (kc * kKB + 8 * nt + 2 * (lane & 3) + e < K1) {
-            ca = fmaxf(ca, acc[nt][e] * sc);
-            cb = fmaxf(cb, acc[nt][2 + e] * sc);
-          }
-#pragma unroll
-      for (int o = 1; o < 4; o <<= 1) {
-        ca = fmaxf(ca, __shfl_xor_sync(0xffffffffu, ca, o));
-        cb = fmaxf(cb, __shfl_xor_sync(0xffffffffu, cb, o));
-      }
-      const float na = fmaxf(ma, ca), nb = fmaxf(mb, cb);
-      float pa = 0.f, pb = 0.f;
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e)
-          if (kc * kKB + 8 * nt + 2 * (lane & 3) + e < K1) {
-            pa += exp2f(acc[nt][e] * sc - na);
-            pb += exp2f(acc[nt][2 + e] * sc - nb);
-          }
-#pragma unroll
-      for (int o = 1; o < 4; o <<= 1) {
-        pa += __shfl_xor_sync(0xffffffffu, pa, o);
-        pb += __shfl_xor_sync(0xffffffffu, pb, o);
-      }
-      sa = sa * exp2f(ma - na) + pa;   // exp2(-inf) = 0 on the first chunk
-      sb = sb * exp2f(mb - nb) + pb;
-      ma = na;
-      mb = nb;
-      if (it == nkc - 1) {
-        // full-sequence variant: the row's non-visual mass joins the denominator
-        float oa = -INFINITY, ob = -INFINITY;
-        if (a.lse) {
-          const float* lr = a.lse + (long long)h * a.lse_hs + (long long)r.l_off * a.lse_rs;
-          if (ra < L) oa = __ldg(lr + (long long)ra * a.lse_rs) * kLog2e;
-          if (rb < L) ob = __ldg(lr + (long long)rb * a.lse_rs) * kLog2e;
-        }
-        const float ta = fmaxf(ma, oa), tb = fmaxf(mb, ob);
-        const float sva = sa * exp2f(ma - ta), svb = sb * exp2f(mb - tb);   // visual mass, rescaled
-        ia = 1.0f / (sva + exp2f(oa - ta));
-        ib = 1.0f / (svb + exp2f(ob - tb));
-        ma = ta;
-        mb = tb;
-        // Eq. 8 takes the variance about each row's mean: 1 / K1, or its visual mass / K1
-        mna = a.lse ? (sva * ia) / (float)K1 : 1.0f / (float)K1;
-        mnb = a.lse ? (svb * ib) / (float)K1 : 1.0f / (float)K1;
-        if ((lane & 3) == 0) {
-          float* st = a.rstat + 2 * ((long long)h * a.stats_ld + r.l_off);
-          if (ra < L) { st[2 * ra] = ma; st[2 * ra + 1] = ia; }
-          if (rb < L) { st[2 * rb] = mb; st[2 * rb + 1] = ib; }
-        }
-      }
-    } else {
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int key = kc * kKB + 8 * nt + 2 * (lane & 3) + e;
-          if (key < K1) {
-            const float pa = exp2f(acc[nt][e] * sc - ma) * ia;
-            const float pb = exp2f(acc[nt][2 + e] * sc - mb) * ib;
-            va = fmaf(pa - mna, pa - mna, va);
-            vb = fmaf(pb - mnb, pb - mnb, vb);
-            if (A) {
-              if (ra < L) A[(long long)ra * K1 + key] = pa;
-              if (rb < L) A[(long long)rb * K1 + key] = pb;
-            }
-          }
-        }
+    for (int nt = 0; nt < NT; ++nt) {
+      const int key = kc * kKB + kslice * KW + 8 * nt + 2 * (lane & 3);
+      const int row = 16 * mt + (lane >> 2);
+      *reinterpret_cast<float2*>(lg + row * k1_ld + key) = make_float2(acc[nt][0] * sc, acc[nt][1] * sc);
+      *reinterpret_cast<float2*>(lg + (row + 8) * k1_ld + key) = make_float2(acc[nt][2] * sc, acc[nt][3] * sc);
     }
-    __syncthreads();   // the buffer just read is refilled in the next iteration
+    __syncthreads();
   }
+
+  // row statistics, TPR threads per row (all rows of the chunk in parallel)
+  constexpr int TPR = 128 / QC;
+  __shared__ float s_inv[64];
+  __shared__ float s_mean[64];
+  const int k1 = r.k1;
+  {
+    const int rr = tid / TPR, sub = tid % TPR;
+    float* row = lg + rr * k1_ld;
+    // full-sequence variant: the row's non-visual mass joins the denominator (log2 units)
+    float other = -INFINITY;
+    if (a.lse && q0 + rr < r.l)
+      other = __ldg(a.lse + (long long)h * a.lse_hs + (long long)(r.l_off + q0 + rr) * a.lse_rs) *
+              1.4426950408889634f;
+    float mx = -INFINITY;
+#pragma unroll 4
+    for (int i = sub; i < k1; i += TPR) mx = fmaxf(mx, row[i]);
 #pragma unroll
-  for (int o = 1; o < 4; o <<= 1) {
-    va += __shfl_xor_sync(0xffffffffu, va, o);
-    vb += __shfl_xor_sync(0xffffffffu, vb, o);
+    for (int o = 1; o < TPR; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    mx = fmaxf(mx, other);
+    float sum = 0.f;
+#pragma unroll 4
+    for (int i = sub; i < k1; i += TPR) {
+      const float e = exp2f(row[i] - mx);
+      row[i] = e;
+      sum += e;
+    }
+#pragma unroll
+    for (int o = 1; o < TPR; o <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (sub == 0) {
+      const float tot = sum + exp2f(other - mx);   // + 0 without the variant
+      s_inv[rr] = 1.0f / tot;
+      // Eq. 8 takes the variance about the row's mean: 1 / K1, or its visual mass / K1
+      s_mean[rr] = a.lse ? (sum / tot) / (float)k1 : 1.0f / (float)k1;
+    }
   }
-  if ((lane & 3) == 0) {
-    float* rv = a.row_var + (long long)h * a.stats_ld + r.l_off;
-    if (ra < L) rv[ra] = va / (float)K1;
-    if (rb < L) rv[rb] = vb / (float)K1;
+  __syncthreads();
+  // A[h][q][i] = e / sum, written along i by whole warps, and the two-pass variance of the
+  // row about its mean (Eq. 8)
+  {
+    const int rows = min(QC, r.l - q0);
+    float* A = a.attn + r.attn_off + ((long long)h * r.l + q0) * k1;
+    for (int rr = warp; rr < rows; rr += 4) {
+      const float inv = s_inv[rr];
+      const float mean = s_mean[rr];
+      const float* row = lg + rr * k1_ld;
+      float* out = A + (long long)rr * k1;
+      float v = 0.f;
+#pragma unroll 2
+      for (int i = lane; i < k1; i += 32) {
+        const float p = row[i] * inv;
+        out[i] = p;
+        const float dlt = p - mean;
+        v = fmaf(dlt, dlt, v);
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (lane == 0) a.row_var[(long long)h * a.stats_ld + r.l_off + q0 + rr] = v / (float)k1;
+    }
   }
 
   // completion of this grid implies completion of the preceding one
@@ -216,383 +187,16 @@ __global__ void __launch_bounds__(32 * NW) in_head_stats_kernel(const __grid_con
   __threadfence();
   if (tid == 0) a.cnt_hs[b] = 0u;
   // u_h = mean over text rows of the row variances: one warp per head, lanes over rows
-  for (int hh = warp; hh < a.Hq; hh += NW) {
+  for (int hh = warp; hh < a.Hq; hh += 4) {
     const float* rv = a.row_var + (long long)hh * a.stats_ld + r.l_off;
     float s = 0.f;
-    for (int q = lane; q < L; q += 32) s += __ldcg(rv + q);
+    for (int q = lane; q < r.l; q += 32) s += __ldcg(rv + q);
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) a.u[(long long)b * a.u_ld + hh] = s / (float)L;
+    if (lane == 0) a.u[(long long)b * a.u_ld + hh] = s / (float)r.l;
   }
   if (a.zero_p)
-    for (int i = tid; i < K1; i += NTH) a.p_bits[r.k1_off + i] = 0u;
-}
-
-// ------------------------------------------------------------------ attention statistics on tcgen05
-//
-// Block (request, head h, 128 text rows): the 5th-generation tensor cores form the logits
-// S = Q_h . K_g^T of the block's rows (UMMA M = 128 rows, N = 128 keys, K = 128 dims) chunk by
-// chunk into a double-buffered TMEM accumulator, twice over the K1 keys: pass 1 for each row's
-// running max and sum of exp (online softmax; with the full-sequence variant the row's
-// non-visual mass joins at the end), pass 2 for the probabilities and the two-pass Eq. 8
-// variance about the row's mean. TMEM lane r holds text row r, so each epilogue thread owns a
-// whole row and its reductions need no shuffles. Q_h is copied once and K_g streams in
-// 128-key chunks through a two-stage ring (cp.async by one warp, into the 128-byte swizzled
-// K-major layout the UMMA descriptors state). Each row's max and 1 / sum go to the workspace
-// for the token scores. The last block of a request averages the row variances into u_h and
-// clears p.
-//
-// Warps: 0 = loader, 1 = TMEM owner and MMA issuer, 2..5 = epilogue (warp w reads TMEM lanes
-// 32*(w%4) .. +31, so the four cover the 128 rows).
-constexpr int kTcKeys = 128;                       // keys per chunk (UMMA N)
-constexpr int kTcThreads = 192;
-constexpr int kTcTileBytes = 128 * kRowBytes;      // 128 rows x 128 dims, two 64-dim slices
-constexpr int kTcStages = 2;
-constexpr int kTcSmem = (1 + kTcStages) * kTcTileBytes + 1024;
-
-// 16-byte pieces of `rows` rows (128 bf16 each) into a 128-byte swizzled, slice-major tile:
-// slice c (64 dims) of row r at c * rows * 128 + r * 128, piece q at (q ^ (r & 7)) * 16.
-__device__ __forceinline__ void load_rows_sw128(uint32_t dst, const __nv_bfloat16* base, long long row_stride,
-                                                int row0, int rows, int valid, int lane) {
-  for (int idx = lane; idx < rows * 16; idx += 32) {
-    const int rr = idx >> 4, p = idx & 15, c = p >> 3, q = p & 7;
-    const bool ok = row0 + rr < valid;
-    const void* src = ok ? (const void*)(base + (long long)(row0 + rr) * row_stride + p * 8) : (const void*)base;
-    cp_async16(dst + c * rows * 128 + rr * 128 + (swz(rr, q) << 4), src, ok ? 16 : 0);
-  }
-}
-
-__global__ void __launch_bounds__(kTcThreads, 1) in_head_stats_tc_kernel(const __grid_constant__ InMeta meta,
-                                                                          const InArgs a) {
-  using namespace sm100;
-  extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t qfull, kfull[kTcStages], kempty[kTcStages];
-  __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
-  __shared__ uint32_t tmem_base_s;
-  __shared__ volatile int s_abort;
-  __shared__ int s_last;
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t qs = smem_u32(smem), ks = qs + kTcTileBytes;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].hs_off; });
-  const InReq r = meta.r[b];
-  const int nqc = (r.l + 127) / 128;
-  const int t = blockIdx.x - r.hs_off;
-  const int h = t / nqc, qc = t - h * nqc;
-  const int g = (h * a.Hkv) / a.Hq;
-  const int q0 = qc * 128;
-  const int K1 = r.k1, L = r.l, nkc = (K1 + kTcKeys - 1) / kTcKeys;
-  const int nj = 2 * nkc;                          // pass 1 and pass 2 over the key chunks
-
-  if (tid == 0) {
-    mbar_init(smem_u32(&qfull), 32);
-    for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(smem_u32(&kfull[s]), 32);          // the loader's lanes, once their copies land
-      mbar_init(smem_u32(&kempty[s]), 1);          // MMA commit
-    }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_u32(&acc_full[i]), 1);
-      mbar_init(smem_u32(&acc_empty[i]), 4);       // the epilogue warps
-    }
-    s_abort = 0;
-    mbar_fence_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(smem_u32(&tmem_base_s), 2 * kTcKeys);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = tmem_base_s;
-  if (!a.overlap && !a.independent) pdl_wait();   // Q, K may come from the preceding grid
-  pdl_launch_dependents();
-
-  if (warp == 0) {
-    const __nv_bfloat16* Qb = a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs;
-    const __nv_bfloat16* Kb = a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs;
-    load_rows_sw128(qs, Qb, a.q_ts, q0, 128, L, lane);
-    cp_async_arrive_noinc(smem_u32(&qfull));
-    for (int j = 0; j < nj; ++j) {
-      const int s = j % kTcStages, ph = j / kTcStages;
-      if (j >= kTcStages && !mbar_wait(smem_u32(&kempty[s]), (ph - 1) & 1, &s_abort)) {
-        s_abort = 1;
-        break;
-      }
-      const int kc = j < nkc ? j : j - nkc;
-      load_rows_sw128(ks + s * kTcTileBytes, Kb, a.k_ts, kc * kTcKeys, kTcKeys, K1, lane);
-      cp_async_arrive_noinc(smem_u32(&kfull[s]));
-    }
-    cp_async_wait_all();
-  } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(128, kTcKeys);
-      bool ok = mbar_wait(smem_u32(&qfull), 0, &s_abort);
-      for (int j = 0; ok && j < nj; ++j) {
-        const int s = j % kTcStages, ph = j / kTcStages, buf = j & 1, use = j >> 1;
-        if (!mbar_wait(smem_u32(&kfull[s]), ph & 1, &s_abort)) ok = false;
-        if (ok && j >= 2 && !mbar_wait(smem_u32(&acc_empty[buf]), (use - 1) & 1, &s_abort)) ok = false;
-        if (!ok) break;
-        fence_proxy_async_smem();   // the stages were written by cp.async (generic proxy)
-        tc_fence_after();
-        const uint32_t kst = ks + s * kTcTileBytes, dt = tmem + (uint32_t)(buf * kTcKeys);
-#pragma unroll
-        for (int c = 0; c < 2; ++c)
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_bf16(dt, umma_desc_sw128(qs + c * kTcTileBytes / 2 + 32 * k),
-                      umma_desc_sw128(kst + c * kTcTileBytes / 2 + 32 * k), idesc, (c | k) != 0 ? 1u : 0u);
-        umma_commit(smem_u32(&kempty[s]));   // frees the K stage once these MMAs have read it
-        umma_commit(smem_u32(&acc_full[buf]));
-      }
-      if (!ok) s_abort = 1;
-    }
-  } else {
-    const int q = warp & 3, row = 32 * q + lane;   // TMEM lane quarter; the block's text row
-    const int rq = q0 + row;                       // request-local text row
-    const float sc = a.scale * kLog2e;            // logits in log2 units
-    float m = -INFINITY, ssum = 0.f, inv = 0.f, mean = 0.f, var = 0.f;
-    for (int j = 0; j < nj; ++j) {
-      const int buf = j & 1, use = j >> 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&acc_full[buf]), use & 1, &s_abort) && !s_abort);
-      if (!ok) {
-        s_abort = 1;
-        break;
-      }
-      tc_fence_after();
-      const int kc = j < nkc ? j : j - nkc;
-      const int nv = min(kTcKeys, K1 - kc * kTcKeys);   // valid keys of the chunk
-      const uint32_t lb = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kTcKeys);
-      if (j < nkc) {
-        float cm = -INFINITY;
-        float v[32];
-        for (int c0 = 0; c0 < nv; c0 += 32) {
-          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (c0 + e < nv) cm = fmaxf(cm, v[e] * sc);
-        }
-        const float nm = fmaxf(m, cm);
-        float cs = 0.f;
-        for (int c0 = 0; c0 < nv; c0 += 32) {
-          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (c0 + e < nv) cs += exp2f(v[e] * sc - nm);
-        }
-        ssum = ssum * exp2f(m - nm) + cs;   // exp2(-inf) = 0 on the first chunk
-        m = nm;
-        if (j == nkc - 1) {
-          // full-sequence variant: the row's non-visual mass joins the denominator
-          const float o = (a.lse && rq < L)
-                              ? __ldg(a.lse + (long long)h * a.lse_hs + (long long)(r.l_off + rq) * a.lse_rs) * kLog2e
-                              : -INFINITY;
-          const float tm = fmaxf(m, o);
-          const float sv = ssum * exp2f(m - tm);   // visual mass, rescaled
-          inv = 1.0f / (sv + exp2f(o - tm));
-          m = tm;
-          // Eq. 8 takes the variance about the row's mean: 1 / K1, or its visual mass / K1
-          mean = a.lse ? (sv * inv) / (float)K1 : 1.0f / (float)K1;
-          if (rq < L) {
-            float* st = a.rstat + 2 * ((long long)h * a.stats_ld + r.l_off + rq);
-            st[0] = m;
-            st[1] = inv;
-          }
-        }
-      } else {
-        float v[32];
-        for (int c0 = 0; c0 < nv; c0 += 32) {
-          tmem_ld_32x32b_x32(lb + (uint32_t)c0, v);
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (c0 + e < nv) {
-              const float p = exp2f(v[e] * sc - m) * inv;
-              var = fmaf(p - mean, p - mean, var);
-            }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
-    }
-    if (!s_abort && rq < L) a.row_var[(long long)h * a.stats_ld + r.l_off + rq] = var / (float)K1;
-  }
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, 2 * kTcKeys);
-  }
-  if (s_abort) {
-    if (tid == 0) atomicOr(a.err, 1u);   // the loader's copies have landed (cp.async.wait_all)
-    return;
-  }
-
-  // completion of this grid implies completion of the preceding one
-  if (a.overlap && !a.independent) pdl_wait();
-  if (!a.hs_finalize) return;
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    const unsigned prev = atomicAdd(&a.cnt_hs[b], 1u);
-    s_last = (prev == (unsigned)(a.Hq * nqc) - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (tid == 0) a.cnt_hs[b] = 0u;
-  // u_h = mean over text rows of the row variances: one warp per head, lanes over rows
-  for (int hh = warp; hh < a.Hq; hh += kTcThreads / 32) {
-    const float* rv = a.row_var + (long long)hh * a.stats_ld + r.l_off;
-    float s = 0.f;
-    for (int x = lane; x < L; x += 32) s += __ldcg(rv + x);
-#pragma unroll
-    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) a.u[(long long)b * a.u_ld + hh] = s / (float)L;
-  }
-  if (a.zero_p)
-    for (int i = tid; i < K1; i += kTcThreads) a.p_bits[r.k1_off + i] = 0u;
-}
-
-// ------------------------------------------------------------------ token scores by recomputation
-//
-// Block (request, chunk of QR text rows, 64-key block): H* from u (ties to the lower head),
-// then for each head of H* in ascending order the logits of the block's rows and keys again
-// (mma.sync), the probabilities from the row max and 1 / sum of the statistics grid, and
-// their sum over the heads in registers (Eq. 9, head mean); then the max over the rows, merged
-// across blocks with an integer atomicMax on the (non-negative) float bits, exact and order
-// independent. Each head's Q rows and K chunk stream through a two-buffer cp.async ring. The
-// last block of a request (a self-resetting ticket) selects TopK(p, K2) and writes H*.
-template <int NW>
-__global__ void __launch_bounds__(32 * NW) in_token_score_qk_kernel(const __grid_constant__ InMeta meta,
-                                                                    const InArgs a, int sel_off) {
-  constexpr int QR = 16 * NW;
-  constexpr int NT = kKB / 8;
-  constexpr int NTH = 32 * NW;
-  constexpr int BUF = QR * kRowBytes + kKB * kRowBytes;   // one head's Q rows and K chunk
-  extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ SelShared ss;
-  __shared__ float s_u[kMaxHeads];
-  __shared__ int s_heads[kMaxHeads];
-  __shared__ int s_sel[kMaxHeads];
-  __shared__ float s_red[NW][kKB];
-  __shared__ int s_nh, s_last;
-  pdl_wait();   // u, the row statistics and the cleared p come from the preceding grid
-  pdl_launch_dependents();
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].ts_off; });
-  const InReq r = meta.r[b];
-  const int K1 = r.k1, L = r.l;
-  const int nib = (K1 + kKB - 1) / kKB;
-  const int t = blockIdx.x - r.ts_off;
-  const int qc = t / nib, ib = t - qc * nib;
-  const int q0 = qc * QR, i0 = ib * kKB;
-
-  // H*: the n_keep heads of largest u, ties to the lower head; at most n_keep even if u holds NaN
-  const float* u = a.u + (long long)b * a.u_ld;
-  for (int hh = tid; hh < a.Hq; hh += NTH) s_u[hh] = __ldcg(u + hh);
-  __syncthreads();
-  for (int hh = tid; hh < a.Hq; hh += NTH) {
-    const float uh = s_u[hh];
-    int rank = 0;
-    for (int x = 0; x < a.Hq; ++x) rank += (s_u[x] > uh) || (s_u[x] == uh && x < hh);
-    s_sel[hh] = rank < a.n_keep;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    int cnt = 0;
-    for (int hh = 0; hh < a.Hq && cnt < a.n_keep; ++hh)
-      if (s_sel[hh]) s_heads[cnt++] = hh;
-    s_nh = cnt;
-  }
-  __syncthreads();
-  const int nh = s_nh;
-
-  const float sc = a.scale * kLog2e;
-  const int ra = q0 + 16 * warp + (lane >> 2), rb = ra + 8;
-  const uint32_t base = smem_u32(smem);
-  auto issue = [&](int x) {   // head x of H*: its Q rows and the block's K chunk
-    const int h = s_heads[x], g = (h * a.Hkv) / a.Hq;
-    const uint32_t qs = base + (x & 1) * BUF, ks = qs + QR * kRowBytes;
-    load_rows(qs, a.Q + (long long)r.l_off * a.q_ts + (long long)h * a.q_hs, a.q_ts, q0, QR, L, tid, NTH);
-    load_rows(ks, a.K + (long long)r.k1_off * a.k_ts + (long long)g * a.k_hs, a.k_ts, i0, kKB, K1, tid, NTH);
-  };
-  float ps[NT][4];   // sum over the heads of H* of the probabilities of rows ra, rb
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int e = 0; e < 4; ++e) ps[nt][e] = 0.f;
-  if (nh > 0) issue(0);
-  cp_async_commit();
-  for (int x = 0; x < nh; ++x) {
-    if (x + 1 < nh) issue(x + 1);
-    cp_async_commit();
-    const int h = s_heads[x];
-    const float* st = a.rstat + 2 * ((long long)h * a.stats_ld + r.l_off);
-    const float2 sa = ra < L ? __ldcg(reinterpret_cast<const float2*>(st) + ra) : make_float2(0.f, 0.f);
-    const float2 sb = rb < L ? __ldcg(reinterpret_cast<const float2*>(st) + rb) : make_float2(0.f, 0.f);
-    cp_async_wait<1>();
-    __syncthreads();
-    const uint32_t qs = base + (x & 1) * BUF;
-    uint32_t af[8][4];
-    load_afrag(qs, 16 * warp, lane, af);
-    float acc[NT][4];
-    qk_tile<NT>(af, qs + QR * kRowBytes, 0, lane, acc);
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        ps[nt][e] += exp2f(acc[nt][e] * sc - sa.x) * sa.y;       // rows past L: 1 / sum = 0
-        ps[nt][2 + e] += exp2f(acc[nt][2 + e] * sc - sb.x) * sb.y;
-      }
-    __syncthreads();   // the buffer just read is refilled two heads later
-  }
-  // Eq. 9: max over the rows of the head mean; probabilities are positive, so 0 never wins
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      float m = fmaxf(ps[nt][e], ps[nt][2 + e]);
-#pragma unroll
-      for (int o = 4; o < 32; o <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-      if (lane < 4) s_red[warp][8 * nt + 2 * lane + e] = m;
-    }
-  __syncthreads();
-  if (tid < kKB && i0 + tid < K1) {
-    float m = 0.f;
-#pragma unroll
-    for (int w = 0; w < NW; ++w) m = fmaxf(m, s_red[w][tid]);
-    const float inv_nh = nh > 0 ? 1.0f / (float)nh : 0.f;
-    atomicMax(a.p_bits + r.k1_off + i0 + tid, __float_as_uint(m * inv_nh));
-  }
-
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    const int nqc = (L + QR - 1) / QR;
-    const unsigned prev = atomicAdd(&a.cnt_ts[b], 1u);
-    s_last = (prev == (unsigned)(nqc * nib) - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (tid == 0) a.cnt_ts[b] = 0u;
-  if (a.heads_out)
-    for (int x = tid; x < nh; x += NTH) a.heads_out[(long long)b * a.n_keep + x] = s_heads[x];
-  if (r.k2 <= 0) return;
-  uint32_t* keys = reinterpret_cast<uint32_t*>(smem + sel_off);   // K1 keys, then K1 flags
-  uint8_t* flags = smem + sel_off + (size_t)K1 * 4;
-  for (int i = tid; i < K1; i += NTH) flags[i] = 0;
-  uint32_t lo, hi, tau;
-  int need, n_eq;
-  block_fill_keys(keys, reinterpret_cast<const float*>(a.p_bits + r.k1_off), K1,
-                  [&](float x, int) { return score_key(x); }, ss, lo, hi);
-  if (K1 <= NTH) {
-    block_mark_topk_small(keys, K1, r.k2, flags);
-  } else {
-    block_kth_largest(keys, K1, r.k2, ss, lo, hi, tau, need, n_eq);
-    block_mark_selected(keys, K1, tau, need, n_eq, flags, ss);
-  }
-  block_compact_flags(flags, K1, a.kept_local + r.k2_off, ss);
+    for (int i = tid; i < r.k1; i += 128) a.p_bits[r.k1_off + i] = 0u;
 }
 
 // ------------------------------------------------------------------ token scores
@@ -986,31 +590,29 @@ __global__ void __launch_bounds__(kSelThreads) in_select_small_kernel(const __gr
 
 // ------------------------------------------------------------------ host-side launchers
 
-// Statistics and recomputed token scores for larger requests: 4 warps (64 text rows) per
-// block, or 8 (128 rows) when some request has more than 64 text rows.
-cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_l, cudaStream_t st) {
-  if (meta.total_hs == 0) return cudaSuccess;
-  const int nw = stats_warps(max_l);
-  const int smem = 16 * nw * kRowBytes + 2 * kKB * kRowBytes;   // Q rows and two K chunks
-  return nw == 8 ? launch_kernel(in_head_stats_kernel<8>, dim3(meta.total_hs), dim3(256), smem, st, true, meta, a)
-                 : launch_kernel(in_head_stats_kernel<4>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a);
-}
+// Row stride of the logits tile: 2 mod 32 words keeps the row-parallel passes conflict-free.
+int in_head_stats_ld(int max_k1) { return ((max_k1 + kKB - 1) / kKB) * kKB + 2; }
 
-// The statistics of the batched path on tcgen05: one block per (request, head, 128 text rows).
-cudaError_t launch_in_head_stats_tc(const InMeta& meta, const InArgs& a, cudaStream_t st) {
+cudaError_t launch_in_head_stats(const InMeta& meta, const InArgs& a, int max_k1, cudaStream_t st) {
   if (meta.total_hs == 0) return cudaSuccess;
-  return launch_kernel(in_head_stats_tc_kernel, dim3(meta.total_hs), dim3(kTcThreads), kTcSmem, st, true, meta, a);
-}
-
-cudaError_t launch_in_token_score_qk(const InMeta& meta, const InArgs& a, int max_l, int max_k1, cudaStream_t st) {
-  if (meta.total_ts == 0) return cudaSuccess;
-  const int nw = stats_warps(max_l);
-  const int bufs = 2 * (16 * nw * kRowBytes + kKB * kRowBytes);
-  const int smem = bufs + max_k1 * 5 + 16;   // then the keys and flags of the last block's TopK
-  return nw == 8 ? launch_kernel(in_token_score_qk_kernel<8>, dim3(meta.total_ts), dim3(256), smem, st, true, meta,
-                                 a, bufs)
-                 : launch_kernel(in_token_score_qk_kernel<4>, dim3(meta.total_ts), dim3(128), smem, st, true, meta,
-                                 a, bufs);
+  const int ld = in_head_stats_ld(max_k1);
+  const int qc = stats_text_rows(max_k1);
+  const int smem = qc * kRowBytes + 2 * kKB * kRowBytes + qc * ld * 4;   // two K chunk buffers
+  cudaError_t e;
+  switch (qc) {
+    case 64:
+      e = ensure_dynamic_smem(in_head_stats_kernel<4>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<4>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+    case 32:
+      e = ensure_dynamic_smem(in_head_stats_kernel<2>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<2>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+    default:
+      e = ensure_dynamic_smem(in_head_stats_kernel<1>, smem);
+      if (e != cudaSuccess) return e;
+      return launch_kernel(in_head_stats_kernel<1>, dim3(meta.total_hs), dim3(128), smem, st, true, meta, a, ld);
+  }
 }
 
 // The two-grid small path when every request has L <= 64 and K1 <= 128.

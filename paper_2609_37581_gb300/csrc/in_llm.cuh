@@ -9,10 +9,8 @@ constexpr int kMaxHeads = 128;
 constexpr int kKeyBlock = 64;        // visual keys per stage-2 block / shared-memory chunk
 constexpr int kScoreTextRows = 16;   // text rows per token-score block
 
-// Warps per head-statistics and recomputed-token-score block (16 text rows each): 8 when some
-// request of the launch has more than 64 text rows, else 4.
-inline int stats_warps(int max_l) { return max_l > 64 ? 8 : 4; }
-inline int stats_rows(int max_l) { return 16 * stats_warps(max_l); }
+// Text rows per head-statistics block: the block keeps rows x K1 fp32 logits on chip.
+inline int stats_text_rows(int max_k1) { return max_k1 <= 128 ? 64 : (max_k1 <= 512 ? 32 : 16); }
 
 struct InArgs {
   const __nv_bfloat16* Q;
@@ -22,9 +20,7 @@ struct InArgs {
   int Hq, Hkv, n_keep;
   float scale;
   float* attn;              // attention probabilities, request b at attn_off: [Hq][l][k1]
-  int write_attn;           // the statistics grid also writes the probabilities to attn
   float* row_var;           // [Hq][stats_ld]: Var_i A[q, i]
-  float* rstat;             // [Hq][stats_ld][2]: each row's max (log2 units) and 1 / sum
   long long stats_ld;       // total text rows of the launch
   float* u;                 // [B][u_ld] head variances (Eq. 8)
   int u_ld;
@@ -40,7 +36,6 @@ struct InArgs {
   int overlap;              // head statistics need not wait for the preceding grid at start
   int independent;          // Q and K do not come from the preceding grid: the first
                             // stage-2 grid never waits for it (it may run beside it)
-  uint32_t* err;            // device status word: bit 0 = a bounded wait gave up
   const float* lse;         // full-sequence variant: log of the non-visual mass of row (h, q),
                             // at lse + h * lse_hs + (launch text row) * lse_rs; null: off
   long long lse_hs, lse_rs;
