@@ -110,6 +110,19 @@ TREVS_API trevs_status trevs_workspace_status(const void* workspace, size_t byte
 /* Zero-fills `bytes` of workspace on `stream` (cudaMemsetAsync). */
 TREVS_API trevs_status trevs_workspace_init(void* workspace, size_t bytes, void* stream);
 
+/* Test hooks of the failure paths; neither has a counterpart in the paper, and neither faults,
+ * traps or hangs the GPU.
+ * trevs_workspace_set_wait_limit: every bounded device-side wait of the calls that use this
+ *   workspace gives up after `microseconds` instead of 2 s (0 restores 2 s); a wait that gives
+ *   up makes its kernel stop, let its copies in flight land, release what it holds and set the
+ *   status word (trevs_workspace_status then reports TREVS_ERR_TIMEOUT). The limit lives in the
+ *   workspace header (written on `stream`), so trevs_workspace_init clears it.
+ * trevs_test_fail_launch: the n-th kernel launch attempt of this host thread from now on fails
+ *   without launching, as if the launch had failed (TREVS_ERR_CUDA); n <= 0 disarms it. */
+TREVS_API trevs_status trevs_workspace_set_wait_limit(void* workspace, size_t bytes, uint32_t microseconds,
+                                            void* stream);
+TREVS_API void trevs_test_fail_launch(int32_t n);
+
 /* ===================================================================== stage 1, one request
  *
  * Z   [N, d] bf16, row r at Z + r*z_row_stride   projected visual features z_i (Sec. 4.1)

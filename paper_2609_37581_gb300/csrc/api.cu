@@ -107,6 +107,7 @@ namespace {
 
 thread_local char g_err[512] = "";
 thread_local int g_launches = 0;     // kernels enqueued by the current call
+thread_local int g_fail_in = 0;      // launch attempts until the one the test hook fails (0: none)
 
 // Counts one enqueued kernel or memset of the current call.
 inline cudaError_t counted(cudaError_t e) {
@@ -125,6 +126,8 @@ trevs_status fail(trevs_status s, const char* fmt, ...) {
 trevs_status cuda_fail(cudaError_t e, const char* where) {
   return fail(TREVS_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
 }
+// cudaErrorLaunchFailure never comes back from an enqueue: a launch that reports it was the one
+// the test hook failed (launch_fault_injected), which made no launch.
 
 #define TREVS_TRY_CUDA(expr, where)            \
   do {                                         \
@@ -742,6 +745,7 @@ namespace trevs {
 // and trevs_last_launch_count.
 trevs_status record_error(trevs_status s, const char* msg) { return fail(s, "%s", msg); }
 void record_launches(int n) { g_launches = n; }
+bool launch_fault_injected() { return g_fail_in > 0 && --g_fail_in == 0; }
 }  // namespace trevs
 
 // ======================================================================== C ABI
@@ -767,6 +771,18 @@ trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* s
   if (word & 1u) return fail(TREVS_ERR_TIMEOUT, "a bounded device-side wait gave up (status word 0x%x)", word);
   if (word & 2u)
     return fail(TREVS_ERR_INVALID_ARGUMENT, "farthest point sampling found no candidate left (status word 0x%x)", word);
+  return TREVS_OK;
+}
+
+void trevs_test_fail_launch(int32_t n) { g_fail_in = n > 0 ? n : 0; }
+
+trevs_status trevs_workspace_set_wait_limit(void* workspace, size_t bytes, uint32_t microseconds, void* stream) {
+  g_launches = 0;
+  if (!workspace || bytes < 2 * sizeof(uint32_t)) return fail(TREVS_ERR_WORKSPACE, "workspace is NULL or too small");
+  const uint32_t us = microseconds;   // pageable source: copied out before the call returns
+  TREVS_TRY_CUDA(cudaMemcpyAsync(reinterpret_cast<uint32_t*>(workspace) + 1, &us, sizeof(us), cudaMemcpyHostToDevice,
+                                 (cudaStream_t)stream),
+                 "wait limit write");
   return TREVS_OK;
 }
 

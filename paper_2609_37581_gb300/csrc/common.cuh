@@ -601,11 +601,16 @@ inline cudaError_t ensure_dynamic_smem(Kernel kernel, int bytes) {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// Test hook of the host-side error paths (trevs_test_fail_launch): true when this launch
+// attempt of the calling thread is the one set to fail; the launch is then not made.
+bool launch_fault_injected();
+
 // Launches `kernel`, optionally allowed to start before the preceding work of the stream
 // completes (it must then call pdl_wait() before it touches that work's results).
 template <class... KArgs, class... Args>
 inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                                  bool pdl, Args... args) {
+  if (launch_fault_injected()) return cudaErrorLaunchFailure;
   const cudaError_t e = ensure_dynamic_smem(kernel, (int)smem);   // carveout, dynamic limit
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};

@@ -99,7 +99,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t zfull[kMaxZStages], zempty[kMaxZStages];
   __shared__ __align__(8) uint64_t tfull[kMaxTSlots], tempty[kMaxTSlots];
-  __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], norm_full[2], norm_empty[2];
+  __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2], norm_full[2], norm_empty[2], mma_drain;
   __shared__ uint32_t tmem_base_s;
   __shared__ float rinv_s[4][256];   // one row per epilogue warp (no cross-warp barrier)
   __shared__ float zsq_s[2][2][kTileRows];   // [buffer][half of the columns][row]
@@ -116,6 +116,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   const long long W = (long long)meta.total_tiles * nzs, P = gridDim.x;
   const long long u0 = W * blockIdx.x / P, u1 = W * (blockIdx.x + 1) / P;
   const bool ragged = (d % (kChunk * kZSlices)) != 0;       // last Z stage copied slice by slice
+  // word 1 of the workspace header, when set, replaces the 2 s limit of every wait (microseconds)
+  const uint32_t lim_us = __ldcg(a.err + 1);
+  const uint64_t lim = lim_us ? (uint64_t)lim_us * 1000ull : 2000000000ull;
   const int SZ = L.z_stages, ST = L.t_slots, TS = L.t_slot_slices;
   const int t_slot_bytes = TS * L.t_slice_bytes;
 
@@ -134,6 +137,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       mbar_init(smem_u32(&norm_full[i]), kZNormWarps);
       mbar_init(smem_u32(&norm_empty[i]), 4);
     }
+    mbar_init(smem_u32(&mma_drain), 1);
     s_abort = 0;
     s_zissued = 0;
     mbar_fence_init();
@@ -160,7 +164,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         const int y0 = r.n_off + t.row0;
         for (int zs = t.zs0; zs < t.zs1; ++zs, ++gz) {
           const int s = gz % SZ, it = gz / SZ;
-          if (gz >= SZ && !mbar_wait(smem_u32(&zempty[s]), (it - 1) & 1, &s_abort)) {
+          if (gz >= SZ && !mbar_wait(smem_u32(&zempty[s]), (it - 1) & 1, &s_abort, lim)) {
             s_abort = 1;
             return false;
           }
@@ -188,7 +192,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       int gz = 0, gt = 0, j = 0;
       for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& t) {
         const int buf = j & 1, use = j >> 1;
-        if (j >= 2 && !mbar_wait(smem_u32(&acc_empty[buf]), (use - 1) & 1, &s_abort)) {
+        if (j >= 2 && !mbar_wait(smem_u32(&acc_empty[buf]), (use - 1) & 1, &s_abort, lim)) {
           s_abort = 1;
           return false;
         }
@@ -198,7 +202,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         int kc = 0;   // slice index within the sub-tile
         for (int zs = t.zs0; zs < t.zs1; ++zs, ++gz) {
           const int s = gz % SZ, it = gz / SZ;
-          if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort)) {
+          if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort, lim)) {
             s_abort = 1;
             return false;
           }
@@ -206,7 +210,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
           const int ns = min(kZSlices, nk - zs * kZSlices);
           for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
             const int ts = gt % ST, tit = gt / ST;
-            if (!mbar_wait(smem_u32(&tfull[ts]), tit & 1, &s_abort)) {
+            if (!mbar_wait(smem_u32(&tfull[ts]), tit & 1, &s_abort, lim)) {
               s_abort = 1;
               return false;
             }
@@ -228,6 +232,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         ++j;
         return true;
       });
+      if (s_abort) {
+        // no MMA may still write TMEM when it is released: wait for every one issued
+        const volatile int no_abort = 0;
+        umma_commit(smem_u32(&mma_drain));
+        mbar_wait(smem_u32(&mma_drain), 0, &no_abort, 500000000ull);
+      }
     }
   } else if (warp < 4) {
     // T copies: the slices of the next slot from the request's M text rows, piece p = 16
@@ -243,7 +253,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         const int ns = min(kZSlices, nk - zs * kZSlices);
         for (int c0 = 0; c0 < ns; c0 += TS, ++gt) {
           const int ts = gt % ST, tit = gt / ST;
-          if (gt >= ST && !mbar_wait(smem_u32(&tempty[ts]), (tit - 1) & 1, &s_abort)) {
+          if (gt >= ST && !mbar_wait(smem_u32(&tempty[ts]), (tit - 1) & 1, &s_abort, lim)) {
             s_abort = 1;
             return false;
           }
@@ -277,7 +287,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       const bool mine = row < st.h;
       for (int zs = st.zs0; zs < st.zs1; ++zs, ++gz) {
         const int s = gz % SZ, it = gz / SZ;
-        if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort)) {
+        if (!mbar_wait(smem_u32(&zfull[s]), it & 1, &s_abort, lim)) {
           s_abort = 1;
           return false;
         }
@@ -296,7 +306,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&zempty[s]));
       }
-      if (j >= 2 && !mbar_wait(smem_u32(&norm_empty[buf]), (use - 1) & 1, &s_abort)) {
+      if (j >= 2 && !mbar_wait(smem_u32(&norm_empty[buf]), (use - 1) & 1, &s_abort, lim)) {
         s_abort = 1;
         return false;
       }
@@ -319,8 +329,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       __syncwarp();
       for (int c = lane; c < m; c += 32) rt[c] = __ldcg(a.t_rinv + r.m_off + c);
       __syncwarp();
-      bool ok = mbar_wait(smem_u32(&acc_full[buf]), use & 1, &s_abort);
-      ok = ok && mbar_wait(smem_u32(&norm_full[buf]), use & 1, &s_abort);
+      bool ok = mbar_wait(smem_u32(&acc_full[buf]), use & 1, &s_abort, lim);
+      ok = ok && mbar_wait(smem_u32(&norm_full[buf]), use & 1, &s_abort, lim);
       ok = __all_sync(0xffffffffu, ok && !s_abort);
       if (!ok) {
         s_abort = 1;
@@ -767,6 +777,7 @@ cudaError_t launch_pre_saliency(const PreMeta& meta, const PreArgs& a, int max_n
   (void)max_n;   // requests above kRegSelMaxN keep their keys in the global scratch
   cudaError_t e = ensure_dynamic_smem(pre_saliency_kernel, 0);   // the scoring grid's carveout
   if (e != cudaSuccess) return e;
+  if (launch_fault_injected()) return cudaErrorLaunchFailure;
   pre_saliency_kernel<<<(unsigned)(n_sal + tn_blocks), 512, 0, st>>>(meta, a, 0, n_sal);
   return cudaGetLastError();
 }

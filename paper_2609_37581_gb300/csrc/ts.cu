@@ -140,6 +140,7 @@ trevs_status trevs_textual_sensitivity(const float* attn1, int32_t L1, const flo
   a.part = reinterpret_cast<float*>(ws + L.part);
   a.cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
   a.ts = ts_out;
+  if (launch_fault_injected()) return record_error(TREVS_ERR_CUDA, "injected launch failure (test hook)");
   textual_sensitivity_kernel<<<dim3((unsigned)a.nchunk, (unsigned)Hq), kTsKeys, 0,
                                static_cast<cudaStream_t>(stream)>>>(a);
   const cudaError_t e = cudaGetLastError();

@@ -266,3 +266,9 @@ def test_textual_sensitivity_validation(lib):
     assert ts(None, 4, FAKE, 4, 2, 10, FAKE, None, None, FAKE, need, None) == t.TREVS_ERR_INVALID_ARGUMENT
     assert ts(FAKE, 4, FAKE, 4, 28, 1024, FAKE, None, None, FAKE, need - 1, None) == t.TREVS_ERR_WORKSPACE
     assert ts(FAKE, 4, FAKE, 4, 28, 1024, FAKE, None, None, None, need, None) == t.TREVS_ERR_WORKSPACE
+
+
+def test_failure_hooks_validate_on_the_host(lib):
+    assert lib.trevs_workspace_set_wait_limit(None, 1 << 20, 5, None) == t.TREVS_ERR_WORKSPACE
+    assert lib.trevs_workspace_set_wait_limit(FAKE, 4, 5, None) == t.TREVS_ERR_WORKSPACE
+    lib.trevs_test_fail_launch(0)   # disarmed: nothing to check without a GPU
