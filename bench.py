@@ -236,10 +236,11 @@ OTHER_CONFIGS = {   # the benchmark spec's other single-GPU configurations, each tim
 }
 
 
-def time_workload(T, w, stream, sampler, steps, peak, src):
+def time_workload(T, w, stream, sampler, steps, peak, src, method=False):
     """us per trevs_prune_varlen call on workload `w`: CUDA-event timing around graph replays
     over ROTATING_SETS input sets (each set > L2), the scoring grid timed alone with the
-    library's event hook, the clocks sampled meanwhile."""
+    library's event hook, the clocks sampled meanwhile; with `method`, also the paper's
+    Method settings (fused score, K_r:K_d = 3:1 diversity draws) the same way."""
     import torch
     from workloads.device import build_batches, dev_bf16, dev_f32
     params = T.default_params(T.SELECT_RATIO)
@@ -287,6 +288,35 @@ def time_workload(T, w, stream, sampler, steps, peak, src):
             T.trevs_pre_llm_varlen_timed(q, wsq, evs[i][0], evs[i][1], params, stream)
         torch.cuda.synchronize()
         kernel_ms = statistics.median(x.elapsed_time(y) for x, y in evs[8:])
+        method_out = None
+        if method:
+            mparams = T.default_params(T.SELECT_FUSED, diversity=METHOD_RHO)
+            mcalls = [T.PreparedCall(p, i, ws, mparams) for p, i in batches]
+            for c in mcalls:
+                c(stream)
+            mlaunches = T.last_launch_count()
+            mgraphs = []
+            for c in mcalls:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    c(stream)
+                mgraphs.append(g)
+            for i in range(4):
+                mgraphs[i % ROTATING_SETS].replay()
+            msteps = max(20, steps // 4)
+            a.record(stream)
+            for i in range(msteps):
+                mgraphs[i % ROTATING_SETS].replay()
+            b.record(stream)
+            torch.cuda.synchronize()
+            mms = a.elapsed_time(b) / msteps
+            mb = algorithmic_bytes(w)["method_step"]
+            kr = sorted({r.k1 - int(np.floor(np.float32(METHOD_RHO) * r.k1 + 0.5)) for r in w.reqs})
+            method_out = {"select": "fused (Eq. 6-7)", "diversity": METHOD_RHO, "K_r": kr,
+                          "us_per_prune": round(mms * 1e3, 2), "value": w.visual_tokens() / (mms * 1e-3),
+                          "unit": UNIT, "steps": msteps, "launches_per_step": mlaunches, "algorithmic_bytes": mb,
+                          "frac": round(mb / (mms * 1e-3) / 1e9 / peak, 4), "peak_source": src}
+            del mgraphs, mcalls
     t1 = time.monotonic()
     nbytes = algorithmic_bytes(w)
     del graphs, calls, score_only, sets, batches, ws
@@ -305,7 +335,8 @@ def time_workload(T, w, stream, sampler, steps, peak, src):
                          "frac": round(nbytes["score_kernel"] / (kernel_ms * 1e-3) / 1e9 / peak, 4)},
         "clocks": sampler.summary(t0, t1),
         "timed": f"CUDA events around {steps} graph replays of trevs_prune_varlen, {ROTATING_SETS} rotating "
-                 "input sets (> L2)"}
+                 "input sets (> L2)",
+        **({"method_path": method_out} if method_out else {})}
 
 
 def gpu_arm(args, rank, world, w, cpu_baseline):
@@ -437,7 +468,8 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         if not args.no_configs:
             del csets, cs_v, cws
             for name, make in OTHER_CONFIGS.items():
-                others[name] = time_workload(T, make(), stream, sampler, max(50, min(args.steps, 2000)), peak, src)
+                others[name] = time_workload(T, make(), stream, sampler, max(50, min(args.steps, 2000)), peak, src,
+                                             method=name == "long_16384_b2_gqa")
 
     if distributed:
         elapsed_ms = max_over_ranks(elapsed_ms, dev)

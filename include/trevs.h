@@ -187,7 +187,8 @@ TREVS_API size_t trevs_pre_llm_fps_workspace_size(int32_t N, int32_t K_r, int32_
  * draw when made (+inf for the first draw without pivots). `pool` is the number of
  * candidates whose pairwise cosines are kept on chip (0: automatic; at most 128); the draws
  * do not depend on it beyond rounding. A pivot outside [0, N) reads as a zero row and
- * excludes nothing. Limits: K_r <= TREVS_MAX_TEXT_TOKENS, K_r + K_d <= N, d % 8 == 0. */
+ * excludes nothing. Limits: K_r + K_d <= N, d % 8 == 0 (more than TREVS_MAX_TEXT_TOKENS pivots
+ * take one more pass over Z per TREVS_MAX_TEXT_TOKENS pivots). */
 TREVS_API trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t N, int32_t d,
                                const int32_t* pivots, int32_t K_r, int32_t K_d, int32_t pool,
                                int32_t* picks, float* pick_dist,
@@ -355,8 +356,9 @@ TREVS_API size_t trevs_prune_varlen_workspace_size(const trevs_pre_batch* pre, c
  * and gather of the kept rows. With p->diversity = rho > 0 (Sec. 3.1 context preservation)
  * the rule keeps K_r = K1 - K_d pivots (the ratio split applies to K_r), farthest point
  * sampling (as trevs_pre_llm_fps) adds K_d = floor(rho*K1 + 1/2) tokens, and kept_idx holds
- * both sets together in ascending order. TREVS_ERR_UNSUPPORTED if some request would have
- * more than TREVS_MAX_TEXT_TOKENS pivots. */
+ * both sets together in ascending order. The distances to the pivots take one pass over Z per
+ * TREVS_MAX_TEXT_TOKENS pivots of the request with the most (the paper's K_r:K_d = 3:1 at
+ * K1 = 1024 gives 768 pivots: three passes). */
 TREVS_API trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_params* p,
                                   void* workspace, size_t workspace_bytes, void* stream);
 

@@ -227,7 +227,9 @@ FpsWs fps_ws(size_t o, long long total_n, long long piv_space, int max_kr, int d
   w.zero = o;    o = al256(o + 256);
   w.prow = o;    o = al256(o + 2 * (size_t)piv_space * (size_t)(d > 0 ? d : 0));
   w.t_rinv = o;  o = al256(o + 4 * (size_t)(piv_space > 0 ? piv_space : 0));
-  w.part = o;    o = al256(o + (total_n > 0 && max_kr > 0 ? pre_score_part_bytes(max_kr) : 0));
+  w.part = o;    o = al256(o + (total_n > 0 && max_kr > 0
+                                      ? pre_score_part_bytes(max_kr < TREVS_MAX_TEXT_TOKENS ? max_kr : TREVS_MAX_TEXT_TOKENS)
+                                      : 0));
   w.maxcos = o;  o = al256(o + 4 * (size_t)total_n);
   w.ub = o;      o = al256(o + 4 * (size_t)total_n);
   w.stamp = o;   o = al256(o + 4 * (size_t)total_n);
@@ -331,13 +333,37 @@ int diversity_count(int k1, float rho) {
   return kd < 0 ? 0 : (kd > k1 ? k1 : kd);
 }
 
-// Pivots above TREVS_MAX_TEXT_TOKENS do not fit the contraction that measures distances.
-trevs_status validate_diversity(const trevs_pre_batch* bt, const trevs_pre_params& p) {
-  if (p.diversity <= 0.f) return TREVS_OK;
-  for (int b = 0; b < bt->B; ++b) {
-    const int k1 = bt->reqs[b].k1, kd = diversity_count(k1, p.diversity);
-    if (kd > 0 && k1 - kd > TREVS_MAX_TEXT_TOKENS)
-      return fail(TREVS_ERR_UNSUPPORTED, "request %d: %d pivots (K1 - K_d) > %d", b, k1 - kd, TREVS_MAX_TEXT_TOKENS);
+// The distances of farthest point sampling take any number of pivots (in passes of at most
+// TREVS_MAX_TEXT_TOKENS columns of the contraction); nothing to check beyond the batch.
+trevs_status validate_diversity(const trevs_pre_batch*, const trevs_pre_params&) { return TREVS_OK; }
+
+// The largest cosine of every row of the requests of `dm` to that request's pivot rows (the
+// "text" rows of `da`, their norms already computed): the scoring contraction over at most
+// TREVS_MAX_TEXT_TOKENS pivot columns per pass (its TMEM accumulator), each pass after the
+// first keeping the max of what s_t holds (Sec. 3.1 distances are minima over the pivots).
+trevs_status run_pivot_contraction(const PreMeta& dm, const PreArgs& da, long long z_rows, int max_n, cudaStream_t st) {
+  static thread_local PreMeta pm;
+  int max_kr = 0;
+  for (int i = 0; i < dm.B; ++i) max_kr = dm.r[i].m > max_kr ? dm.r[i].m : max_kr;
+  for (int p0 = 0; p0 < max_kr; p0 += TREVS_MAX_TEXT_TOKENS) {
+    pm.B = 0;
+    int tiles = 0, mm = 0;
+    for (int i = 0; i < dm.B; ++i) {
+      const PreReq& r = dm.r[i];
+      if (r.n <= 0 || r.m <= p0) continue;   // no pivot columns left in this pass
+      PreReq q = r;
+      q.m_off = r.m_off + p0;
+      q.m = r.m - p0 < TREVS_MAX_TEXT_TOKENS ? r.m - p0 : TREVS_MAX_TEXT_TOKENS;
+      q.tile_off = tiles;
+      tiles += (r.n + kScoreTileRows - 1) / kScoreTileRows;
+      pm.r[pm.B++] = q;
+      mm = q.m > mm ? q.m : mm;
+    }
+    pm.total_tiles = tiles;
+    PreArgs pa = da;
+    pa.seed_merge = p0 > 0 ? 1 : 0;
+    TREVS_TRY_CUDA(counted(launch_pre_score(pm, pa, mm, z_rows, st, true)), "pivot contraction launch");
+    TREVS_TRY_CUDA(counted(launch_pre_finish(pm, pa, mm, max_n, true, st, true)), "pivot fixup launch");
   }
   return TREVS_OK;
 }
@@ -454,8 +480,8 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     da.total_m = ko;
     da.action = kActFpsSeed;
     TREVS_TRY_CUDA(counted(launch_pre_saliency(dm, da, max_n, false, ts)), "pivot norms launch");
-    TREVS_TRY_CUDA(counted(launch_pre_score(dm, da, max_kr, no, ts, true)), "pivot contraction launch");
-    TREVS_TRY_CUDA(counted(launch_pre_finish(dm, da, max_kr, max_n, true, ts, true)), "pivot fixup launch");
+    const trevs_status cs = run_pivot_contraction(dm, da, no, max_n, ts);
+    if (cs != TREVS_OK) return cs;
     FpsArgs f;
     memset(&f, 0, sizeof(f));
     f.Z = a.Z; f.z_stride = a.z_stride; f.d = a.d;
@@ -926,8 +952,6 @@ trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t 
   TREVS_CHECK(N >= 0 && K_r >= 0 && K_d >= 0, "N = %d, K_r = %d, K_d = %d: none may be negative", N, K_r, K_d);
   TREVS_CHECK((long long)K_r + K_d <= N, "K_r + K_d = %lld exceeds N = %d", (long long)K_r + K_d, N);
   TREVS_CHECK(pool >= 0, "pool = %d < 0", pool);
-  if (K_r > TREVS_MAX_TEXT_TOKENS)
-    return fail(TREVS_ERR_UNSUPPORTED, "K_r = %d > %d pivots", K_r, TREVS_MAX_TEXT_TOKENS);
   if (K_d == 0) return TREVS_OK;
   TREVS_CHECK(d >= 8 && d % 8 == 0, "d = %d must be a positive multiple of 8", d);
   TREVS_CHECK(Z != nullptr && aligned16(Z), "Z must be non-NULL and 16-byte aligned");
@@ -972,8 +996,8 @@ trevs_status trevs_pre_llm_fps(const uint16_t* Z, int64_t z_row_stride, int32_t 
     a.err = reinterpret_cast<uint32_t*>(ws);
     a.d = d; a.mode = kModeRatio; a.action = kActFpsSeed;
     TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, N, false, st)), "pivot norms launch");
-    TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, kr, N, st, true)), "pivot contraction launch");
-    TREVS_TRY_CUDA(counted(launch_pre_finish(meta, a, kr, N, true, st, true)), "pivot fixup launch");
+    const trevs_status cs = run_pivot_contraction(meta, a, N, N, st);
+    if (cs != TREVS_OK) return cs;
   }
   static thread_local FpsMeta fm;
   fm.B = 1;

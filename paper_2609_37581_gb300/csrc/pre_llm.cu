@@ -378,7 +378,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         mbar_arrive(smem_u32(&acc_empty[buf]));
         mbar_arrive(smem_u32(&norm_empty[buf]));
       }
-      if (st.slot < 0 && row < st.h) a.s_t[r.n_off + st.row0 + row] = kSeed ? mx : sqrtf(sum / (float)m);
+      if (st.slot < 0 && row < st.h) {
+        float* out = a.s_t + r.n_off + st.row0 + row;
+        if constexpr (kSeed) *out = a.seed_merge ? fmaxf(mx, __ldcg(out)) : mx;
+        else *out = sqrtf(sum / (float)m);
+      }
       ++j;
       return true;
     });
@@ -492,7 +496,10 @@ __device__ inline void fixup_tile(const FinJob& jb, const PreReq& r, int mld, co
     }
     if constexpr (kSeed) {
       for (int o = P >> 1; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = mx;
+      if (gl == 0 && row < h) {
+        float* out = a.s_t + r.n_off + row0 + row;
+        *out = a.seed_merge ? fmaxf(mx, __ldcg(out)) : mx;
+      }
     } else {
       for (int o = P >> 1; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
       if (gl == 0 && row < h) a.s_t[r.n_off + row0 + row] = sqrtf(sum / (float)m);

@@ -38,6 +38,8 @@ struct PreArgs {
   float tau_v, tau_t, lambda, eps;
   int action;          // kActScores / kActScoresFused / kActSelect
   int s_fused_given;   // select kernel: s_fused already holds Eq. 7 scores
+  int seed_merge;      // kActFpsSeed: s_t already holds the largest cosine to earlier pivots
+                       // (a pass over further pivot columns keeps the max)
 };
 
 // Saliency side of the selection, which depends on inputs only. Ratio mode: the rule for

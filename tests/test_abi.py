@@ -98,7 +98,9 @@ def test_fps_validation(lib):
     assert "exceeds" in _err(lib)
     assert fps(K_d=-1) == t.TREVS_ERR_INVALID_ARGUMENT
     assert fps(pool=-2) == t.TREVS_ERR_INVALID_ARGUMENT
-    assert fps(K_r=257, N=1000) == t.TREVS_ERR_UNSUPPORTED               # pivots play the text rows
+    # more than 256 pivots run in passes; they need a larger workspace, nothing else
+    assert fps(K_r=257, N=1000) == t.TREVS_ERR_WORKSPACE
+    assert lib.trevs_pre_llm_fps_workspace_size(1000, 257, 4096) > need
     assert fps(d=4100, zs=4100) == t.TREVS_ERR_INVALID_ARGUMENT
     assert fps(zs=4000) == t.TREVS_ERR_INVALID_ARGUMENT
     assert fps(Z=ctypes.c_void_p(0x10002)) == t.TREVS_ERR_INVALID_ARGUMENT
@@ -201,15 +203,14 @@ def test_varlen_diversity_validation(lib):
         assert lib.trevs_pre_llm_varlen(ctypes.byref(ok), ctypes.byref(p), FAKE, need, None) == \
             t.TREVS_ERR_INVALID_ARGUMENT
         assert "diversity" in _err(lib)
-    # K1 = 1024 at rho = 0.25 leaves 768 pivots: more than the contraction takes
+    # K1 = 1024 at rho = 0.25 leaves 768 pivots (three passes of the contraction): validation
+    # passes up to the workspace, for any share
     big = _pre_batch([(16384, 128, 1024, 0.5)], d=3584)
     nb = lib.trevs_pre_llm_varlen_workspace_size(ctypes.byref(big))
-    p = t.default_params(t.SELECT_FUSED, diversity=0.25)
-    assert lib.trevs_pre_llm_varlen(ctypes.byref(big), ctypes.byref(p), FAKE, nb, None) == t.TREVS_ERR_UNSUPPORTED
-    assert "pivots" in _err(lib)
-    # at rho = 0.75 the same request has 256 pivots, which fit: validation passes up to the workspace
-    p = t.default_params(t.SELECT_FUSED, diversity=0.75)
-    assert lib.trevs_pre_llm_varlen(ctypes.byref(big), ctypes.byref(p), FAKE, nb - 256, None) == t.TREVS_ERR_WORKSPACE
+    for rho in (0.25, 0.75):
+        p = t.default_params(t.SELECT_FUSED, diversity=rho)
+        assert lib.trevs_pre_llm_varlen(ctypes.byref(big), ctypes.byref(p), FAKE, nb - 256, None) == \
+            t.TREVS_ERR_WORKSPACE
 
 
 def test_varlen_timed_validation(lib):

@@ -145,8 +145,29 @@ def test_fps_zero_rows_tie_to_lower_index():
     check_draws(Z, piv, picks, dist, 12)
 
 
+@pytest.mark.parametrize("k_r", [257, 600])
+def test_fps_pivots_beyond_one_pass(k_r):
+    # more than 256 pivots: the distances take one pass of the contraction per 256 pivot
+    # columns, each later pass keeping the max cosine
+    Z = _clusters(31 + k_r, 3000, 256, 60, noise=0.5)
+    rng = np.random.default_rng(k_r)
+    piv = rng.choice(3000, size=k_r, replace=False).tolist()
+    picks, dist = run_fps(Z, piv, 50)
+    check_draws(Z, piv, picks, dist, 50)
+
+
+def test_fps_exact_distances_beyond_one_pass():
+    # 300 pivots over the exact-cosine hypercube rows: every draw and distance has one answer
+    Z = _hypercube_rows(3, 128, 37)
+    piv = list(range(0, 600, 2))
+    picks, dist = run_fps(Z, piv, 100)
+    ref, ref_d = O.farthest_point_sampling(O.bf16_bits_to_f64(Z), piv, 100)
+    np.testing.assert_array_equal(picks, ref)
+    np.testing.assert_array_equal(dist, ref_d.astype(np.float32))
+
+
 def test_fps_large_request_and_many_pivots():
-    # above 4096 rows the pool is chosen with the keys in memory; 256 pivots at most
+    # above 4096 rows the pool is chosen with the keys in memory
     Z = _clusters(13, 5000, 512, 40, noise=0.5)
     rng = np.random.default_rng(17)
     piv = rng.choice(5000, size=256, replace=False).tolist()
@@ -197,3 +218,16 @@ def test_method_path_llava_batch32_both_stages():
     assert exact + near == w.B and exact >= w.B - 8, (exact, near)
     ref = O.run_workload(w, "fused", stage1=False)
     H.check_workload(w, g, ref, "fused")
+
+
+@pytest.mark.parametrize("mode", ["fused", "ratio"])
+def test_method_path_k1_1024(mode):
+    # the Method settings at K1 = 1024 (768 pivots and 256 draws, K_r:K_d = 3:1) on requests
+    # shaped like the long-video batch but narrower (d' = 256, so that the oracle stays quick)
+    w = synth.small_case(seed_cfg=170, n=(6000, 4096), m=(128, 60), d=256, k1=(1024, 700),
+                         ratio=(0.5, 0.5), k2=(0, 0), planted=0.02)
+    m = T.SELECT_FUSED if mode == "fused" else T.SELECT_RATIO
+    g, ws = H.run_gpu(w, m, params=T.default_params(m, diversity=0.25), stages="pre")
+    T.workspace_status(ws)
+    exact, near = check_method_stage1(w, g, mode, 0.25)
+    assert exact + near == w.B
