@@ -641,6 +641,56 @@ def profile_run(w, stage="stage1", launches=5):
     print(json.dumps({"profile": stage, "launches": launches}))
 
 
+def reserve_sweep(names, values, steps=1000, repeats=3):
+    """us per trevs_prune_varlen call for each overlap reserve (SMs the scoring grid leaves to
+    stage 2; -1 = the library's estimate), CUDA events around graph replays over
+    ROTATING_SETS input sets; one JSON line per (workload, reserve)."""
+    import torch
+    from paper_2609_37581_gb300 import trevs as T
+    from workloads.device import build_batches, dev_bf16, dev_f32
+    lib = T.load()
+    params = T.default_params(T.SELECT_RATIO)
+    stream = torch.cuda.Stream()
+    for name in names:
+        w = workload() if name == "llava15_576_b32" else synth.WORKLOADS[name]()
+        with torch.cuda.stream(stream):
+            base = {"Z": dev_bf16(w.Z), "T": dev_bf16(w.T), "s_v": dev_f32(w.s_v), "Q": dev_bf16(w.Q),
+                    "K": dev_bf16(w.K), "V": dev_bf16(w.V), "hidden": dev_bf16(w.hidden)}
+            sets = [base] + [{k: v.clone() for k, v in base.items()} for _ in range(ROTATING_SETS - 1)]
+            batches = [build_batches(w, T.SELECT_RATIO, dev=x) for x in sets]
+            ws = T.workspace(max(T.trevs_prune_varlen_workspace_size(p, i) for p, i in batches))
+        for r in values:
+            lib.trevs_set_overlap_reserve(r)
+            try:
+                with torch.cuda.stream(stream):
+                    calls = [T.PreparedCall(p, i, ws, params) for p, i in batches]
+                    for c in calls:
+                        c(stream)
+                    graphs = []
+                    for c in calls:
+                        g = torch.cuda.CUDAGraph()
+                        with torch.cuda.graph(g, stream=stream):
+                            c(stream)
+                        graphs.append(g)
+                    us = []
+                    for _ in range(repeats):
+                        for i in range(20):
+                            graphs[i % ROTATING_SETS].replay()
+                        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                        a.record(stream)
+                        for i in range(steps):
+                            graphs[i % ROTATING_SETS].replay()
+                        b.record(stream)
+                        torch.cuda.synchronize()
+                        us.append(round(a.elapsed_time(b) / steps * 1e3, 2))
+            finally:
+                lib.trevs_set_overlap_reserve(-1)
+            print(json.dumps({"workload": w.name, "reserve": r, "us_per_prune": us}), flush=True)
+            del graphs, calls
+        del sets, batches, ws
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -656,6 +706,9 @@ def main():
     ap.add_argument("--workload", default="llava15_576_b32", choices=sorted(synth.WORKLOADS),
                     help="workload of --profile (default: the bench batch)")
     ap.add_argument("--launches", type=int, default=5, help="calls made by --profile")
+    ap.add_argument("--reserve-sweep", metavar="R,R,...",
+                    help="time the two-stage call of every configuration with each overlap reserve "
+                         "(-1 = the library's estimate) instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -671,6 +724,9 @@ def main():
         print(json.dumps(reference_arm(args, w)), flush=True)
         return
 
+    if args.reserve_sweep:
+        reserve_sweep(["llava15_576_b32", *OTHER_CONFIGS], [int(x) for x in args.reserve_sweep.split(",")])
+        return
     if args.profile:
         pw = workload() if args.workload == "llava15_576_b32" else synth.WORKLOADS[args.workload]()
         profile_run(pw, args.profile, args.launches)

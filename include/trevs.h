@@ -391,6 +391,14 @@ TREVS_API trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trev
                                 const trevs_in_batch* in,
                                 void* workspace, size_t workspace_bytes, void* stream);
 
+/* Tuning knob of trevs_prune_varlen (no counterpart in the paper): how many SMs the scoring
+ * grid leaves to stage 2 when the two stages overlap. sms < 0 (the default) restores the
+ * built-in estimate, which weighs the bytes the scoring grid streams against the attention
+ * work of stage 2; sms = 0 runs stage 2 after the scoring grid; larger values are clamped to
+ * half the SM count. Process-wide, read at the start of each call (a captured graph keeps the
+ * value of its capture). */
+TREVS_API void trevs_set_overlap_reserve(int32_t sms);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/trevs.h: argument validation, workspace
 // layout, per-launch request metadata and the launch sequence of each entry point.
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -726,11 +727,15 @@ constexpr double kScoreBytesPerUsPerSm = 37e3;    // 37 GB/s
 constexpr double kSmallUsPer1024Heads = 5.0;
 constexpr double kLargeUsPerMLogits = 2.5;
 
+std::atomic<int> g_reserve_override{-1};   // trevs_set_overlap_reserve; < 0: the estimate
+
 int overlap_reserve(const trevs_pre_batch* pre, const trevs_in_batch* in, const PreTotals& tp, bool small) {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 16)
     return 0;
+  const int forced = g_reserve_override.load(std::memory_order_relaxed);
+  if (forced >= 0) return forced < sms / 2 ? forced : sms / 2;
   const double score_us = (double)tp.n * pre->d * 2.0 / (kScoreBytesPerUsPerSm * sms);
   double logits = 0.0;
   for (int b = 0; b < in->B; ++b) logits += (double)in->Hq * in->reqs[b].l * in->reqs[b].k1;
@@ -801,6 +806,8 @@ trevs_status trevs_workspace_status(const void* workspace, size_t bytes, void* s
 }
 
 void trevs_test_fail_launch(int32_t n) { g_fail_in = n > 0 ? n : 0; }
+
+void trevs_set_overlap_reserve(int32_t sms) { g_reserve_override.store(sms < 0 ? -1 : sms); }
 
 trevs_status trevs_workspace_set_wait_limit(void* workspace, size_t bytes, uint32_t microseconds, void* stream) {
   g_launches = 0;

@@ -77,6 +77,7 @@ _SIGS = {
     "trevs_workspace_status": (_c_i32, [_vp, _c_sz, _vp]),
     "trevs_workspace_set_wait_limit": (_c_i32, [_vp, _c_sz, ctypes.c_uint32, _vp]),
     "trevs_test_fail_launch": (None, [_c_i32]),
+    "trevs_set_overlap_reserve": (None, [_c_i32]),
     "trevs_pre_llm_workspace_size": (_c_sz, [_c_i32]),
     "trevs_pre_llm_scores": (_c_i32, [_vp, _c_i64, _c_i32, _c_i32, _vp, _c_i64, _c_i32, _vp,
                                       ctypes.POINTER(PreParams), _vp, _vp, _vp, _c_sz, _vp]),

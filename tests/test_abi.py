@@ -273,3 +273,5 @@ def test_failure_hooks_validate_on_the_host(lib):
     assert lib.trevs_workspace_set_wait_limit(None, 1 << 20, 5, None) == t.TREVS_ERR_WORKSPACE
     assert lib.trevs_workspace_set_wait_limit(FAKE, 4, 5, None) == t.TREVS_ERR_WORKSPACE
     lib.trevs_test_fail_launch(0)   # disarmed: nothing to check without a GPU
+    lib.trevs_set_overlap_reserve(7)   # host-side setting only
+    lib.trevs_set_overlap_reserve(-1)

@@ -132,3 +132,18 @@ def test_tiles_split_between_scoring_ctas(d, m):
         mm = T.SELECT_FUSED if mode == "fused" else T.SELECT_RATIO
         g, _ = H.run_gpu(w, mm, stages="pre")
         H.check_workload(w, g, O.run_workload(w, mode=mode, stage2=False), mode)
+
+
+@pytest.mark.parametrize("make,reserve", [(synth.llava15_batch32, 0), (synth.llava15_batch32, 60),
+                                          (synth.llava_next_batch8, 0), (synth.llava_next_batch8, 8),
+                                          (synth.llava_next_batch8, 500)],
+                         ids=["b32_after", "b32_r60", "next_after", "next_r8", "next_clamped"])
+def test_overlap_reserve_settings(make, reserve):
+    # The reserve moves stage 2 behind (0) or beside the scoring grid and changes how the
+    # tiles split between scoring CTAs; the results stay those of the oracle.
+    w = make()
+    T.load().trevs_set_overlap_reserve(reserve)
+    try:
+        _run_and_check(w)
+    finally:
+        T.load().trevs_set_overlap_reserve(-1)
