@@ -189,7 +189,7 @@ PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1
 }
 
 struct InWs {
-  size_t cnt_hs, cnt_ts, attn, row_var, u, p, keys, flags, end;
+  size_t cnt_hs, cnt_ts, attn, row_var, rstat, u, p, keys, flags, end;
 };
 
 // total_lk1 = sum over requests of l * k1 (attention probabilities per head).
@@ -200,6 +200,7 @@ InWs in_ws(long long total_l, long long total_k1, long long total_lk1, int Hq, i
   w.cnt_ts = o;    o = al256(o + 4 * (size_t)kMaxChunk);
   w.attn = o;      o = al256(o + 4 * (size_t)Hq * (size_t)total_lk1);
   w.row_var = o;   o = al256(o + 4 * (size_t)Hq * (size_t)total_l);
+  w.rstat = o;     o = al256(o + 8 * (size_t)Hq * (size_t)total_l);
   w.u = o;         o = al256(o + 4 * (size_t)Hq * (size_t)(B > 0 ? B : 1));
   w.p = o;         o = al256(o + 4 * (size_t)total_k1);
   const size_t padded = (size_t)total_k1 + 4 * (size_t)kMaxChunk + 4;   // per-request 16-byte alignment
@@ -653,18 +654,6 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
     max_k1 = q.k1 > max_k1 ? q.k1 : max_k1;
     max_l = q.l > max_l ? q.l : max_l;
   }
-  // block counts per request: text chunks of the head-statistics and token-score grids
-  const int qc = stats_text_rows(max_k1);
-  for (int b = b0; b < b1; ++b) {
-    const trevs_in_request& q = bt->reqs[b];
-    InReq& r = meta.r[b - b0];
-    r.hs_off = hs;
-    r.ts_off = ts;
-    hs += bt->Hq * ((q.l + qc - 1) / qc);
-    ts += ((q.l + kScoreTextRows - 1) / kScoreTextRows) * ((q.k1 + kKeyBlock - 1) / kKeyBlock);
-  }
-  meta.total_hs = hs;
-  meta.total_ts = ts;
   InArgs a;
   memset(&a, 0, sizeof(a));
   a.Q = reinterpret_cast<const __nv_bfloat16*>(bt->Q) + l_base * bt->q_tok_stride;
@@ -675,6 +664,8 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   a.scale = bt->softmax_scale > 0.f ? bt->softmax_scale : 1.0f / sqrtf((float)bt->d_h);
   a.attn = reinterpret_cast<float*>(ws + L.attn);
   a.row_var = reinterpret_cast<float*>(ws + L.row_var);
+  a.rstat = reinterpret_cast<float2*>(ws + L.rstat);
+  a.err = reinterpret_cast<uint32_t*>(ws);
   a.stats_ld = lo;
   a.u = (bt->u ? bt->u : reinterpret_cast<float*>(ws + L.u)) + (long long)b0 * bt->Hq;
   a.u_ld = bt->Hq;
@@ -694,9 +685,28 @@ trevs_status run_in_chunk(const trevs_in_batch* bt, int b0, int b1, long long l_
   }
   a.overlap = overlap ? 1 : 0;
   a.independent = independent ? 1 : 0;
-  if (in_small_fits(bt->Hq, max_l, max_k1)) {
+  // block counts per request: text chunks of the head-statistics and token-score grids
+  static thread_local InTcMaps maps;
+  const bool small = in_small_fits(bt->Hq, max_l, max_k1);
+  const bool tc = !small && make_in_tc_maps(a, lo, ko, maps) == cudaSuccess;
+  const int qc = tc ? in_tc_text_rows() : stats_text_rows(max_k1);
+  const int sq = tc ? in_tc_text_rows() : kScoreTextRows, sk = tc ? in_tc_score_keys() : kKeyBlock;
+  for (int b = b0; b < b1; ++b) {
+    const trevs_in_request& q = bt->reqs[b];
+    InReq& r = meta.r[b - b0];
+    r.hs_off = hs;
+    r.ts_off = ts;
+    hs += bt->Hq * ((q.l + qc - 1) / qc);
+    ts += ((q.l + sq - 1) / sq) * ((q.k1 + sk - 1) / sk);
+  }
+  meta.total_hs = hs;
+  meta.total_ts = ts;
+  if (small) {
     TREVS_TRY_CUDA(counted(launch_in_small(meta, a, max_k1, st)), "stage-2 launch");
     ++g_launches;   // two grids
+  } else if (tc) {
+    TREVS_TRY_CUDA(counted(launch_in_stats_tc(meta, a, maps, st)), "head statistics launch");
+    TREVS_TRY_CUDA(counted(launch_in_score_tc(meta, a, maps, st)), "token scores launch");
   } else {
     TREVS_TRY_CUDA(counted(launch_in_head_stats(meta, a, max_k1, st)), "head_stats launch");
     TREVS_TRY_CUDA(counted(launch_in_token_score(meta, a, max_k1, st)), "token_score launch");

@@ -1,6 +1,8 @@
 // Stage 2 (in-LLM, Sec. 4.2) kernel arguments.
 #pragma once
 
+#include <cuda.h>
+
 #include "common.cuh"
 
 namespace trevs {
@@ -39,6 +41,28 @@ struct InArgs {
   const float* lse;         // full-sequence variant: log of the non-visual mass of row (h, q),
                             // at lse + h * lse_hs + (launch text row) * lse_rs; null: off
   long long lse_hs, lse_rs;
+  float2* rstat;            // [Hq][stats_ld]: (T, 1 / total) of each text row, log2 units, so that
+                            // A[h][q][i] = exp2(logit * scale * log2 e - T) / total
+  uint32_t* err;            // device status word: bit 0 = a bounded wait gave up
 };
+
+// Tensor map of a [rows][heads][128] bf16 tensor, boxes of box_rows rows x 64 dims of one head.
+cudaError_t make_tmap_heads(CUtensorMap* tm, const void* base, long long rows, int heads, long long tok_stride,
+                            long long head_stride, int box_rows);
+
+// Stage 2 on the tensor cores (in_llm_tc.cu): tensor maps of Q and K, rows per block and keys
+// per token-score block (for the host's block offsets), and the two grids.
+struct InQMaps {
+  CUtensorMap q128, q64, q32;   // Q boxes of 128, 64 and 32 rows
+};
+struct InTcMaps {
+  InQMaps q;
+  CUtensorMap k128, k64;
+};
+cudaError_t make_in_tc_maps(const InArgs& a, long long q_rows, long long k_rows, InTcMaps& m);
+int in_tc_text_rows();
+int in_tc_score_keys();
+cudaError_t launch_in_stats_tc(const InMeta& meta, const InArgs& a, const InTcMaps& m, cudaStream_t st);
+cudaError_t launch_in_score_tc(const InMeta& meta, const InArgs& a, const InTcMaps& m, cudaStream_t st);
 
 }  // namespace trevs

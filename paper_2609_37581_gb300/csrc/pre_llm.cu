@@ -672,6 +672,25 @@ static cudaError_t make_tmap_sliced(CUtensorMap* tm, const void* base, long long
   return res == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// Tensor map of a [rows][heads][128] bf16 tensor with element strides tok_stride (rows) and
+// head_stride (heads): boxes of box_rows rows x 64 dims of one head, 128-byte swizzle, zero
+// fill past the last row. A head count of 1 ignores head_stride.
+cudaError_t make_tmap_heads(CUtensorMap* tm, const void* base, long long rows, int heads, long long tok_stride,
+                            long long head_stride, int box_rows) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return cudaErrorNotSupported;
+  if (tok_stride <= 0 || (heads > 1 && head_stride <= 0)) return cudaErrorInvalidValue;
+  const cuuint64_t dims[3] = {128, (cuuint64_t)(rows > 0 ? rows : 1), (cuuint64_t)(heads > 0 ? heads : 1)};
+  const cuuint64_t strides[2] = {(cuuint64_t)tok_stride * 2,
+                                 (cuuint64_t)(heads > 1 ? head_stride : tok_stride) * 2};
+  const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult res = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 static int sm_count() {
   static int cached[64] = {0};
   int dev = 0;
