@@ -1,5 +1,7 @@
 // Stage 1 (pre-LLM, Sec. 4.1): textual-relevance scores (Eq. 4-5), selection (Sec. 3.1 ratio
 // split or Eq. 6-7 fused score) and gather of the kept feature rows.
+#include <cmath>
+
 #include "pre_llm.cuh"
 #include "sm100.cuh"
 
@@ -55,6 +57,7 @@ struct ScoreLaunch {
   int t_slice_bytes;  // bytes of one slice of T in a slot (M rounded up to 16 rows x 128)
   int acc_cols;       // TMEM columns of one accumulator (power of two >= 32)
   int mld;            // row length of a partial G (max M rounded up to 4)
+  int bound[kMaxScoreCtas + 1];   // CTA c takes stage units [bound[c], bound[c + 1])
 };
 
 // Floats of one partial-sum slot: G [128][mld], then ||z||^2 [128].
@@ -67,9 +70,15 @@ struct SubTile {
   int slot;         // -1: the whole tile; 0 / 1: partial sums of the range's first / last tile
 };
 
-// Scoring CTA whose stage units [W c / P, W (c + 1) / P) contain unit u (32-bit arithmetic:
-// W * P < 2^31 by construction).
-__host__ __device__ inline int score_cta_of(int u, int W, int P) { return (int)(((long long)(u + 1) * P - 1) / W); }
+// Scoring CTA whose stage units [bound[c], bound[c + 1]) contain unit u.
+inline int score_cta_of(int u, const int* bound, int P) {
+  int lo = 0, hi = P - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (bound[mid] <= u) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
 
 // Calls f(segment) for the tiles of stage units [u0, u1) in order; f returns false to stop.
 template <class F>
@@ -113,8 +122,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   const int d = a.d;
   const int nk = (d + kChunk - 1) / kChunk;                 // 64-column slices
   const int nzs = (nk + kZSlices - 1) / kZSlices;           // Z stages per tile
-  const long long W = (long long)meta.total_tiles * nzs, P = gridDim.x;
-  const long long u0 = W * blockIdx.x / P, u1 = W * (blockIdx.x + 1) / P;
+  const long long u0 = L.bound[blockIdx.x], u1 = L.bound[blockIdx.x + 1];
   const bool ragged = (d % (kChunk * kZSlices)) != 0;       // last Z stage copied slice by slice
   // word 1 of the workspace header, when set, replaces the 2 s limit of every wait (microseconds)
   const uint32_t lim_us = __ldcg(a.err + 1);
@@ -714,6 +722,47 @@ static int score_grid(const PreMeta& meta, int d, int reserve) {
   return P < 1 ? 1 : (int)P;
 }
 
+// Unit boundaries of a scoring grid of P CTAs: every CTA takes about the same time. On GB300
+// a stage costs the same up to 64 text rows and then grows with the MMA's N = M rounded up to
+// 16: per-CTA times of a ragged batch (M from 8 to 256, all CTAs streaming at once) give 2.4 us
+// per stage at N <= 64, 2.8 us at N = 128 and 4.0 us at N = 256. A 64-column slice is weighted
+// 256 + 0.8 max(N - 64, 0) + 0.3 max(N - 128, 0), so that batches with N <= 64 throughout split
+// evenly.
+static void score_bounds(const PreMeta& meta, int d, int P, int* bound) {
+  const int nk = (d + kChunk - 1) / kChunk;
+  const int nzs = (nk + kZSlices - 1) / kZSlices;
+  const int W = meta.total_tiles * nzs;
+  double total = 0.0;
+  for (int b = 0; b < meta.B; ++b) {
+    const PreReq& r = meta.r[b];
+    const int tn = (r.m + 15) & ~15;
+    const double slice = 256.0 + 0.8 * (tn > 64 ? tn - 64 : 0) + 0.3 * (tn > 128 ? tn - 128 : 0);
+    total += slice * nk * ((r.n + kTileRows - 1) / kTileRows);
+  }
+  bound[0] = 0;
+  bound[P] = W;
+  int c = 1;
+  double acc = 0.0;   // cost of the tiles before tile t
+  for (int b = 0, t = 0; b < meta.B && c < P; ++b) {
+    const PreReq& r = meta.r[b];
+    const int tn = (r.m + 15) & ~15;
+    const double slice = 256.0 + 0.8 * (tn > 64 ? tn - 64 : 0) + 0.3 * (tn > 128 ? tn - 128 : 0), tile = slice * nk;
+    for (int row0 = 0; row0 < r.n && c < P; row0 += kTileRows, ++t) {
+      while (c < P && total * c / P <= acc + tile) {
+        // the first stage boundary of the tile at or past CTA c's share
+        int j = (int)std::ceil((total * c / P - acc) / (slice * kZSlices) - 1e-9);
+        j = j < 0 ? 0 : (j > nzs ? nzs : j);
+        bound[c++] = t * nzs + j;
+      }
+      acc += tile;
+    }
+  }
+  for (; c < P; ++c) bound[c] = W;
+  // every CTA at least one unit
+  for (c = 1; c < P; ++c) bound[c] = bound[c] > bound[c - 1] + 1 ? bound[c] : bound[c - 1] + 1;
+  for (c = P - 1; c >= 1; --c) bound[c] = bound[c] < bound[c + 1] - 1 ? bound[c] : bound[c + 1] - 1;
+}
+
 // pdl: the preceding grid of the stream is the pre-pass, which this grid may overlap.
 cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, long long z_rows, cudaStream_t st,
                              bool pdl) {
@@ -739,7 +788,9 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   auto kernel = a.action == kActFpsSeed ? pre_score_kernel<true> : pre_score_kernel<false>;
   e = ensure_dynamic_smem(kernel, smem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(kernel, dim3(score_grid(meta, a.d, a.score_reserve)), dim3(kScoreThreads), smem, st, pdl, tmZ3,
+  const int P = score_grid(meta, a.d, a.score_reserve);
+  score_bounds(meta, a.d, P, L.bound);
+  return launch_kernel(kernel, dim3(P), dim3(kScoreThreads), smem, st, pdl, tmZ3,
                        tmZ2, meta, a, L);
 }
 
@@ -756,21 +807,22 @@ cudaError_t launch_pre_finish(const PreMeta& meta, const PreArgs& a, int max_m, 
   if (scored && meta.total_tiles > 0) {
     const int nzs = ((a.d + kChunk - 1) / kChunk + kZSlices - 1) / kZSlices;
     const int P = score_grid(meta, a.d, a.score_reserve);
-    const int W = meta.total_tiles * nzs;
+    static thread_local int bound[kMaxScoreCtas + 1];
+    score_bounds(meta, a.d, P, bound);
     int b = 0;
     for (int c = 1; c < P; ++c) {
-      const int bc = (int)((long long)W * c / P);
+      const int bc = bound[c];
       if (bc % nzs == 0) continue;
       const int t = bc / nzs, t_start = t * nzs;
-      const int c0 = score_cta_of(t_start, W, P);
+      const int c0 = score_cta_of(t_start, bound, P);
       if (c0 != c - 1) continue;                     // the tile's first boundary lists it
       while (b + 1 < meta.B && meta.r[b + 1].tile_off <= t) ++b;
       FinJob& j = fm.job[fm.njobs++];
       j.tile = t;
       j.b = b;
       j.c0 = c0;
-      j.nc = score_cta_of(t_start + nzs - 1, W, P) - c0 + 1;
-      j.slot0 = (int)((long long)W * c0 / P) < t_start ? 1 : 0;
+      j.nc = score_cta_of(t_start + nzs - 1, bound, P) - c0 + 1;
+      j.slot0 = bound[c0] < t_start ? 1 : 0;
       ++jobs_of[b];
     }
   }
