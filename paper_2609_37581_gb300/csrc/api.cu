@@ -22,6 +22,7 @@ cudaError_t launch_pre_finish(const PreMeta&, const PreArgs&, int max_m, int max
 cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
+cudaError_t launch_fps_gram(const FpsMeta&, const FpsArgs&, int tiles, cudaStream_t);
 cudaError_t launch_cls_saliency(const ClsMeta&, const ClsArgs&, int dh, int max_n, cudaStream_t);
 cudaError_t launch_in_head_stats(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
 cudaError_t launch_in_token_score(const InMeta&, const InArgs&, int max_k1, cudaStream_t);
@@ -151,7 +152,7 @@ constexpr size_t kStatusBytes = 256;
 
 struct PreWs {
   size_t counters, sal, t_rinv, part, s_t, s_fused, keys, flags;
-  size_t fps_zero, fps_prow, fps_rinv, fps_maxcos, fps_ub, fps_stamp, fps_picks, end;
+  size_t fps_zero, fps_prow, fps_rinv, fps_maxcos, fps_ub, fps_stamp, fps_picks, fps_pooln, fps_pool, fps_gram, end;
 };
 
 // Scratch keys / flags hold sum n entries plus 16-byte alignment padding per request;
@@ -161,8 +162,16 @@ struct PreWs {
 // fps_* regions serve farthest point sampling (Sec. 3.1) when the call asks for it: a
 // 256-byte zero block, copies of the pivot rows (d columns), 1 / ||z|| of the pivots and the
 // draws (all indexed like kept_idx), and the largest pivot cosine, bound and stamp of every row.
+// Rows of the pool-cosine matrix a request with k1 kept tokens may need for its diversity
+// draws (K_d <= K1): the automatic pool, at most kFpsMaxPoolBig, rounded up to whole tiles.
+inline int fps_gram_ld(int k1) {
+  if (k1 <= 0) return 0;
+  const int w = fps_auto_pool(k1);
+  return ((w < kFpsMaxPoolBig ? w : kFpsMaxPoolBig) + kFpsGramTile - 1) / kFpsGramTile * kFpsGramTile;
+}
+
 PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1 = 0, int max_k1 = 0,
-             int d = 0) {
+             int d = 0, long long fps_pool = 0, long long fps_gram = 0) {
   PreWs w;
   const size_t padded = (size_t)total_n + 4 * (size_t)kMaxChunk + 4;
   const int max_kr = max_k1 < TREVS_MAX_TEXT_TOKENS ? max_k1 : TREVS_MAX_TEXT_TOKENS;
@@ -184,6 +193,10 @@ PreWs pre_ws(long long total_n, long long total_m, int max_m, long long total_k1
   w.fps_maxcos = o; o = al256(o + 4 * fn);
   w.fps_ub = o;     o = al256(o + 4 * fn);
   w.fps_stamp = o;  o = al256(o + 4 * fn);
+  // pools above kFpsMaxPool: pool sizes, pool rows and their dot products (sum of ld^2)
+  w.fps_pooln = o;  o = al256(o + (fps_gram > 0 ? 4 * (size_t)kMaxChunk : 0));
+  w.fps_pool = o;   o = al256(o + 4 * (size_t)(fps_pool > 0 ? fps_pool : 0));
+  w.fps_gram = o;   o = al256(o + 4 * (size_t)(fps_gram > 0 ? fps_gram : 0));
   w.end = o;
   return w;
 }
@@ -273,6 +286,7 @@ int textual_count(int k1, float ratio) {
 struct PreTotals {
   long long n = 0, m = 0, k1 = 0;
   int max_n = 0, max_m = 0, max_k1 = 0;
+  long long fps_pool = 0, fps_gram = 0;   // room for pools above kFpsMaxPool (fps_gram_ld)
 };
 
 trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
@@ -295,6 +309,9 @@ trevs_status validate_pre_batch(const trevs_pre_batch* bt, PreTotals& t) {
       TREVS_CHECK(r.m >= 0, "request %d: m = %d < 0", b, r.m);
     }
     t.n += r.n; t.m += r.m; t.k1 += r.k1;
+    const long long gl = fps_gram_ld(r.k1);
+    t.fps_pool += gl;
+    t.fps_gram += gl * gl;
     t.max_n = r.n > t.max_n ? r.n : t.max_n;
     t.max_k1 = r.k1 > t.max_k1 ? r.k1 : t.max_k1;
     if (r.n > 0) t.max_m = r.m > t.max_m ? r.m : t.max_m;   // requests without visual rows score nothing
@@ -445,6 +462,12 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     dm.B = 0;
     fm.B = 0;
     int dtiles = 0, max_kr = 0;
+    // pools above kFpsMaxPool keep their cosines in the workspace: then every request of the
+    // launch takes the three-grid form (pool, pool cosines, draws)
+    bool big = false;
+    for (int i = 0; i < meta.B; ++i) big = big || fps_auto_pool(kd_of[i]) > kFpsMaxPool;
+    int pool_off = 0, gt_off = 0;
+    long long gram_off = 0;
     for (int i = 0; i < meta.B; ++i) {
       const int kd = kd_of[i];
       if (kd <= 0) continue;
@@ -456,7 +479,11 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
       dm.r[dm.B++] = PreReq{r.n_off, r.n, r.k1_off, kr, 0, 0, 0, dtiles};
       dtiles += (r.n + kScoreTileRows - 1) / kScoreTileRows;
       max_kr = kr > max_kr ? kr : max_kr;
-      fm.r[fm.B++] = FpsReq{r.n_off, r.n, r.k1_off, kr, kd, lead, r.k1_off, r.k1_off};
+      const int gl = big ? fps_gram_ld(kd) : 0;
+      fm.r[fm.B++] = FpsReq{r.n_off, r.n, r.k1_off, kr, kd, lead, r.k1_off, r.k1_off, pool_off, gl, gt_off, gram_off};
+      pool_off += gl;
+      gt_off += (gl / kFpsGramTile) * (gl / kFpsGramTile);
+      gram_off += (long long)gl * gl;
     }
     dm.total_tiles = dtiles;
     // copies of every request's kept slots (the pivots lead each request's K1 slots)
@@ -492,7 +519,18 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
     f.flags = a.flags; f.keys = a.keys;
     f.picks = reinterpret_cast<int*>(ws + L.fps_picks); f.pick_dist = nullptr;
     f.kept = a.kept; f.pool = 0; f.err = a.err;
-    TREVS_TRY_CUDA(counted(launch_fps(fm, f, ts, true)), "farthest point sampling launch");
+    if (!big) {
+      TREVS_TRY_CUDA(counted(launch_fps(fm, f, ts, true)), "farthest point sampling launch");
+    } else {
+      f.pool_n = reinterpret_cast<int*>(ws + L.fps_pooln);
+      f.pool_idx = reinterpret_cast<int*>(ws + L.fps_pool);
+      f.gram = reinterpret_cast<float*>(ws + L.fps_gram);
+      f.phase = 1;
+      TREVS_TRY_CUDA(counted(launch_fps(fm, f, ts, true)), "diversity pool launch");
+      TREVS_TRY_CUDA(counted(launch_fps_gram(fm, f, gt_off, ts)), "pool cosines launch");
+      f.phase = 2;
+      TREVS_TRY_CUDA(counted(launch_fps(fm, f, ts, true)), "farthest point sampling launch");
+    }
   }
   GatherMeta& g = gm_out ? *gm_out : gm;
   g.njobs = 0;
@@ -1223,17 +1261,20 @@ trevs_status trevs_in_llm_compact(const uint16_t* hidden, int64_t hidden_row_str
 
 size_t trevs_pre_llm_varlen_workspace_size(const trevs_pre_batch* batch) {
   if (!batch || batch->B <= 0 || !batch->reqs) return 0;
-  long long n = 0, m = 0, k1 = 0;
+  long long n = 0, m = 0, k1 = 0, fpool = 0, fgram = 0;
   int max_m = 0, max_k1 = 0;
   for (int b = 0; b < batch->B; ++b) {
     const trevs_pre_request& r = batch->reqs[b];
     n += r.n > 0 ? r.n : 0;
     m += r.m > 0 ? r.m : 0;
     k1 += r.k1 > 0 ? r.k1 : 0;
+    const long long gl = fps_gram_ld(r.k1);
+    fpool += gl;
+    fgram += gl * gl;
     if (r.n > 0 && r.m > max_m) max_m = r.m;
     if (r.k1 > max_k1) max_k1 = r.k1;
   }
-  return pre_ws(n, m, max_m, k1, max_k1, batch->d).end;
+  return pre_ws(n, m, max_m, k1, max_k1, batch->d, fpool, fgram).end;
 }
 
 size_t trevs_in_llm_varlen_workspace_size(const trevs_in_batch* batch) {
@@ -1262,7 +1303,7 @@ trevs_status trevs_pre_llm_varlen(const trevs_pre_batch* batch, const trevs_pre_
   if (s != TREVS_OK || batch->B == 0) return s;
   s = validate_diversity(batch, prm);
   if (s != TREVS_OK) return s;
-  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d, t.fps_pool, t.fps_gram);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_batch(batch, prm, reinterpret_cast<uint8_t*>(workspace), L, (cudaStream_t)stream);
@@ -1283,7 +1324,7 @@ trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, const trev
   if (batch->B > kMaxChunk) return fail(TREVS_ERR_UNSUPPORTED, "B = %d > %d requests", batch->B, kMaxChunk);
   s = validate_diversity(batch, prm);
   if (s != TREVS_OK) return s;
-  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d);
+  const PreWs L = pre_ws(t.n, t.m, t.max_m, t.k1, t.max_k1, batch->d, t.fps_pool, t.fps_gram);
   s = check_ws(workspace, workspace_bytes, L.end);
   if (s != TREVS_OK) return s;
   return run_pre_chunk(batch, prm, 0, batch->B, 0, 0, 0, reinterpret_cast<uint8_t*>(workspace), L,
@@ -1316,7 +1357,7 @@ trevs_status trevs_prune_varlen(const trevs_pre_batch* pre, const trevs_pre_para
   if (s != TREVS_OK) return s;
   s = validate_diversity(pre, prm);
   if (s != TREVS_OK) return s;
-  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1, pre->d);
+  const PreWs LP = pre_ws(tp.n, tp.m, tp.max_m, tp.k1, tp.max_k1, pre->d, tp.fps_pool, tp.fps_gram);
   const size_t pre_bytes = pre->B > 0 ? al256(LP.end) : 0;
   const InWs LI = in_ws(ti.l, ti.k1, ti.lk1, in->B > 0 ? in->Hq : 0, in->B);
   const size_t need = pre_bytes + (in->B > 0 ? LI.end : 0);

@@ -124,6 +124,18 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
   float* pdist = reinterpret_cast<float*>(pool + kFpsMaxPool);
   float* prinv = pdist + kFpsMaxPool;
   int* ppick = reinterpret_cast<int*>(prinv + kFpsMaxPool);
+  const int phase = a.phase;
+  const int cap = phase == 0 ? kFpsMaxPool : min(kFpsMaxPoolBig, r.gram_ld);
+  const float* ggram = phase == 2 ? a.gram + r.gram_off : nullptr;   // pool dot products (phase 2)
+  if (phase == 1) {
+    pool = a.pool_idx + r.pool_off;          // the pool goes to the workspace
+  } else if (phase == 2) {
+    // the staging ring is not used: the pool's arrays take its place
+    pool = reinterpret_cast<int*>(stage);
+    pdist = reinterpret_cast<float*>(pool + kFpsMaxPoolBig);
+    prinv = pdist + kFpsMaxPoolBig;
+    ppick = reinterpret_cast<int*>(prinv + kFpsMaxPoolBig);
+  }
   pdl_wait();   // the pivots and their cosines come from the preceding grids
   if (kd <= 0 || n <= 0) return;
   const __nv_bfloat16* Zb = a.Z + (long long)r.n_off * a.z_stride;
@@ -153,15 +165,17 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
   __syncthreads();
   const int ncand = s_n;
   const int t0 = r.lead;       // draws made before the loop
-  int W = a.pool > 0 ? a.pool : max(2 * kd, kd + 32);
-  W = min(W, min(ncand, kFpsMaxPool));   // 0 only when the lead draw is the only one
+  int W = a.pool > 0 ? a.pool : fps_auto_pool(kd);
+  W = min(W, min(ncand, cap));   // 0 only when the lead draw is the only one
   if (ncand < kd - t0) {   // the host checks K_d <= N - K_r; nothing to draw from otherwise
-    if (tid == 0) atomicOr(a.err, 2u);
+    if (tid == 0 && phase != 2) atomicOr(a.err, 2u);
     return;
   }
 
   // ---- the pool
-  if (n <= 512) fps_pool_reg<1>(n, flags, mc, seeded, W, pool, sh.rs);
+  if (phase == 2) {
+    for (int p = tid; p < W; p += nthr) pool[p] = __ldcg(a.pool_idx + r.pool_off + p);
+  } else if (n <= 512) fps_pool_reg<1>(n, flags, mc, seeded, W, pool, sh.rs);
   else if (n <= 1024) fps_pool_reg<2>(n, flags, mc, seeded, W, pool, sh.rs);
   else if (n <= kRegSelMaxN) fps_pool_reg<8>(n, flags, mc, seeded, W, pool, sh.rs);
   else {
@@ -177,27 +191,43 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
   __syncthreads();
 
   // ---- bounds of the candidates outside the pool (exact for the pivots and the lead draw)
-  if (t0 && tid == 0) {
-    picks[0] = 0;
-    if (a.pick_dist) a.pick_dist[r.pick_off] = INFINITY;
+  if (phase != 2) {
+    if (t0 && tid == 0) {
+      picks[0] = 0;
+      if (a.pick_dist) a.pick_dist[r.pick_off] = INFINITY;
+    }
+    for (int i = tid; i < n; i += nthr) {
+      const bool cand = flags[i] == 0;
+      stamp[i] = cand ? t0 : -1;
+      ub[i] = cand ? (seeded ? 1.f - __ldcg(mc + i) : INFINITY) : 0.f;
+    }
+    __syncthreads();
   }
-  for (int i = tid; i < n; i += nthr) {
-    const bool cand = flags[i] == 0;
-    stamp[i] = cand ? t0 : -1;
-    ub[i] = cand ? (seeded ? 1.f - __ldcg(mc + i) : INFINITY) : 0.f;
+  if (phase == 1) {   // the pool's own stamps; the cosines and draws follow in later grids
+    for (int p = tid; p < W; p += nthr) stamp[pool[p]] = -1;
+    if (tid == 0) a.pool_n[blockIdx.x] = W;
+    return;
   }
-  __syncthreads();
   for (int p = tid; p < W; p += nthr) {
     const int i = pool[p];
-    stamp[i] = -1;
+    if (phase == 0) stamp[i] = -1;
     pdist[p] = seeded ? 1.f - __ldcg(mc + i) : INFINITY;
     ppick[p] = 0;
+  }
+
+  // ---- phase 2: 1 / ||z|| of the pool rows from the diagonal of their dot products
+  if (phase == 2) {
+    __syncthreads();
+    for (int p = tid; p < W; p += nthr) {
+      const float gpp = __ldcg(ggram + (long long)p * r.gram_ld + p);
+      prinv[p] = gpp > 0.f ? 1.0f / sqrtf(gpp) : 0.f;
+    }
   }
 
   // ---- cosines within the pool: G = Z_pool Z_pool^T (bf16 mma.sync, fp32), then normalised.
   // The pool rows stream through a ring of S chunks of 256 columns (S = 2..4 as W allows),
   // so that 64-96 KB are in flight while the block computes.
-  if (W > 0) {
+  if (phase == 0 && W > 0) {
     const int W16 = (W + 15) & ~15, nmt = W16 >> 4, nblk = nmt * nmt;
     const int slice_bytes = W16 * 128, chunk_bytes = kFpsSlices * slice_bytes;
     const int S = min(4, kFpsRingBytes / chunk_bytes);
@@ -325,7 +355,13 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
           ppick[gp] = 1;
           flags[gi] = 2;
         }
-        for (int p = tid; p < W; p += nthr) pdist[p] = fminf(pdist[p], 1.f - gram[gp * kFpsGramLd + p]);
+        if (phase == 0) {
+          for (int p = tid; p < W; p += nthr) pdist[p] = fminf(pdist[p], 1.f - gram[gp * kFpsGramLd + p]);
+        } else {
+          const float* grow = ggram + (long long)gp * r.gram_ld;
+          const float rg = prinv[gp];
+          for (int p = tid; p < W; p += nthr) pdist[p] = fminf(pdist[p], 1.f - __ldcg(grow + p) * rg * prinv[p]);
+        }
         __syncthreads();
         break;
       }
@@ -371,9 +407,101 @@ __global__ void __launch_bounds__(kFpsThreads, 1) fps_kernel(const __grid_consta
   }
 }
 
+// Dot products of the pool rows of the requests drawing from pools above kFpsMaxPool, for
+// phase 2: one block of four warps per 64 x 64 tile of a request's W x W matrix. The two row
+// sets stream through shared memory in 64-column chunks (cp.async, two stages, 128-byte
+// swizzled rows); each warp takes 16 rows x 64 columns with mma.sync (bf16 in, fp32 out).
+constexpr int kGramThreads = 128;
+constexpr int kGramChunk = 64;                                  // columns per staged chunk
+constexpr int kGramStage = 2 * kFpsGramTile * kGramChunk * 2;   // rows of both sets: 16 KB
+
+__global__ void __launch_bounds__(kGramThreads) fps_gram_kernel(const __grid_constant__ FpsMeta meta,
+                                                                const FpsArgs a) {
+  __shared__ __align__(128) uint8_t stage[2 * kGramStage];
+  pdl_wait();   // the pools come from the preceding grid
+  const int b = find_request(meta.B, blockIdx.x, [&](int i) { return meta.r[i].gt_off; });
+  const FpsReq& r = meta.r[b];
+  const int nt = r.gram_ld / kFpsGramTile;
+  const int t = blockIdx.x - r.gt_off;
+  const int ti = t / nt, tj = t - ti * nt;
+  const int W = __ldcg(a.pool_n + b);
+  if (ti * kFpsGramTile >= W || tj * kFpsGramTile >= W) return;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int* pool = a.pool_idx + r.pool_off;
+  const __nv_bfloat16* Zb = a.Z + (long long)r.n_off * a.z_stride;
+  const int d = a.d, nch = (d + kGramChunk - 1) / kGramChunk;
+  const uint32_t sbase = smem_u32(stage);
+  // row x of a chunk: set 0 (rows ti), set 1 (rows tj); 8 pieces of 16 bytes each
+  auto load_chunk = [&](int ch, int slot) {
+    for (int idx = tid; idx < 2 * kFpsGramTile * 8; idx += kGramThreads) {
+      const int row = idx >> 3, c = idx & 7, set = row / kFpsGramTile, rr = row - set * kFpsGramTile;
+      const int p = (set ? tj : ti) * kFpsGramTile + rr;
+      const int col = ch * kGramChunk + c * 8;
+      const bool ok = p < W && col < d;
+      const void* src = ok ? (const void*)(Zb + (long long)__ldcg(pool + p) * a.z_stride + col) : (const void*)a.Z;
+      cp_async16(sbase + slot * kGramStage + row * 128 + (swz(row, c) << 4), src, ok ? 16 : 0);
+    }
+  };
+  float acc[4][2][4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int x = 0; x < 2; ++x)
+#pragma unroll
+      for (int y = 0; y < 4; ++y) acc[j][x][y] = 0.f;
+  load_chunk(0, 0);
+  cp_async_commit();
+  for (int ch = 0; ch < nch; ++ch) {
+    if (ch + 1 < nch) load_chunk(ch + 1, (ch + 1) & 1);
+    cp_async_commit();
+    cp_async_wait<1>();
+    __syncthreads();
+    const uint32_t A = sbase + (ch & 1) * kGramStage, B = A + kFpsGramTile * 128;
+#pragma unroll
+    for (int ks = 0; ks < kGramChunk / 16; ++ks) {
+      uint32_t af[4];
+      const int ar = warp * 16 + (lane & 15), ac = 2 * ks + (lane >> 4);
+      ldmatrix_x4(A + ar * 128 + (swz(ar, ac) << 4), af[0], af[1], af[2], af[3]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {   // 16-column block j of the tile
+        const int mi = lane >> 3;
+        const int br = j * 16 + 8 * (mi >> 1) + (lane & 7), bc = 2 * ks + (mi & 1);
+        uint32_t b0, b1, b2, b3;
+        ldmatrix_x4(B + br * 128 + (swz(br + kFpsGramTile, bc) << 4), b0, b1, b2, b3);
+        mma_bf16_16816(acc[j][0], af, b0, b1);
+        mma_bf16_16816(acc[j][1], af, b2, b3);
+      }
+    }
+    __syncthreads();   // the slot is refilled next
+  }
+  cp_async_wait<0>();
+  const int g = lane >> 2, t4 = lane & 3;
+  float* out = a.gram + r.gram_off;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int x = 0; x < 2; ++x) {
+      const int col = tj * kFpsGramTile + j * 16 + 8 * x + 2 * t4;
+      const int r0 = ti * kFpsGramTile + warp * 16 + g;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int row = r0 + 8 * h;
+        if (row < W) {
+          if (col < W) out[(long long)row * r.gram_ld + col] = acc[j][x][2 * h];
+          if (col + 1 < W) out[(long long)row * r.gram_ld + col + 1] = acc[j][x][2 * h + 1];
+        }
+      }
+    }
+}
+
 cudaError_t launch_fps(const FpsMeta& meta, const FpsArgs& a, cudaStream_t st, bool pdl) {
   if (meta.B == 0) return cudaSuccess;
   return launch_kernel(fps_kernel, dim3(meta.B), dim3(kFpsThreads), kFpsSmem + 128, st, pdl, meta, a);
+}
+
+cudaError_t launch_fps_gram(const FpsMeta& meta, const FpsArgs& a, int tiles, cudaStream_t st) {
+  if (meta.B == 0 || tiles == 0) return cudaSuccess;
+  return launch_kernel(fps_gram_kernel, dim3(tiles), dim3(kGramThreads), 0, st, true, meta, a);
 }
 
 }  // namespace trevs
