@@ -442,6 +442,7 @@ trevs_status run_pre_chunk(const trevs_pre_batch* bt, const trevs_pre_params& pr
   a.tau_v = prm.tau_v; a.tau_t = prm.tau_t; a.lambda = prm.lambda; a.eps = prm.eps;
   a.action = kActSelect;
   a.score_reserve = reserve;
+  a.big_sel = 1;
   TREVS_TRY_CUDA(counted(launch_pre_saliency(meta, a, max_n, true, st)), "pre-pass launch");
   if (before_score) TREVS_TRY_CUDA(cudaEventRecord(before_score, st), "event before scoring");
   TREVS_TRY_CUDA(counted(launch_pre_score(meta, a, max_m, no, st, true)), "pre_score launch");

@@ -544,7 +544,28 @@ __global__ void __launch_bounds__(kFinishThreads, 1) pre_finish_kernel(const __g
   } else {
     __syncthreads();
   }
+  if (a.big_sel && r.n > kRegSelMaxN) return;   // pre_select_big_kernel selects it
   select_request_512(a, r, jb.b, smem, smem_bytes, sh);
+}
+
+// Selection of the requests above kRegSelMaxN tokens, after the finishing grid: one block of
+// 1,024 threads per request, keys and flags in shared memory (in global memory past its size),
+// so that each pass over the keys takes half as long as with the finishing grid's 512.
+constexpr int kBigSelThreads = 1024;
+struct BigSel {
+  int n;
+  int b[kMaxChunk];
+};
+
+__global__ void __launch_bounds__(kBigSelThreads, 1) pre_select_big_kernel(const __grid_constant__ PreMeta meta,
+                                                                           const __grid_constant__ BigSel bs,
+                                                                           const PreArgs a, int smem_bytes) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ SelShared ss;
+  pdl_wait();   // the finishing grid's s^t rows
+  const int b = bs.b[blockIdx.x];
+  select_request(a, meta.r[b], b, smem, smem_bytes, ss, a.mode == kModeFused && !a.s_fused_given,
+                 a.action == kActSelect);
 }
 
 // Pre-pass, run ahead of the scoring grid. Blocks [0, n_sal): the saliency side of the
@@ -837,8 +858,18 @@ cudaError_t launch_pre_finish(const PreMeta& meta, const PreArgs& a, int max_m, 
   if (fm.njobs == 0) return cudaSuccess;
   for (int i = 0; i < fm.njobs; ++i) fm.job[i].count = per_request ? jobs_of[fm.job[i].b] : 1;
   int smem = 0;   // keys and flags of the block-wide selection, for requests above kRegSelMaxN
-  if (per_request && max_n > kRegSelMaxN && (size_t)max_n * 5 + 16 <= (size_t)160 * 1024) smem = max_n * 5 + 16;
-  return launch_kernel(pre_finish_kernel, dim3(fm.njobs), dim3(kFinishThreads), smem, st, pdl, meta, fm, a, smem);
+  const bool big = per_request && a.big_sel && max_n > kRegSelMaxN;
+  if (per_request && !big && max_n > kRegSelMaxN && (size_t)max_n * 5 + 16 <= (size_t)160 * 1024)
+    smem = max_n * 5 + 16;
+  cudaError_t e = launch_kernel(pre_finish_kernel, dim3(fm.njobs), dim3(kFinishThreads), smem, st, pdl, meta, fm, a,
+                                smem);
+  if (e != cudaSuccess || !big) return e;
+  static thread_local BigSel bs;
+  bs.n = 0;
+  for (int b = 0; b < meta.B; ++b)
+    if (meta.r[b].n > kRegSelMaxN) bs.b[bs.n++] = b;
+  const int sbig = (size_t)max_n * 5 + 16 <= (size_t)200 * 1024 ? max_n * 5 + 16 : 0;
+  return launch_kernel(pre_select_big_kernel, dim3(bs.n), dim3(kBigSelThreads), sbig, st, true, meta, bs, a, sbig);
 }
 
 // Workspace bytes of the partial sums for up to max_m text rows.

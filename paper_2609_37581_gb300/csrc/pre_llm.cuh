@@ -40,6 +40,7 @@ struct PreArgs {
   int s_fused_given;   // select kernel: s_fused already holds Eq. 7 scores
   int seed_merge;      // kActFpsSeed: s_t already holds the largest cosine to earlier pivots
                        // (a pass over further pivot columns keeps the max)
+  int big_sel;         // requests above kRegSelMaxN are selected by pre_select_big_kernel
 };
 
 // Saliency side of the selection, which depends on inputs only. Ratio mode: the rule for
