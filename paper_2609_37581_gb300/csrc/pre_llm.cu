@@ -35,7 +35,11 @@ namespace trevs {
 //
 // Warp roles: 0 = TMA producer (Z), 1 = TMEM owner and MMA issuer, 2..3 = T copies,
 // 4..7 = epilogue (warp w reads TMEM lanes 32*(w%4) .. +31), 8..15 = Z norms (two threads
-// per row, two slices each).
+// per row, two slices each). When every request has more than 112 text rows (kTHeavy), a
+// stage brings in as much T as Z and the MMA issuer waits on T: warps 8..11 copy T as well,
+// and warps 12..15 take the Z norms, one thread per row. (Measured on GB300: the 2 x 16,384
+// batch with 128 text rows drops from 111.9 to 105.6 us per call; batches with at most 64
+// text rows lose 5-8 us the same way, as their norms, not T, hold the stages.)
 
 constexpr int kTileRows = kScoreTileRows;
 constexpr int kChunk = 64;                     // d' columns per slice (one 128-byte swizzle row)
@@ -46,8 +50,8 @@ constexpr int kZStageBytes = kTileRows * kZSlices * 128;
 constexpr int kMaxZStages = 4;
 constexpr int kMaxTSlots = 8;
 constexpr int kScoreThreads = 512;
-constexpr int kZNormWarps = 8;
-constexpr int kTCopyThreads = 64;
+template <bool kTHeavy> constexpr int kZNormWarps = kTHeavy ? 4 : 8;
+template <bool kTHeavy> constexpr int kTCopyThreads = kTHeavy ? 192 : 64;
 constexpr int kRingBudget = 200 * 1024;
 
 struct ScoreLaunch {
@@ -100,7 +104,7 @@ __device__ __forceinline__ void for_each_subtile(const PreMeta& meta, int nzs, l
 
 // kSeed: the "text" rows are the pivot rows of Z (gathered beforehand) and each row's output
 // is the largest cosine to them, unrectified (the distances of farthest point sampling, Sec. 3.1).
-template <bool kSeed>
+template <bool kSeed, bool kTHeavy>
 __global__ void __launch_bounds__(kScoreThreads, 1)
     pre_score_kernel(const __grid_constant__ CUtensorMap tmZ3, const __grid_constant__ CUtensorMap tmZ2,
                      const __grid_constant__ PreMeta meta, const PreArgs a, const ScoreLaunch L) {
@@ -133,16 +137,16 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < SZ; ++s) {
       mbar_init(smem_u32(&zfull[s]), 1);
-      mbar_init(smem_u32(&zempty[s]), 1 + kZNormWarps);   // MMA commit + the Z-norm warps
+      mbar_init(smem_u32(&zempty[s]), 1 + kZNormWarps<kTHeavy>);   // MMA commit + the Z-norm warps
     }
     for (int s = 0; s < ST; ++s) {
-      mbar_init(smem_u32(&tfull[s]), kTCopyThreads);      // the copy lanes, once their copies land
+      mbar_init(smem_u32(&tfull[s]), kTCopyThreads<kTHeavy>);      // the copy lanes, once their copies land
       mbar_init(smem_u32(&tempty[s]), 1);                 // MMA commit
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&acc_full[i]), 1);
       mbar_init(smem_u32(&acc_empty[i]), 4);              // the epilogue warps
-      mbar_init(smem_u32(&norm_full[i]), kZNormWarps);
+      mbar_init(smem_u32(&norm_full[i]), kZNormWarps<kTHeavy>);
       mbar_init(smem_u32(&norm_empty[i]), 4);
     }
     mbar_init(smem_u32(&mma_drain), 1);
@@ -247,11 +251,11 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         mbar_wait(smem_u32(&mma_drain), 0, &no_abort, 500000000ull);
       }
     }
-  } else if (warp < 4) {
+  } else if (warp < 4 || (kTHeavy && warp >= 8 && warp < 12)) {
     // T copies: the slices of the next slot from the request's M text rows, piece p = 16
     // bytes (row p / 8, 16-byte column p % 8 of a slice), swizzled like a TMA
     // 128-byte-swizzle box; slice c of a slot lies t_slice_bytes after slice c - 1
-    const int ct = tid - 64;
+    const int ct = warp < 4 ? tid - 64 : 64 + (tid - 256);
     int gt = 0;
     for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
       const PreReq& r = meta.r[st.b];
@@ -270,7 +274,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
           for (int c = 0; c < nsl; ++c) {
             const int kc = zs * kZSlices + c0 + c;
             const uint32_t Bc = B + c * L.t_slice_bytes;
-            for (int p = ct; p < pieces; p += kTCopyThreads) {
+            for (int p = ct; p < pieces; p += kTCopyThreads<kTHeavy>) {
               const int row = p >> 3, q = p & 7;
               const int col = kc * kChunk + q * 8;
               const uint8_t* src = tsrc + ((long long)row * a.t_stride + (col < d ? col : 0)) * 2;
@@ -283,11 +287,12 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
       return true;
     });
     cp_async_wait_all();
-  } else if (warp >= 8) {
+  } else if (warp >= (kTHeavy ? 12 : 8)) {
     // Z norms: thread zt owns row zt % 128 of every sub-tile, slices 2 (zt / 128) and + 1 of
-    // every stage
-    const int zt = tid - 256;
-    const int row = zt & (kTileRows - 1), half = zt >> 7;
+    // every stage (with kTHeavy, all four slices)
+    const int zt = tid - (kTHeavy ? 384 : 256);
+    const int row = zt & (kTileRows - 1), half = kTHeavy ? 0 : zt >> 7;
+    constexpr int kSl = kTHeavy ? kZSlices : 2;   // slices of a stage per thread
     int gz = 0, j = 0;
     for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
       const int buf = j & 1, use = j >> 1;
@@ -303,7 +308,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
           const uint8_t* rowp = smem + s * kZStageBytes + (row >> 3) * kZBoxBytes + (row & 7) * 128;
           const int ncols = min(kZSlices * kChunk, d - zs * kZSlices * kChunk);   // columns of this stage
 #pragma unroll
-          for (int c = 2 * half; c < 2 * half + 2; ++c) {
+          for (int c = kSl * half; c < kSl * half + kSl; ++c) {
 #pragma unroll
             for (int qq = 0; qq < 8; ++qq) {
               if (c * kChunk + qq * 8 < ncols)   // d' is a multiple of 8: whole 16-byte pieces
@@ -319,6 +324,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         return false;
       }
       zsq_s[buf][half][row] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      if (kTHeavy) zsq_s[buf][1][row] = 0.f;
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&norm_full[buf]));
       ++j;
@@ -806,7 +812,11 @@ cudaError_t launch_pre_score(const PreMeta& meta, const PreArgs& a, int max_m, l
   if (e != cudaSuccess) return e;
   e = make_tmap(&tmZ2, a.Z, z_rows, a.d, a.z_stride, kZBoxRows);
   if (e != cudaSuccess) return e;
-  auto kernel = a.action == kActFpsSeed ? pre_score_kernel<true> : pre_score_kernel<false>;
+  bool heavy = true;   // every request has more than 112 text rows
+  for (int b = 0; b < meta.B; ++b)
+    if (meta.r[b].n > 0 && meta.r[b].m <= 112) heavy = false;
+  auto kernel = a.action == kActFpsSeed ? (heavy ? pre_score_kernel<true, true> : pre_score_kernel<true, false>)
+                                        : (heavy ? pre_score_kernel<false, true> : pre_score_kernel<false, false>);
   e = ensure_dynamic_smem(kernel, smem);
   if (e != cudaSuccess) return e;
   const int P = score_grid(meta, a.d, a.score_reserve);

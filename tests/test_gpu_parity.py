@@ -122,7 +122,8 @@ def test_full_sequence_softmax_stage2(k1, l):
     assert tally.stage2_near_ties <= 1, tally
 
 
-@pytest.mark.parametrize("d,m", [(200, (5, 17, 128, 64)), (512, (128, 100, 1, 33)), (576, (64, 64, 64, 64))])
+@pytest.mark.parametrize("d,m", [(200, (5, 17, 128, 64)), (512, (128, 100, 1, 33)), (576, (64, 64, 64, 64)),
+                                 (512, (128, 200, 113, 256))])
 def test_tiles_split_between_scoring_ctas(d, m):
     """Several 128-row tiles per scoring CTA, tiles split between CTAs, odd tile counts, text
     lengths from 1 to 128 and a partial last slice of d'."""
