@@ -678,6 +678,16 @@ __device__ __forceinline__ void bf16_sq_acc8(uint4 v, float (&acc)[4]) {
   }
 }
 
+// The same with packed fp32 FMAs (sm_100 family): eight partial sums in four pairs.
+__device__ __forceinline__ void bf16_sq_acc8x2(uint4 v, float2 (&acc)[4]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 e = make_float2(__uint_as_float(w[j] << 16), __uint_as_float(w[j] & 0xFFFF0000u));
+    acc[j] = __ffma2_rn(e, e, acc[j]);
+  }
+}
+
 // Block-wide min of the non-zero keys and max of all keys (key 0 marks an excluded entry).
 __device__ inline void block_key_range(uint32_t lo, uint32_t hi, SelShared& s, uint32_t& lo_out, uint32_t& hi_out) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;

@@ -296,7 +296,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
     int gz = 0, j = 0;
     for_each_subtile(meta, nzs, u0, u1, [&](const SubTile& st) {
       const int buf = j & 1, use = j >> 1;
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      float2 acc2[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       const bool mine = row < st.h;
       for (int zs = st.zs0; zs < st.zs1; ++zs, ++gz) {
         const int s = gz % SZ, it = gz / SZ;
@@ -312,7 +312,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
 #pragma unroll
             for (int qq = 0; qq < 8; ++qq) {
               if (c * kChunk + qq * 8 < ncols)   // d' is a multiple of 8: whole 16-byte pieces
-                bf16_sq_acc8(*reinterpret_cast<const uint4*>(rowp + c * 1024 + (swz(row, qq) << 4)), acc);
+                bf16_sq_acc8x2(*reinterpret_cast<const uint4*>(rowp + c * 1024 + (swz(row, qq) << 4)), acc2);
             }
           }
         }
@@ -323,7 +323,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1)
         s_abort = 1;
         return false;
       }
-      zsq_s[buf][half][row] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      zsq_s[buf][half][row] = ((acc2[0].x + acc2[0].y) + (acc2[1].x + acc2[1].y)) + ((acc2[2].x + acc2[2].y) + (acc2[3].x + acc2[3].y));
       if (kTHeavy) zsq_s[buf][1][row] = 0.f;
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&norm_full[buf]));
