@@ -211,8 +211,9 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     }
   } else {
     // epilogue warp w: TMEM lane quarter w % 4 (the text rows), column half (w - 2) / 4 of
-    // every chunk
+    // every chunk; a warp whose 32 rows all lie past the request's L only keeps pace
     const int q = warp & 3, row = 32 * q + lane, half = (warp - 2) >> 2;
+    const bool live = 32 * q < L - q0;
     const float sc = a.scale * kLog2e;            // logits in log2 units: exp(x) = exp2(x log2 e)
     // running state over this thread's keys so far (see merge_state)
     float m = -INFINITY, n = 0.f, S = 0.f, M2 = 0.f;
@@ -226,7 +227,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
       tc_fence_after();
       const int nv = min(kStatKeys, K1 - j * kStatKeys) - half * kStatHalf;   // valid keys of this half
       const uint32_t lb = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kStatKeys + half * kStatHalf);
-      if (nv > 0) {
+      if (live && nv > 0) {
         const int nh = min(nv, kStatHalf);
         float v[32], w[32];
         float cm = -INFINITY;
@@ -447,7 +448,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     }
   }
   // epilogue: thread (warp 2..9, lane) owns text row 32 (warp % 4) + lane of the block and
-  // the keys of column half (warp - 2) / 4
+  // the keys of column half (warp - 2) / 4; a warp whose 32 rows all lie past L only keeps pace
   constexpr int kHalf = kScoreKeys / 2;
   float acc[kHalf];
 #pragma unroll
@@ -468,10 +469,12 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         break;
       }
       tc_fence_after();
-      float v[32];
-      tmem_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kScoreKeys + half * kHalf), v);
+      if (32 * q < L - q0) {
+        float v[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * kScoreKeys + half * kHalf), v);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) acc[e] += exp2f(v[e] * sc - rs.x) * rs.y;
+        for (int e = 0; e < 32; ++e) acc[e] += exp2f(v[e] * sc - rs.x) * rs.y;
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&acc_empty[buf]));
