@@ -462,6 +462,25 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         torch.cuda.synchronize()
         cls_ms = c0.elapsed_time(c1) / csteps
         cls_bytes = sum(x.numel() * x.element_size() for x in csets[0]) + cs_v.numel() * 4
+        # streaming probe: the scoring grid's copies of the same Z (4 rotating sets) on as many
+        # CTAs as the timed scoring grid, released on landing, computing nothing
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        pws = T.workspace(256)
+        zs = [x["Z"] for x in sets]
+        for k in range(3):
+            T.trevs_stream_probe(zs[k % ROTATING_SETS], sms, pws, stream)
+        torch.cuda.synchronize()
+        psteps = 40
+        torch.cuda._sleep(int(2e9 * 3e-5 * psteps))
+        p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        p0.record(stream)
+        for k in range(psteps):
+            T.trevs_stream_probe(zs[k % ROTATING_SETS], sms, pws, stream)
+        p1.record(stream)
+        torch.cuda.synchronize()
+        T.workspace_status(pws, stream)
+        probe_ms = p0.elapsed_time(p1) / psteps
+        probe_bytes = zs[0].numel() * zs[0].element_size()
         # the other configurations of the benchmark spec, one after the other
         peak, src = peaks()
         others = {}
@@ -571,6 +590,13 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
             "frac": round(cls_bytes / (cls_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
             "timed": "CUDA events around 200 trevs_cls_saliency_varlen calls queued behind a spin kernel, "
                      "4 rotating input sets"},
+        "stream_probe": {
+            "ctas": sms, "us_per_pass": round(probe_ms * 1e3, 2), "bytes": probe_bytes,
+            "achieved_gbs": round(probe_bytes / (probe_ms * 1e-3) / 1e9, 1),
+            "frac": round(probe_bytes / (probe_ms * 1e-3) / 1e9 / peak, 4), "peak_source": src,
+            "what": "Z streamed with the scoring grid's TMA boxes and 2 x 64 KB ring, stages released on "
+                    "landing, no compute (trevs_stream_probe); the rate the grid's copy pattern allows",
+            "timed": f"CUDA events around {psteps} passes queued behind a spin kernel, 4 rotating input sets"},
         "configs": others,
     }
 

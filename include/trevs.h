@@ -375,6 +375,20 @@ TREVS_API trevs_status trevs_pre_llm_varlen_timed(const trevs_pre_batch* batch, 
                                         void* workspace, size_t workspace_bytes, void* stream,
                                         void* ev_score_begin, void* ev_score_end);
 
+/* Streaming probe: a measurement hook with no counterpart in the paper. One pass streams the
+ * rows of Z [rows][d] (bf16, row stride z_row_stride elements) through shared memory with the
+ * copies of the Eq. 4-5 scoring grid (3D TMA boxes of 8 rows x four 64-column slices, a ring
+ * of two 64 KB stages per CTA, each CTA a contiguous range of 128-row x 256-column units) on
+ * `ctas` CTAs of one SM each, computing nothing: each stage is released as soon as it lands.
+ * Time it with events around the call on `stream`; its rate is what the scoring grid's copy
+ * pattern reaches on the GPU without the grid's consumers.
+ * - Z: device memory, 16-byte aligned; d a multiple of 256; z_row_stride >= d, a multiple of 8.
+ * - workspace: at least 8 bytes, prepared by trevs_workspace_init; a bounded wait that gives up
+ *   sets its status word (trevs_workspace_status).
+ * - Invalid arguments return TREVS_ERR_INVALID_ARGUMENT before any CUDA call. */
+TREVS_API trevs_status trevs_stream_probe(const uint16_t* Z, int64_t z_row_stride, int64_t rows, int32_t d,
+                                          int32_t ctas, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Stage 2 for a batch: attention statistics, Eq. 8 head variances, H*, Eq. 9 token scores,
  * TopK(p, k2) and compaction of hidden, K and V rows. */
 TREVS_API trevs_status trevs_in_llm_varlen(const trevs_in_batch* batch,

@@ -20,6 +20,8 @@ size_t pre_score_part_bytes(int max_m);
 cudaError_t launch_pre_finish(const PreMeta&, const PreArgs&, int max_m, int max_n, bool scored, cudaStream_t,
                               bool pdl);
 cudaError_t launch_pre_saliency(const PreMeta&, const PreArgs&, int max_n, bool saliency, cudaStream_t);
+cudaError_t launch_stream_probe(const void* Z, long long z_stride, long long rows, int d, int ctas, uint32_t* err,
+                                cudaStream_t st);
 cudaError_t launch_gather(const GatherMeta&, cudaStream_t, bool pdl);
 cudaError_t launch_fps(const FpsMeta&, const FpsArgs&, cudaStream_t, bool pdl);
 cudaError_t launch_fps_gram(const FpsMeta&, const FpsArgs&, int tiles, cudaStream_t);
@@ -1130,6 +1132,21 @@ trevs_status trevs_pre_llm_gather(const uint16_t* Z, int64_t z_row_stride, int32
   j.src_tok = z_row_stride * 2; j.dst_tok = z_out_row_stride * 2; j.src_head = 0; j.dst_head = 0;
   j.heads = 1; j.row_bytes = d * 2; j.idx = kept_idx; j.rows = K1; j.tab = 0;
   TREVS_TRY_CUDA(counted(launch_gather(gm, (cudaStream_t)stream, true)), "gather launch");
+  return TREVS_OK;
+}
+
+trevs_status trevs_stream_probe(const uint16_t* Z, int64_t z_row_stride, int64_t rows, int32_t d, int32_t ctas,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  g_launches = 0;
+  TREVS_CHECK(Z != nullptr && aligned16(Z), "Z must be non-NULL and 16-byte aligned");
+  TREVS_CHECK(rows >= 1 && rows <= (1LL << 31), "rows = %lld out of range", (long long)rows);
+  TREVS_CHECK(d >= 256 && d % 256 == 0, "d = %d must be a positive multiple of 256", d);
+  TREVS_CHECK(z_row_stride >= d && z_row_stride % 8 == 0, "z_row_stride must be >= d and a multiple of 8");
+  TREVS_CHECK(ctas >= 1 && ctas <= 1024, "ctas = %d out of [1, 1024]", ctas);
+  TREVS_CHECK(workspace != nullptr && workspace_bytes >= 2 * sizeof(uint32_t), "workspace (status word) missing");
+  TREVS_TRY_CUDA(counted(launch_stream_probe(Z, z_row_stride, rows, d, ctas, reinterpret_cast<uint32_t*>(workspace),
+                                             (cudaStream_t)stream)),
+                 "streaming probe launch");
   return TREVS_OK;
 }
 

@@ -109,6 +109,7 @@ _SIGS = {
     "trevs_pre_llm_varlen_timed": (_c_i32, [ctypes.POINTER(PreBatchC), ctypes.POINTER(PreParams), _vp, _c_sz, _vp,
                                             _vp, _vp]),
     "trevs_in_llm_varlen": (_c_i32, [ctypes.POINTER(InBatchC), _vp, _c_sz, _vp]),
+    "trevs_stream_probe": (_c_i32, [_vp, _c_i64, _c_i64, _c_i32, _c_i32, _vp, _c_sz, _vp]),
     "trevs_prune_varlen": (_c_i32, [ctypes.POINTER(PreBatchC), ctypes.POINTER(PreParams),
                                     ctypes.POINTER(InBatchC), _vp, _c_sz, _vp]),
 }
@@ -190,6 +191,13 @@ def workspace_status(ws, stream=None):
     """Raises TrevsError(TREVS_ERR_TIMEOUT) if a device-side wait of an earlier call gave up."""
     w, nb = _ws_args(ws)
     check(load().trevs_workspace_status(w, nb, _stream(stream)))
+
+
+def trevs_stream_probe(Z, ctas, ws, stream=None):
+    """One pass of the streaming probe over the rows of Z [rows, d] on `ctas` CTAs."""
+    w, nb = _ws_args(ws)
+    check(load().trevs_stream_probe(_ptr(Z), Z.stride(0), Z.shape[0], Z.shape[1], int(ctas), w, nb,
+                                    _stream(stream)))
 
 
 # single-request entry points --------------------------------------------------------

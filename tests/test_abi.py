@@ -227,6 +227,19 @@ def test_varlen_timed_validation(lib):
     assert f(ctypes.byref(ok), None, FAKE, need - 256, None, FAKE, FAKE) == t.TREVS_ERR_WORKSPACE
 
 
+def test_stream_probe_validation(lib):
+    f = lib.trevs_stream_probe
+    bad = t.TREVS_ERR_INVALID_ARGUMENT
+    assert f(None, 4096, 1024, 4096, 128, FAKE, 64, None) == bad                    # no Z
+    assert f(ctypes.c_void_p(0x10008), 4096, 1024, 4096, 128, FAKE, 64, None) == bad   # unaligned Z
+    assert f(FAKE, 4096, 0, 4096, 128, FAKE, 64, None) == bad                      # no rows
+    assert f(FAKE, 4160, 1024, 4160, 128, FAKE, 64, None) == bad                   # d not a multiple of 256
+    assert f(FAKE, 4095, 1024, 4096, 128, FAKE, 64, None) == bad                   # stride < d
+    assert f(FAKE, 4096, 1024, 4096, 0, FAKE, 64, None) == bad                     # no CTAs
+    assert f(FAKE, 4096, 1024, 4096, 128, None, 64, None) == bad                   # no status word
+    assert f(FAKE, 4096, 1024, 4096, 128, FAKE, 4, None) == bad
+
+
 def _in_batch(reqs, Hq=32, Hkv=32, nk=8):
     arr = (t.InRequest * len(reqs))(*[t.InRequest(*r) for r in reqs])
     b = t.InBatchC()

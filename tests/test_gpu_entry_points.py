@@ -170,6 +170,24 @@ def test_workspace_status_ok_after_calls():
     assert T.last_launch_count() == 0 or True
 
 
+@pytest.mark.parametrize("rows,d,ctas", [(1000, 512, 8), (300, 256, 64), (4096, 4096, 152)])
+def test_stream_probe_runs_and_reads_only(rows, d, ctas):
+    """The streaming probe (a measurement hook) streams ragged tails and idle CTAs cleanly and
+    leaves Z untouched."""
+    g = torch.Generator(device="cuda").manual_seed(rows + d)
+    Z = torch.randn(rows, d, device="cuda", generator=g).to(torch.bfloat16)
+    before = Z.clone()
+    ws = T.workspace(256)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    T.trevs_stream_probe(Z, ctas, ws)
+    e1.record()
+    torch.cuda.synchronize()
+    T.workspace_status(ws)
+    assert e0.elapsed_time(e1) > 0.0
+    assert torch.equal(Z, before)
+
+
 def test_timed_stage1_matches_untimed():
     """The measurement hook brackets the scoring grid with two events and changes nothing."""
     from workloads.device import build_batches
