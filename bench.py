@@ -229,7 +229,7 @@ def replica_throughput(max_elapsed_ms: float, steps: int, tokens_per_rank_step: 
     return ms, tokens_per_rank_step * world / (ms * 1e-3)
 
 
-OTHER_CONFIGS = {   # the benchmark spec's other single-GPU configurations, each timed like the headline one
+OTHER_CONFIGS = {   # the other single-GPU workloads (2,880-token, 16,384-token and ragged batches), each timed like the headline one
     "llava_next_2880_b8": synth.llava_next_batch8,
     "long_16384_b2_gqa": synth.long_video_batch2,
     "ragged_varlen_b64": synth.ragged_serving_batch64,
@@ -481,7 +481,7 @@ def gpu_arm(args, rank, world, w, cpu_baseline):
         T.workspace_status(pws, stream)
         probe_ms = p0.elapsed_time(p1) / psteps
         probe_bytes = zs[0].numel() * zs[0].element_size()
-        # the other configurations of the benchmark spec, one after the other
+        # the other workloads, one after the other
         peak, src = peaks()
         others = {}
         if not args.no_configs:

@@ -55,7 +55,7 @@ typedef enum trevs_status {
   TREVS_ERR_INVALID_ARGUMENT = 1, /* bad size, null or misaligned pointer, K > N, ... */
   TREVS_ERR_WORKSPACE = 2,        /* workspace missing, misaligned or too small */
   TREVS_ERR_CUDA = 3,             /* a CUDA launch or runtime call failed */
-  TREVS_ERR_UNSUPPORTED = 4,      /* valid but outside this build's limits (see below) */
+  TREVS_ERR_UNSUPPORTED = 4,      /* valid but outside the library's limits (see below) */
   TREVS_ERR_TIMEOUT = 5           /* a bounded device-side wait gave up */
 } trevs_status;
 
@@ -82,7 +82,7 @@ typedef struct trevs_pre_params {
                           Default 0 (no draws). Batched calls only. */
 } trevs_pre_params;
 
-/* Limits of this build (TREVS_ERR_UNSUPPORTED beyond them). */
+/* Limits of the library (TREVS_ERR_UNSUPPORTED beyond them). */
 #define TREVS_MAX_TEXT_TOKENS 256    /* M per request, stage 1 */
 #define TREVS_HEAD_DIM 128           /* d_h, stage 2 */
 #define TREVS_MAX_STAGE2_TOKENS 2048 /* K1 per request entering stage 2 */
